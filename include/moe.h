@@ -1,0 +1,176 @@
+/*
+ * moe.h - C ABI of libmoe.so: one decode step of a Mixture-of-Experts FFN
+ * layer on one GB300 GPU (sm_103a).
+ *
+ * The operation is the decode-lane work of the paper's served MoE models
+ * (Qwen3-Coder-480B FP8 and Qwen3-235B-A22B NVFP4, Section 4 "Setup"); the
+ * paper states that decode is weight-read bound (Section 2.1) and that MoE
+ * sparsity leaves the decode lane under-saturated (Appendix A.3).  The paper
+ * gives no kernel or number format for it; the numeric readings below are
+ * this library's.
+ *
+ *   logits[t,e] = sum_h x[t,h] * Wr[e,h] (+ bias[e])          fp32
+ *   ids[t,:]    = top-k of logits[t,:], by (value desc, index asc)
+ *   w[t,j]      = exp(l_j - l_max) / sum_{i in top-k} exp(l_i - l_max)
+ *   h           = silu(x_t Wg_e^T) * (x_t Wu_e^T),  silu(z) = z / (1 + e^-z)
+ *   y           = h Wd_e^T
+ *   out[t]      = bf16( sum_j w[t,j] * y_{t,ids[t,j]}  (+ residual[t]) )
+ *
+ * Conventions shared by every entry point
+ * - Pointers named x, out, residual point to bf16 data (IEEE binary32 top
+ *   halves); every other pointer has the element type stated.  All data
+ *   pointers are DEVICE pointers unless a comment says otherwise.
+ * - Row-major, innermost index contiguous.  T tokens, H hidden, E experts,
+ *   k experts per token, I expert intermediate size.
+ * - `stream` is a cudaStream_t (NULL = the legacy default stream).  Every
+ *   call only enqueues work on it and returns; nothing synchronises.
+ * - The caller owns every buffer.  The library allocates no device memory.
+ * - Return value: MOE_OK (0) or a negative moe_status_t.  Argument errors
+ *   are detected on the host before anything is enqueued.  Errors detected
+ *   by a running kernel (a bounded wait that expired, an expert id out of
+ *   range) are recorded in a status word inside the workspace and read
+ *   with moe_read_status().  No exception or abort crosses the ABI.
+ *
+ * Expert weight formats (moe_expert_weights_t)
+ *   gate and up are [E, I, H]-shaped (N = I rows, K = H contiguous),
+ *   down is [E, H, I]-shaped (N = H rows, K = I contiguous).
+ * - MOE_FMT_FP8_B128: codes are OCP OFP8 E4M3 bytes [E, N, K]; scales are
+ *   float32 [E, N/128, K/128], one per 128x128 tile; W = e4m3(code)*scale.
+ *   Codes 0x7F/0xFF (NaN) must not occur.
+ * - MOE_FMT_NVFP4: codes are OCP E2M1 nibbles, two per byte [E, N, K/2]
+ *   (low nibble = even K index); scales are E4M3 bytes [E, N, K/16], one per
+ *   16 consecutive K elements; ts_* are float32 [E], one per expert matrix;
+ *   W = e2m1(code) * e4m3(scale) * ts.
+ *
+ * Supported shapes: H % 256 == 0; I % 128 == 0 (FP8) or I % 256 == 0
+ * (NVFP4); 1 <= k <= E <= 512; 0 <= T; T*k <= 65536; H, I <= 32768.
+ * T == 0 is a no-op.  Anything else returns MOE_ERR_UNSUPPORTED_SHAPE.
+ */
+#ifndef MOE_H_
+#define MOE_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  MOE_OK = 0,
+  MOE_ERR_INVALID_ARG = -1,        /* null pointer, negative size, bad flag */
+  MOE_ERR_UNSUPPORTED_SHAPE = -2,  /* shape outside the supported set above */
+  MOE_ERR_WORKSPACE_TOO_SMALL = -3,
+  MOE_ERR_CUDA = -4,               /* a CUDA runtime call or launch failed */
+  MOE_ERR_DEVICE_TIMEOUT = -5,     /* a kernel's bounded wait expired */
+  MOE_ERR_BAD_EXPERT_ID = -6,      /* moe_permute met an id outside [0, E) */
+  MOE_ERR_UNSUPPORTED_DEVICE = -7  /* not an sm_103 (GB300) device */
+} moe_status_t;
+
+typedef enum { MOE_FMT_FP8_B128 = 1, MOE_FMT_NVFP4 = 2 } moe_format_t;
+
+/* Flags of moe_decode_layer. */
+#define MOE_FLAG_NO_RENORM 0x1   /* gates = full-softmax probabilities at the top-k */
+#define MOE_FLAG_PRENORM_RMS 0x2 /* route and run the experts on bf16(RMSNorm(x)),
+                                    unit weight, eps 1e-6; residual is still added */
+
+/* The expert weights of one layer.  All pointers are device pointers to the
+ * caller's buffers; the struct itself is read on the host during the call. */
+typedef struct {
+  int fmt; /* moe_format_t */
+  int E, H, I;
+  const uint8_t *w_gate, *w_up, *w_down;
+  const void *s_gate, *s_up, *s_down;     /* float32 (FP8) or uint8 E4M3 (NVFP4) */
+  const float *ts_gate, *ts_up, *ts_down; /* NVFP4 only; NULL for FP8 */
+} moe_expert_weights_t;
+
+/* Human-readable name of a status code.  Never NULL; static storage. */
+const char* moe_status_string(int status);
+
+/* ABI version (major*10000 + minor*100 + patch). */
+int moe_version(void);
+
+/* Bytes of device workspace needed by moe_decode_layer / moe_expert_ffn for
+ * these weights and T tokens with k experts each (*bytes, host pointer).
+ * Pure host computation. */
+int moe_workspace_size(const moe_expert_weights_t* w, int T, int k, size_t* bytes);
+
+/* Bytes of device workspace needed by moe_route_topk for T tokens, E experts. */
+int moe_route_workspace_size(int T, int E, size_t* bytes);
+
+/* Zero a workspace (cudaMemsetAsync).  A workspace must be zeroed once
+ * before its first use; the library keeps it consistent afterwards. */
+int moe_workspace_init(void* ws, size_t ws_bytes, void* stream);
+
+/* Copy the device status word of a workspace to *status (host pointer) and
+ * clear it.  Synchronises `stream`.  *status is MOE_OK or the negative code
+ * of the first device-side error since the last read. */
+int moe_read_status(void* ws, size_t ws_bytes, int* status, void* stream);
+
+/* Router GEMV, softmax and top-k (steps a1-a2 of the decode layer).
+ *   x [T, H] bf16; router_w [E, H] float32; router_bias [E] float32 or NULL.
+ *   topk_ids [T, k] int32, topk_w [T, k] float32: outputs, column j is the
+ *     j-th largest logit (ties to the lower expert index).
+ *   logits_out [T, E] float32 or NULL: the fp32 logits the selection used.
+ *   renorm: 1 = gates renormalised over the top-k, 0 = full-softmax values.
+ *   ws: workspace of at least moe_route_workspace_size() bytes. */
+int moe_route_topk(const void* x, const float* router_w, const float* router_bias, int T, int H,
+                   int E, int k, int renorm, int32_t* topk_ids, float* topk_w, float* logits_out,
+                   void* ws, size_t ws_bytes, void* stream);
+
+/* Token-to-expert permutation (step a3).  Assignment a = t*k + j.
+ *   topk_ids [T, k] int32 in [0, E) (out-of-range ids are skipped and
+ *     reported as MOE_ERR_BAD_EXPERT_ID through `ws`-less status: the call
+ *     writes -1 into active[0]).
+ *   counts [E]: assignments per expert; offsets [E+1]: exclusive prefix sum;
+ *   sorted_assign [T*k]: assignments sorted stably by expert;
+ *   inv_perm [T*k]: position of each assignment in sorted_assign;
+ *   active [E+1]: active[0] = number of experts with counts > 0, then their
+ *     ids in increasing order. */
+int moe_permute(const int32_t* topk_ids, int T, int k, int E, int32_t* counts, int32_t* offsets,
+                int32_t* sorted_assign, int32_t* inv_perm, int32_t* active, void* stream);
+
+/* Expert FFN over permuted assignments (steps a4-a5), no gating.
+ *   x [T, H] bf16; w: expert weights; offsets, sorted_assign, active as
+ *   produced by moe_permute for the same T, k, E.
+ *   y_perm [T*k, H] float32 output: row p = expert ids[sorted_assign[p]]
+ *     applied to token sorted_assign[p] / k.
+ *   ws: workspace of at least moe_workspace_size(w, T, k) bytes. */
+int moe_expert_ffn(const void* x, const moe_expert_weights_t* w, const int32_t* offsets,
+                   const int32_t* sorted_assign, const int32_t* active, int T, int k,
+                   float* y_perm, void* ws, size_t ws_bytes, void* stream);
+
+/* Gate-weighted combine (step a6).
+ *   out[t, :] = bf16( sum_j topk_w[t, j] * y_perm[inv_perm[t*k + j], :]
+ *                     (+ residual[t, :]) ),  round to nearest even.
+ *   residual [T, H] bf16 or NULL; out [T, H] bf16 (may alias residual). */
+int moe_combine(const float* y_perm, const float* topk_w, const int32_t* inv_perm, int T, int k,
+                int H, const void* residual, void* out, void* stream);
+
+/* The whole decode layer (steps a1-a6) in three kernels on `stream`.
+ *   x [T, H] bf16; router_w [E, H] float32; router_bias [E] float32 or NULL;
+ *   w: expert weights (w->H must equal the row length of x and router_w);
+ *   flags: MOE_FLAG_*; residual [T, H] bf16 or NULL (may alias out);
+ *   out [T, H] bf16, must not alias x;
+ *   ws: at least moe_workspace_size(w, T, k) bytes, zeroed once before
+ *   first use (moe_workspace_init). */
+int moe_decode_layer(const void* x, const float* router_w, const float* router_bias,
+                     const moe_expert_weights_t* w, int T, int k, int flags, const void* residual,
+                     void* out, void* ws, size_t ws_bytes, void* stream);
+
+/* moe_decode_layer plus optional observation points, for tests and timing.
+ *   logits_out [T, E] float32, topk_ids_out [T, k] int32, topk_w_out [T, k]
+ *   float32: copies of the routing the layer used (each may be NULL).
+ *   events: NULL, or 4 cudaEvent_t handles recorded on `stream` before the
+ *   route kernel, before the gate/up kernel, before the down kernel and
+ *   after it. */
+int moe_decode_layer_ex(const void* x, const float* router_w, const float* router_bias,
+                        const moe_expert_weights_t* w, int T, int k, int flags,
+                        const void* residual, void* out, void* ws, size_t ws_bytes,
+                        float* logits_out, int32_t* topk_ids_out, float* topk_w_out,
+                        void* const* events, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* MOE_H_ */

@@ -1,0 +1,509 @@
+// C ABI of libmoe (declared in include/moe.h): argument validation, workspace
+// layout, TMA tensor-map encoding and kernel launches.  Host code only.
+#include <cudaTypedefs.h>
+
+#include <atomic>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+
+#include "../../include/moe.h"
+#include "ffn_launch.cuh"
+#include "route.cuh"
+
+using namespace moe;
+
+namespace {
+
+constexpr int kAbiVersion = 100;  // 0.1.0
+constexpr int kFlagTestStall = 0x100;  // test hook, see the comment in moe.h
+
+// ------------------------------------------------------------------ device facts
+struct DevInfo {
+  std::atomic<int> ready{0};
+  int sms = 0, ok = 0;
+};
+DevInfo g_dev[64];
+
+int device_check(int* sms) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return MOE_ERR_CUDA;
+  DevInfo& d = g_dev[dev];
+  if (!d.ready.load(std::memory_order_acquire)) {
+    int major = 0, minor = 0, n = 0;
+    if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return MOE_ERR_CUDA;
+    d.sms = n;
+    d.ok = (major == 10 && minor == 3);
+    d.ready.store(1, std::memory_order_release);
+  }
+  if (!d.ok) return MOE_ERR_UNSUPPORTED_DEVICE;
+  *sms = d.sms;
+  return MOE_OK;
+}
+
+uint64_t wait_limit_ns() {
+  static std::atomic<uint64_t> cached{0};
+  uint64_t v = cached.load();
+  if (v == 0) {
+    v = kWaitLimitNs;
+    if (const char* s = std::getenv("MOE_WAIT_LIMIT_MS")) {
+      const long ms = std::strtol(s, nullptr, 10);
+      if (ms > 0 && ms <= 60000) v = (uint64_t)ms * 1000000ull;
+    }
+    cached.store(v);
+  }
+  return v;
+}
+
+// ------------------------------------------------------------------ tensor maps
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+  });
+  return fn;
+}
+
+bool map_2d(CUtensorMap* m, CUtensorMapDataType dt, const void* base, uint64_t cols,
+            uint64_t rows, uint64_t row_bytes, uint32_t box_cols, uint32_t box_rows,
+            CUtensorMapSwizzle sw) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {row_bytes};
+  cuuint32_t box[2] = {box_cols, box_rows};
+  cuuint32_t es[2] = {1, 1};
+  return fn(m, dt, 2, const_cast<void*>(base), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// codes of one expert-stacked matrix [E*N, Kbytes], 128 x 128-byte boxes, 128B swizzle
+bool map_codes(CUtensorMap* m, const uint8_t* codes, int E, int N, int Kbytes) {
+  return map_2d(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, codes, (uint64_t)Kbytes, (uint64_t)E * N,
+                (uint64_t)Kbytes, kRowBytes, kRowsHalf, CU_TENSOR_MAP_SWIZZLE_128B);
+}
+
+// NVFP4 scales [E*N, K/16] bytes, 128 x 16-byte boxes
+bool map_sf(CUtensorMap* m, const void* sf, int E, int N, int K) {
+  return map_2d(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, sf, (uint64_t)(K / 16), (uint64_t)E * N,
+                (uint64_t)(K / 16), 16, kRowsHalf, CU_TENSOR_MAP_SWIZZLE_NONE);
+}
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+int nt_for(int T) { return T <= 8 ? 8 : (T <= 16 ? 16 : 32); }
+
+// ------------------------------------------------------------------ validation
+int check_weights(const moe_expert_weights_t* w) {
+  if (!w) return MOE_ERR_INVALID_ARG;
+  if (w->fmt != MOE_FMT_FP8_B128 && w->fmt != MOE_FMT_NVFP4) return MOE_ERR_INVALID_ARG;
+  if (!w->w_gate || !w->w_up || !w->w_down || !w->s_gate || !w->s_up || !w->s_down)
+    return MOE_ERR_INVALID_ARG;
+  if (w->fmt == MOE_FMT_NVFP4 && (!w->ts_gate || !w->ts_up || !w->ts_down))
+    return MOE_ERR_INVALID_ARG;
+  if (w->E < 1 || w->E > kMaxE) return MOE_ERR_UNSUPPORTED_SHAPE;
+  if (w->H < 256 || w->H > 8192 || w->H % 256) return MOE_ERR_UNSUPPORTED_SHAPE;
+  const int imod = (w->fmt == MOE_FMT_FP8_B128) ? 128 : 256;
+  if (w->I < imod || w->I > 16384 || w->I % imod) return MOE_ERR_UNSUPPORTED_SHAPE;
+  if (!aligned(w->w_gate, 16) || !aligned(w->w_up, 16) || !aligned(w->w_down, 16))
+    return MOE_ERR_INVALID_ARG;
+  const size_t sa = (w->fmt == MOE_FMT_NVFP4) ? 16 : 4;
+  if (!aligned(w->s_gate, sa) || !aligned(w->s_up, sa) || !aligned(w->s_down, sa))
+    return MOE_ERR_INVALID_ARG;
+  return MOE_OK;
+}
+
+int check_tk(int T, int k, int E) {
+  if (T < 0 || k < 1) return MOE_ERR_INVALID_ARG;
+  if (k > E || k > kMaxK) return MOE_ERR_UNSUPPORTED_SHAPE;
+  if ((long long)T * k > kMaxTK) return MOE_ERR_UNSUPPORTED_SHAPE;
+  return MOE_OK;
+}
+
+// ------------------------------------------------------------------ the expert steps
+struct ExpertRun {
+  const moe_expert_weights_t* w;
+  int T, k, nt, sms;
+  void* ws;
+  WsLayout L;
+  const int *offsets, *sorted, *active;  // plan inputs (ws or caller)
+  const int* counts;
+  const float* gates;
+  int fused;
+  float* y_perm;
+  __nv_bfloat16* out;
+  const __nv_bfloat16* residual;
+  int test_stall;
+};
+
+int run_experts(const ExpertRun& r, cudaStream_t st, cudaEvent_t ev_mid) {
+  const moe_expert_weights_t* w = r.w;
+  const int E = w->E, H = w->H, I = w->I;
+  const bool fp4 = (w->fmt == MOE_FMT_NVFP4);
+  const int KEL = fp4 ? 256 : 128;
+  const int hb = fp4 ? H / 2 : H, ib = fp4 ? I / 2 : I;  // bytes per row
+  FfnMaps m1{}, m2{};
+  bool ok = map_codes(&m1.a0, w->w_gate, E, I, hb) && map_codes(&m1.a1, w->w_up, E, I, hb) &&
+            map_codes(&m2.a0, w->w_down, E, H, ib);
+  m2.a1 = m2.a0;
+  if (fp4) {
+    ok = ok && map_sf(&m1.s0, w->s_gate, E, I, H) && map_sf(&m1.s1, w->s_up, E, I, H) &&
+         map_sf(&m2.s0, w->s_down, E, H, I);
+    m2.s1 = m2.s0;
+  } else {
+    m1.s0 = m1.s1 = m1.a0;
+    m2.s0 = m2.s1 = m2.a0;
+  }
+  __half* x16 = ws_ptr<__half>(r.ws, r.L.x16);
+  __half* h16 = ws_ptr<__half>(r.ws, r.L.h16);
+  ok = ok && map_2d(&m1.b, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, x16, (uint64_t)H, (uint64_t)r.T,
+                    (uint64_t)H * 2, KEL, 1, CU_TENSOR_MAP_SWIZZLE_NONE);
+  ok = ok && map_2d(&m2.b, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, h16, (uint64_t)I,
+                    (uint64_t)r.T * r.k, (uint64_t)I * 2, KEL, 8, CU_TENSOR_MAP_SWIZZLE_NONE);
+  if (!ok) return MOE_ERR_CUDA;
+
+  FfnParams p{};
+  p.T = r.T;
+  p.k = r.k;
+  p.E = E;
+  p.H = H;
+  p.I = I;
+  p.counts = r.counts;
+  p.offsets = r.offsets;
+  p.sorted = r.sorted;
+  p.active = r.active;
+  p.cprefix = ws_ptr<int>(r.ws, r.L.cprefix);
+  p.gates = r.gates;
+  p.status = ws_ptr<uint32_t>(r.ws, r.L.status);
+  p.wait_ns = wait_limit_ns();
+
+  FfnParams p1 = p;
+  p1.phase = 1;
+  p1.s0 = static_cast<const float*>(w->s_gate);
+  p1.s1 = static_cast<const float*>(w->s_up);
+  p1.ts0 = w->ts_gate;
+  p1.ts1 = w->ts_up;
+  p1.xinv = ws_ptr<float>(r.ws, r.L.xinv);
+  p1.gu = ws_ptr<float>(r.ws, r.L.gu);
+  p1.h16 = h16;
+  p1.hinv = ws_ptr<float>(r.ws, r.L.hinv);
+  p1.cnt = ws_ptr<unsigned>(r.ws, r.L.gu_cnt);
+  p1.test_stall = r.test_stall;
+
+  FfnParams p2 = p;
+  p2.phase = 2;
+  p2.fused = r.fused;
+  p2.s0 = static_cast<const float*>(w->s_down);
+  p2.s1 = p2.s0;
+  p2.ts0 = w->ts_down;
+  p2.ts1 = w->ts_down;
+  p2.xinv = ws_ptr<float>(r.ws, r.L.hinv);
+  p2.oacc = ws_ptr<float>(r.ws, r.L.oacc);
+  p2.y_perm = r.y_perm;
+  p2.out = r.out;
+  p2.residual = r.residual;
+  p2.cnt = ws_ptr<unsigned>(r.ws, r.L.dn_cnt);
+
+  cudaError_t err = fp4 ? launch_ffn<2>(r.nt, r.sms, m1, p1, st, false)
+                        : launch_ffn<1>(r.nt, r.sms, m1, p1, st, false);
+  if (err != cudaSuccess) return MOE_ERR_CUDA;
+  if (ev_mid && cudaEventRecord(ev_mid, st) != cudaSuccess) return MOE_ERR_CUDA;
+  err = fp4 ? launch_ffn<2>(r.nt, r.sms, m2, p2, st, false)
+            : launch_ffn<1>(r.nt, r.sms, m2, p2, st, false);
+  return err == cudaSuccess ? MOE_OK : MOE_ERR_CUDA;
+}
+
+}  // namespace
+
+// ====================================================================== ABI
+extern "C" {
+
+const char* moe_status_string(int s) {
+  switch (s) {
+    case MOE_OK: return "MOE_OK";
+    case MOE_ERR_INVALID_ARG: return "MOE_ERR_INVALID_ARG";
+    case MOE_ERR_UNSUPPORTED_SHAPE: return "MOE_ERR_UNSUPPORTED_SHAPE";
+    case MOE_ERR_WORKSPACE_TOO_SMALL: return "MOE_ERR_WORKSPACE_TOO_SMALL";
+    case MOE_ERR_CUDA: return "MOE_ERR_CUDA";
+    case MOE_ERR_DEVICE_TIMEOUT: return "MOE_ERR_DEVICE_TIMEOUT";
+    case MOE_ERR_BAD_EXPERT_ID: return "MOE_ERR_BAD_EXPERT_ID";
+    case MOE_ERR_UNSUPPORTED_DEVICE: return "MOE_ERR_UNSUPPORTED_DEVICE";
+    default: return "MOE_ERR_UNKNOWN";
+  }
+}
+
+int moe_version(void) { return kAbiVersion; }
+
+int moe_workspace_size(const moe_expert_weights_t* w, int T, int k, size_t* bytes) {
+  if (!bytes) return MOE_ERR_INVALID_ARG;
+  int rc = check_weights(w);
+  if (rc) return rc;
+  rc = check_tk(T, k, w->E);
+  if (rc) return rc;
+  *bytes = ws_layout(T, k, w->E, w->H, w->I).total;
+  return MOE_OK;
+}
+
+int moe_route_workspace_size(int T, int E, size_t* bytes) {
+  if (!bytes || T < 0) return MOE_ERR_INVALID_ARG;
+  if (E < 1 || E > kMaxE) return MOE_ERR_UNSUPPORTED_SHAPE;
+  *bytes = ws_layout(T, 1, E, 256, 0).logits + align_up(4 * (size_t)T * E, 256);
+  return MOE_OK;
+}
+
+int moe_workspace_init(void* ws, size_t ws_bytes, void* stream) {
+  if (!ws) return MOE_ERR_INVALID_ARG;
+  return cudaMemsetAsync(ws, 0, ws_bytes, (cudaStream_t)stream) == cudaSuccess ? MOE_OK
+                                                                               : MOE_ERR_CUDA;
+}
+
+int moe_read_status(void* ws, size_t ws_bytes, int* status, void* stream) {
+  if (!ws || !status || ws_bytes < 4) return MOE_ERR_INVALID_ARG;
+  uint32_t word = 0;
+  cudaStream_t st = (cudaStream_t)stream;
+  if (cudaMemcpyAsync(&word, ws, 4, cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+      cudaStreamSynchronize(st) != cudaSuccess)
+    return MOE_ERR_CUDA;
+  if (word) {
+    if (cudaMemsetAsync(ws, 0, 4, st) != cudaSuccess || cudaStreamSynchronize(st) != cudaSuccess)
+      return MOE_ERR_CUDA;
+  }
+  if (word & (kStatusTimeoutGateUp | kStatusTimeoutDown))
+    *status = MOE_ERR_DEVICE_TIMEOUT;
+  else if (word & kStatusBadExpertId)
+    *status = MOE_ERR_BAD_EXPERT_ID;
+  else
+    *status = MOE_OK;
+  return MOE_OK;
+}
+
+int moe_route_topk(const void* x, const float* router_w, const float* router_bias, int T, int H,
+                   int E, int k, int renorm, int32_t* topk_ids, float* topk_w, float* logits_out,
+                   void* ws, size_t ws_bytes, void* stream) {
+  if (!x || !router_w || !topk_ids || !topk_w || !ws) return MOE_ERR_INVALID_ARG;
+  if (E < 1 || E > kMaxE) return MOE_ERR_UNSUPPORTED_SHAPE;
+  int rc = check_tk(T, k, E);
+  if (rc) return rc;
+  if (H < 256 || H > 8192 || H % 256) return MOE_ERR_UNSUPPORTED_SHAPE;
+  if (!aligned(x, 16) || !aligned(router_w, 16) || !aligned(ws, 256)) return MOE_ERR_INVALID_ARG;
+  size_t need = 0;
+  moe_route_workspace_size(T, E, &need);
+  if (ws_bytes < need) return MOE_ERR_WORKSPACE_TOO_SMALL;
+  if (T == 0) return MOE_OK;
+  int sms = 0;
+  rc = device_check(&sms);
+  if (rc) return rc;
+  const WsLayout L = ws_layout(T, 1, E, 256, 0);
+  RouteParams p{};
+  p.x = static_cast<const __nv_bfloat16*>(x);
+  p.wr = router_w;
+  p.bias = router_bias;
+  p.T = T;
+  p.H = H;
+  p.E = E;
+  p.k = k;
+  p.renorm = renorm ? 1 : 0;
+  p.fmt = 1;
+  p.logits = logits_out ? logits_out : ws_ptr<float>(ws, L.logits);
+  p.ids = topk_ids;
+  p.gates = topk_w;
+  p.chunk_cnt = ws_ptr<unsigned>(ws, L.route_chunk);
+  p.done_cnt = ws_ptr<unsigned>(ws, L.route_done);
+  p.status = ws_ptr<uint32_t>(ws, L.status);
+  return launch_route(p, (cudaStream_t)stream) == cudaSuccess ? MOE_OK : MOE_ERR_CUDA;
+}
+
+int moe_permute(const int32_t* topk_ids, int T, int k, int E, int32_t* counts, int32_t* offsets,
+                int32_t* sorted_assign, int32_t* inv_perm, int32_t* active, void* stream) {
+  if (!topk_ids || !counts || !offsets || !sorted_assign || !inv_perm || !active)
+    return MOE_ERR_INVALID_ARG;
+  if (E < 1 || E > kMaxE) return MOE_ERR_UNSUPPORTED_SHAPE;
+  int rc = check_tk(T, k, E);
+  if (rc) return rc;
+  int sms = 0;
+  rc = device_check(&sms);
+  if (rc) return rc;
+  return launch_permute_standalone(topk_ids, T, k, E, counts, offsets, sorted_assign, inv_perm,
+                                   active, (cudaStream_t)stream) == cudaSuccess
+             ? MOE_OK
+             : MOE_ERR_CUDA;
+}
+
+int moe_expert_ffn(const void* x, const moe_expert_weights_t* w, const int32_t* offsets,
+                   const int32_t* sorted_assign, const int32_t* active, int T, int k,
+                   float* y_perm, void* ws, size_t ws_bytes, void* stream) {
+  if (!x || !offsets || !sorted_assign || !active || !y_perm || !ws) return MOE_ERR_INVALID_ARG;
+  int rc = check_weights(w);
+  if (rc) return rc;
+  rc = check_tk(T, k, w->E);
+  if (rc) return rc;
+  if (!aligned(x, 16) || !aligned(y_perm, 16) || !aligned(ws, 256)) return MOE_ERR_INVALID_ARG;
+  const WsLayout L = ws_layout(T, k, w->E, w->H, w->I);
+  if (ws_bytes < L.total) return MOE_ERR_WORKSPACE_TOO_SMALL;
+  if (T == 0) return MOE_OK;
+  int sms = 0;
+  rc = device_check(&sms);
+  if (rc) return rc;
+  cudaStream_t st = (cudaStream_t)stream;
+  const int nt = nt_for(T);
+  PrepParams pp{};
+  pp.x = static_cast<const __nv_bfloat16*>(x);
+  pp.T = T;
+  pp.H = w->H;
+  pp.E = w->E;
+  pp.k = k;
+  pp.fmt = w->fmt;
+  pp.nt = nt;
+  pp.x16 = ws_ptr<__half>(ws, L.x16);
+  pp.xinv = ws_ptr<float>(ws, L.xinv);
+  pp.offsets = offsets;
+  pp.active = active;
+  pp.counts = ws_ptr<int>(ws, L.counts);
+  pp.cprefix = ws_ptr<int>(ws, L.cprefix);
+  pp.zero_a = reinterpret_cast<float4*>(y_perm);
+  pp.zero_a_n4 = (size_t)T * k * w->H / 4;
+  pp.zero_b = ws_ptr<float4>(ws, L.gu);
+  pp.zero_b_n4 = (size_t)T * k * 2 * w->I / 4;
+  pp.zero_c = ws_ptr<unsigned>(ws, L.gu_cnt);
+  pp.zero_c_n = w->E;
+  if (launch_prep(pp, st) != cudaSuccess) return MOE_ERR_CUDA;
+  ExpertRun r{};
+  r.w = w;
+  r.T = T;
+  r.k = k;
+  r.nt = nt;
+  r.sms = sms;
+  r.ws = ws;
+  r.L = L;
+  r.offsets = offsets;
+  r.sorted = sorted_assign;
+  r.active = active;
+  r.counts = ws_ptr<int>(ws, L.counts);
+  r.fused = 0;
+  r.y_perm = y_perm;
+  return run_experts(r, st, nullptr);
+}
+
+int moe_combine(const float* y_perm, const float* topk_w, const int32_t* inv_perm, int T, int k,
+                int H, const void* residual, void* out, void* stream) {
+  if (!y_perm || !topk_w || !inv_perm || !out) return MOE_ERR_INVALID_ARG;
+  if (T < 0 || k < 1 || H < 4 || H % 4) return MOE_ERR_INVALID_ARG;
+  if (!aligned(y_perm, 16) || !aligned(out, 8) || (residual && !aligned(residual, 8)))
+    return MOE_ERR_INVALID_ARG;
+  if (T == 0) return MOE_OK;
+  CombineParams p{y_perm, topk_w, inv_perm, T, k, H,
+                  static_cast<const __nv_bfloat16*>(residual), static_cast<__nv_bfloat16*>(out)};
+  return launch_combine(p, (cudaStream_t)stream) == cudaSuccess ? MOE_OK : MOE_ERR_CUDA;
+}
+
+int moe_decode_layer_ex(const void* x, const float* router_w, const float* router_bias,
+                        const moe_expert_weights_t* w, int T, int k, int flags,
+                        const void* residual, void* out, void* ws, size_t ws_bytes,
+                        float* logits_out, int32_t* topk_ids_out, float* topk_w_out,
+                        void* const* events, void* stream) {
+  if (!x || !router_w || !out || !ws) return MOE_ERR_INVALID_ARG;
+  if (flags & ~(MOE_FLAG_NO_RENORM | MOE_FLAG_PRENORM_RMS | kFlagTestStall))
+    return MOE_ERR_INVALID_ARG;
+  int rc = check_weights(w);
+  if (rc) return rc;
+  rc = check_tk(T, k, w->E);
+  if (rc) return rc;
+  if (!aligned(x, 16) || !aligned(router_w, 16) || !aligned(ws, 256) || !aligned(out, 2) ||
+      (residual && !aligned(residual, 2)))
+    return MOE_ERR_INVALID_ARG;
+  if (out == x) return MOE_ERR_INVALID_ARG;
+  const int E = w->E, H = w->H, I = w->I;
+  const WsLayout L = ws_layout(T, k, E, H, I);
+  if (ws_bytes < L.total) return MOE_ERR_WORKSPACE_TOO_SMALL;
+  if (T == 0) return MOE_OK;
+  int sms = 0;
+  rc = device_check(&sms);
+  if (rc) return rc;
+  cudaStream_t st = (cudaStream_t)stream;
+  cudaEvent_t ev[4] = {nullptr, nullptr, nullptr, nullptr};
+  if (events)
+    for (int i = 0; i < 4; ++i) ev[i] = static_cast<cudaEvent_t>(events[i]);
+  const int nt = nt_for(T);
+
+  RouteParams p{};
+  p.x = static_cast<const __nv_bfloat16*>(x);
+  p.wr = router_w;
+  p.bias = router_bias;
+  p.T = T;
+  p.H = H;
+  p.E = E;
+  p.k = k;
+  p.renorm = (flags & MOE_FLAG_NO_RENORM) ? 0 : 1;
+  p.prenorm = (flags & MOE_FLAG_PRENORM_RMS) ? 1 : 0;
+  p.fmt = w->fmt;
+  p.fused = 1;
+  p.nt = nt;
+  p.logits = logits_out ? logits_out : ws_ptr<float>(ws, L.logits);
+  p.ids = ws_ptr<int>(ws, L.ids);
+  p.gates = ws_ptr<float>(ws, L.gates);
+  p.ids2 = topk_ids_out;
+  p.gates2 = topk_w_out;
+  p.chunk_cnt = ws_ptr<unsigned>(ws, L.route_chunk);
+  p.done_cnt = ws_ptr<unsigned>(ws, L.route_done);
+  p.x16 = ws_ptr<__half>(ws, L.x16);
+  p.xinv = ws_ptr<float>(ws, L.xinv);
+  p.zero_a = ws_ptr<float4>(ws, L.gu);
+  p.zero_a_n4 = (size_t)T * k * 2 * I / 4;
+  p.zero_b = ws_ptr<float4>(ws, L.oacc);
+  p.zero_b_n4 = (size_t)T * H / 4;
+  p.zero_c = ws_ptr<unsigned>(ws, L.gu_cnt);
+  p.zero_c_n = E;
+  p.zero_d = ws_ptr<unsigned>(ws, L.dn_cnt);
+  p.zero_d_n = H / 256;
+  p.counts = ws_ptr<int>(ws, L.counts);
+  p.offsets = ws_ptr<int>(ws, L.offsets);
+  p.sorted = ws_ptr<int>(ws, L.sorted);
+  p.inv = ws_ptr<int>(ws, L.inv);
+  p.active = ws_ptr<int>(ws, L.active);
+  p.cprefix = ws_ptr<int>(ws, L.cprefix);
+  p.status = ws_ptr<uint32_t>(ws, L.status);
+  if (ev[0] && cudaEventRecord(ev[0], st) != cudaSuccess) return MOE_ERR_CUDA;
+  if (launch_route(p, st) != cudaSuccess) return MOE_ERR_CUDA;
+  if (ev[1] && cudaEventRecord(ev[1], st) != cudaSuccess) return MOE_ERR_CUDA;
+
+  ExpertRun r{};
+  r.w = w;
+  r.T = T;
+  r.k = k;
+  r.nt = nt;
+  r.sms = sms;
+  r.ws = ws;
+  r.L = L;
+  r.offsets = p.offsets;
+  r.sorted = p.sorted;
+  r.active = p.active;
+  r.counts = p.counts;
+  r.gates = p.gates;
+  r.fused = 1;
+  r.out = static_cast<__nv_bfloat16*>(out);
+  r.residual = static_cast<const __nv_bfloat16*>(residual);
+  r.test_stall = (flags & kFlagTestStall) ? 1 : 0;
+  rc = run_experts(r, st, ev[2]);
+  if (rc) return rc;
+  if (ev[3] && cudaEventRecord(ev[3], st) != cudaSuccess) return MOE_ERR_CUDA;
+  return MOE_OK;
+}
+
+int moe_decode_layer(const void* x, const float* router_w, const float* router_bias,
+                     const moe_expert_weights_t* w, int T, int k, int flags, const void* residual,
+                     void* out, void* ws, size_t ws_bytes, void* stream) {
+  return moe_decode_layer_ex(x, router_w, router_bias, w, T, k, flags, residual, out, ws,
+                             ws_bytes, nullptr, nullptr, nullptr, nullptr, stream);
+}
+
+}  // extern "C"

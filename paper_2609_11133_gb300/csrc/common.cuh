@@ -1,0 +1,266 @@
+// Shared device helpers of libmoe: PTX wrappers for mbarriers, TMA tensor
+// copies, bounded waits, warp MMA and the workspace layout.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cuda_fp4.h>
+#include <cuda_fp8.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace moe {
+
+// ------------------------------------------------------------------ limits
+constexpr int kMaxE = 512;          // experts per layer
+constexpr int kMaxTK = 65536;       // T * k
+constexpr int kMaxHI = 32768;       // H and I
+constexpr int kRouteTok = 8;        // tokens per router CTA
+constexpr int kRouteWarps = 8;      // warps per router CTA (one expert row each)
+
+// Device status bits (the first error wins; see moe_read_status).
+constexpr uint32_t kStatusTimeoutGateUp = 1u;
+constexpr uint32_t kStatusTimeoutDown = 2u;
+constexpr uint32_t kStatusBadExpertId = 4u;
+
+// Bounded waits give up after this many nanoseconds of %globaltimer.
+constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s
+
+// ------------------------------------------------------------------ workspace
+// Byte offsets of everything the kernels keep between launches.  Built on the
+// host by ws_layout() and passed by value to the kernels.
+struct WsLayout {
+  // control block (zeroed once; every counter is reset by its last user)
+  size_t status;       // u32 device status word
+  size_t route_chunk;  // u32 [nChunks] per-token-chunk arrival tickets
+  size_t route_done;   // u32 chunk-completion ticket
+  size_t gu_cnt;       // u32 [E] per-active-expert stage counters (gate/up)
+  size_t dn_cnt;       // u32 [H/256] per-row-tile stage counters (down)
+  // routing
+  size_t logits;   // f32 [T, E]
+  size_t ids;      // i32 [T, k]
+  size_t gates;    // f32 [T, k]
+  size_t counts;   // i32 [E]
+  size_t offsets;  // i32 [E+1]
+  size_t sorted;   // i32 [T*k]
+  size_t inv;      // i32 [T*k]
+  size_t active;   // i32 [E+1]
+  size_t cprefix;  // i32 [E+1] token-chunk prefix over active experts
+  // activations
+  size_t xinv;     // f32 [T]   power-of-two inverse scale of x16 rows
+  size_t x16;      // f16 [T, H]
+  size_t gu;       // f32 [T*k, 2I] gate | up pre-activations
+  size_t hinv;     // f32 [T*k]
+  size_t h16;      // f16 [T*k, I]
+  size_t oacc;     // f32 [T, H] combine accumulator
+  size_t total;
+  int nChunks;
+};
+
+inline size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+inline WsLayout ws_layout(int T, int k, int E, int H, int I) {
+  WsLayout L{};
+  size_t o = 0;
+  auto take = [&](size_t bytes) {
+    size_t r = o;
+    o = align_up(o + bytes, 256);
+    return r;
+  };
+  L.nChunks = (T + kRouteTok - 1) / kRouteTok;
+  const size_t TK = (size_t)T * k;
+  L.status = take(4);
+  L.route_chunk = take(4 * (size_t)(L.nChunks > 0 ? L.nChunks : 1));
+  L.route_done = take(4);
+  L.gu_cnt = take(4 * (size_t)E);
+  L.dn_cnt = take(4 * (size_t)(H / 256 > 0 ? H / 256 : 1));
+  L.logits = take(4 * (size_t)T * E);
+  L.ids = take(4 * TK);
+  L.gates = take(4 * TK);
+  L.counts = take(4 * (size_t)E);
+  L.offsets = take(4 * (size_t)(E + 1));
+  L.sorted = take(4 * TK);
+  L.inv = take(4 * TK);
+  L.active = take(4 * (size_t)(E + 1));
+  L.cprefix = take(4 * (size_t)(E + 1));
+  L.xinv = take(4 * (size_t)T);
+  L.x16 = take(2 * (size_t)T * H);
+  L.gu = take(4 * TK * 2 * (size_t)I);
+  L.hinv = take(4 * TK);
+  L.h16 = take(2 * TK * (size_t)I);
+  L.oacc = take(4 * (size_t)T * H);
+  L.total = o;
+  return L;
+}
+
+template <typename Ty>
+__host__ __device__ inline Ty* ws_ptr(void* ws, size_t off) {
+  return reinterpret_cast<Ty*>(static_cast<char*>(ws) + off);
+}
+
+// ------------------------------------------------------------------ PTX helpers
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ uint64_t globaltimer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count)
+               : "memory");
+}
+
+__device__ __forceinline__ void fence_mbar_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Wait for phase `parity` of `bar` to complete.  Gives up (returns false) when
+// the deadline passes or when *abort becomes non-zero.
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity,
+                                                  uint64_t limit_ns, volatile int* abort) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  while (true) {
+    for (int i = 0; i < 64; ++i)
+      if (mbar_try_wait(bar, parity)) return true;
+    if (abort != nullptr && *abort) return false;
+    if (globaltimer_ns() - t0 > limit_ns) return false;
+  }
+}
+
+// 2-D tiled TMA load global -> shared, completion counted on `bar` in bytes.
+// `x` is the innermost (contiguous) coordinate in elements, `y` the row.
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar,
+                                            int x, int y, uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      ".L2::cache_hint [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y), "l"(policy)
+      : "memory");
+}
+
+__device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+
+__device__ __forceinline__ uint64_t policy_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
+__device__ __forceinline__ uint64_t policy_evict_last() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
+// 16-byte shared-memory load.
+__device__ __forceinline__ uint4 lds128(uint32_t addr) {
+  uint4 v;
+  asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "r"(addr));
+  return v;
+}
+
+__device__ __forceinline__ uint32_t lds16(uint32_t addr) {
+  unsigned short v;
+  asm volatile("ld.shared.u16 %0, [%1];" : "=h"(v) : "r"(addr));
+  return v;
+}
+
+// D = A * B + C, m16n8k16, f16 inputs, f32 accumulators.
+__device__ __forceinline__ void mma_f16(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2,
+                                        uint32_t a3, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+      "{%8,%9}, {%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// Two E4M3 bytes (low byte -> low half) to two exact f16 values.
+__device__ __forceinline__ uint32_t e4m3x2_to_f16x2(uint32_t two_bytes) {
+  __half2_raw r = __nv_cvt_fp8x2_to_halfraw2(static_cast<__nv_fp8x2_storage_t>(two_bytes),
+                                             __NV_E4M3);
+  return static_cast<uint32_t>(r.x) | (static_cast<uint32_t>(r.y) << 16);
+}
+
+// One byte of two E2M1 codes (low nibble -> low half) to two exact f16 values.
+__device__ __forceinline__ uint32_t e2m1x2_to_f16x2(uint32_t byte) {
+  __half2_raw r = __nv_cvt_fp4x2_to_halfraw2(static_cast<__nv_fp4x2_storage_t>(byte),
+                                             __NV_E2M1);
+  return static_cast<uint32_t>(r.x) | (static_cast<uint32_t>(r.y) << 16);
+}
+
+__device__ __forceinline__ uint32_t hmul2_u32(uint32_t a, uint32_t b) {
+  __half2 r = __hmul2(*reinterpret_cast<__half2*>(&a), *reinterpret_cast<__half2*>(&b));
+  return *reinterpret_cast<uint32_t*>(&r);
+}
+
+__device__ __forceinline__ void red_add_f32(float* p, float v) {
+  asm volatile("red.global.add.f32 [%0], %1;" ::"l"(p), "f"(v) : "memory");
+}
+
+__device__ __forceinline__ float ld_cg_f32(const float* p) { return __ldcg(p); }
+__device__ __forceinline__ int ld_cg_i32(const int* p) { return __ldcg(p); }
+
+// Power-of-two factor that maps max|v| into [2^14, 2^15): f16 holds the
+// scaled value exactly for every bf16 input and leaves headroom for sums.
+__device__ __forceinline__ float pow2_scale_for(float amax) {
+  if (!(amax > 0.f) || !isfinite(amax)) return 1.f;
+  int e;
+  frexpf(amax, &e);  // amax = m * 2^e, 0.5 <= m < 1
+  return ldexpf(1.f, 15 - e);
+}
+
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+__device__ __forceinline__ void set_status(uint32_t* status, uint32_t bit) {
+  if (status) atomicOr(status, bit);
+}
+
+// Programmatic dependent launch controls (no-ops when not launched as such).
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+}  // namespace moe

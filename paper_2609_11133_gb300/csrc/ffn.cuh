@@ -1,0 +1,552 @@
+// Expert FFN kernels of the MoE decode layer (gate/up + SwiGLU, and down +
+// combine), for FP8 E4M3 with 128x128 fp32 block scales and NVFP4.
+//
+// Shape of the work.  Per active expert e with n_e routed tokens, the
+// gate/up step streams 2*I*H weights and the down step H*I weights, each
+// used against only n_e <= a few dozen token columns: the steps are
+// HBM-bound weight streams (the decode-lane regime of the paper's
+// Section 2.1).  The kernels are built around keeping HBM busy:
+//
+// * Work list.  Items are (active expert, token chunk of <= NT tokens,
+//   row tile); each item is a run of K-blocks ("stages").  The stages of
+//   all items are laid end to end and every CTA of a persistent grid takes
+//   an equal contiguous share of them (stream-K), so every SM streams the
+//   same number of bytes whatever the routing.  Partial sums of an item
+//   split between CTAs meet in fp32 accumulators through red.global.add.
+// * Pipeline.  One producer thread issues 2-D TMA tensor copies of each
+//   stage (two 128-row x 128-byte weight boxes with 128B swizzle, the NVFP4
+//   scale boxes, and the stage's token rows) into a ring of shared-memory
+//   stages guarded by mbarriers; eight consumer warps decode and multiply.
+// * Decode.  E4M3 and E2M1*E4M3 values are exact in f16, so weights are
+//   converted exactly in registers (cvt e4m3x2/e2m1x2 -> f16x2; the NVFP4
+//   per-16 scale multiplied in f16, still exact).  Activations are stored
+//   as f16 after a per-row power-of-two scaling (exact for bf16 inputs).
+//   The tensor pipe (mma m16n8k16, fp32 accumulate) does the multiply-adds
+//   with the tokens as the n=8 side; FP8 block scales and NVFP4 tensor
+//   scales are applied to the fp32 accumulators.
+// * Fusion.  The gate/up step writes fp32 pre-activations; the CTA that
+//   completes an expert's last stage (a ticket counter) applies SwiGLU and
+//   writes the f16 input of the down step.  The down step multiplies by the
+//   gate weight and adds straight into a [T, H] fp32 accumulator (the
+//   scatter-combine); the CTA that completes a row tile's last stage
+//   converts those columns to bf16 (+ residual).  No wait depends on
+//   another CTA: every cross-CTA handoff is a ticket, never a spin.
+#pragma once
+
+#include "common.cuh"
+
+namespace moe {
+
+constexpr int kFfnConsumerWarps = 8;
+constexpr int kFfnThreads = (kFfnConsumerWarps + 1) * 32;
+constexpr int kRowsHalf = 128;  // rows of each of the two weight boxes of a stage
+constexpr int kRowBytes = 128;  // weight bytes per row per stage
+
+template <int FMT>
+struct FmtTraits;
+template <>
+struct FmtTraits<1> {           // FP8 E4M3, 128x128 block scales
+  static constexpr int KEL = 128;  // K elements per stage
+  static constexpr int NU = 2;     // 16-byte activation units per (thread, half)
+  static constexpr int SBYTES = 0; // scale bytes per row per stage (in smem)
+};
+template <>
+struct FmtTraits<2> {           // NVFP4
+  static constexpr int KEL = 256;
+  static constexpr int NU = 4;
+  static constexpr int SBYTES = 16;
+};
+
+// Physical position of 16-byte unit U of an activation row block of one
+// stage.  NVFP4 rows swap units so that the four threads of an MMA quad hit
+// four different bank groups; FP8 rows are stored in order.
+template <int FMT>
+__host__ __device__ __forceinline__ int act_unit(int U) {
+  if (FMT == 2) return U ^ ((U >> 2) & 2);
+  return U;
+}
+
+// Element index within a row of x16 / h16 where logical column `col` lives.
+template <int FMT>
+__host__ __device__ __forceinline__ int act_pos(int col) {
+  constexpr int KEL = FmtTraits<FMT>::KEL;
+  const int kb = col / KEL, q = col % KEL;
+  return kb * KEL + act_unit<FMT>(q >> 3) * 8 + (q & 7);
+}
+
+template <int FMT, int NT>
+struct StageGeom {
+  static constexpr int KEL = FmtTraits<FMT>::KEL;
+  static constexpr int A0 = 0;
+  static constexpr int A1 = kRowsHalf * kRowBytes;                   // 16 KB
+  static constexpr int S0 = 2 * kRowsHalf * kRowBytes;               // 32 KB
+  static constexpr int S1 = S0 + kRowsHalf * FmtTraits<FMT>::SBYTES;
+  static constexpr int B = S0 + 2 * kRowsHalf * FmtTraits<FMT>::SBYTES;
+  static constexpr int BROW = KEL * 2;                               // bytes per token row
+  static constexpr int RAW = B + NT * BROW;
+  static constexpr int BYTES = (RAW + 1023) / 1024 * 1024;
+  static constexpr int STAGES_RAW = (220 * 1024) / BYTES;
+  static constexpr int STAGES = STAGES_RAW > 8 ? 8 : STAGES_RAW;
+  static constexpr int SMEM = STAGES * BYTES + 1024;  // + alignment slack
+};
+
+struct FfnParams {
+  int T, k, E, H, I, phase;  // phase 1 = gate/up, 2 = down
+  int fused;                 // phase 2: 1 = scatter into oacc + bf16 out, 0 = y_perm
+  // routing plan (device)
+  const int* counts;
+  const int* offsets;
+  const int* sorted;
+  const int* active;
+  const int* cprefix;
+  const float* gates;  // [T*k] by assignment (fused only)
+  // scales
+  const float* s0;     // FP8 block scales of the matrix behind box A0/A1
+  const float* s1;
+  const float* ts0;    // NVFP4 tensor scales [E]
+  const float* ts1;
+  // activations / accumulators
+  const float* xinv;   // phase 1: [T]; phase 2: hinv [T*k]
+  float* gu;           // phase 1 out / phase 2 (unused)
+  __half* h16;         // phase 1 ticket output
+  float* hinv;         // phase 1 ticket output
+  float* oacc;         // phase 2 fused accumulator [T, H]
+  float* y_perm;       // phase 2 unfused output [T*k, H]
+  __nv_bfloat16* out;  // phase 2 fused output
+  const __nv_bfloat16* residual;
+  unsigned* cnt;       // ticket counters (phase 1: [E] by slot, phase 2: [H/256])
+  uint32_t* status;
+  uint64_t wait_ns;
+  int test_stall;      // test hook: producer withholds its first stage
+};
+
+// ------------------------------------------------------------------ item decode
+struct ItemInfo {
+  int slot, e, arow0, nvalid, rt;
+};
+
+__device__ __forceinline__ ItemInfo decode_item(long long it, int rtiles, const int* s_cpre,
+                                                int nA, const FfnParams& p, int NT) {
+  ItemInfo r;
+  const int chunk_g = (int)(it / rtiles);
+  r.rt = (int)(it % rtiles);
+  int lo = 0, hi = nA - 1;  // last slot with cprefix[slot] <= chunk_g
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (s_cpre[mid] <= chunk_g) lo = mid; else hi = mid - 1;
+  }
+  r.slot = lo;
+  const int chunk = chunk_g - s_cpre[lo];
+  r.e = __ldg(p.active + 1 + lo);
+  const int n_e = __ldg(p.counts + r.e);
+  r.arow0 = __ldg(p.offsets + r.e) + chunk * NT;
+  const int rem = n_e - chunk * NT;
+  r.nvalid = rem < NT ? rem : NT;
+  return r;
+}
+
+// ------------------------------------------------------------------ the kernel
+template <int FMT, int NT>
+__global__ void __launch_bounds__(kFfnThreads, 1)
+    ffn_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmA1,
+               const __grid_constant__ CUtensorMap tmS0, const __grid_constant__ CUtensorMap tmS1,
+               const __grid_constant__ CUtensorMap tmB, const FfnParams p) {
+  using G = StageGeom<FMT, NT>;
+  constexpr int KEL = G::KEL;
+  constexpr int NTILE = NT / 8;
+  constexpr int S = G::STAGES;
+
+  extern __shared__ __align__(1024) unsigned char smem_raw[];
+  // stage ring, 1024-byte aligned in the shared window (128B-swizzle atoms)
+  unsigned char* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+
+  __shared__ __align__(8) uint64_t full_bar[S];
+  __shared__ __align__(8) uint64_t empty_bar[S];
+  __shared__ int s_cpre[kMaxE + 1];
+  __shared__ int s_tok[NT];
+  __shared__ volatile int s_abort;
+  __shared__ int s_last;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const bool is_producer = (warp == kFfnConsumerWarps);
+
+  pdl_wait();
+
+  const int nA = __ldg(p.active);
+  for (int i = threadIdx.x; i <= nA; i += blockDim.x) s_cpre[i] = __ldg(p.cprefix + i);
+  if (threadIdx.x == 0) {
+    s_abort = 0;
+    for (int i = 0; i < S; ++i) {
+      mbar_init(&full_bar[i], 1);
+      mbar_init(&empty_bar[i], kFfnConsumerWarps);
+    }
+    fence_mbar_init();
+  }
+  __syncthreads();
+
+  const int N = (p.phase == 1) ? p.I : p.H;       // rows of one expert matrix
+  const int K = (p.phase == 1) ? p.H : p.I;       // contraction length
+  const int rtiles = (p.phase == 1) ? p.I / kRowsHalf : p.H / (2 * kRowsHalf);
+  const int KB = K / KEL;
+  const long long items = (long long)s_cpre[nA] * rtiles;
+  const long long total = items * KB;
+  const long long s_begin = total * blockIdx.x / gridDim.x;
+  const long long s_end = total * (blockIdx.x + 1) / gridDim.x;
+  const uint32_t timeout_bit = (p.phase == 1) ? kStatusTimeoutGateUp : kStatusTimeoutDown;
+
+  if (is_producer) {
+    if (lane == 0 && s_end > s_begin) {
+      tma_prefetch_desc(&tmA0);
+      tma_prefetch_desc(&tmA1);
+      tma_prefetch_desc(&tmB);
+      if (FMT == 2) {
+        tma_prefetch_desc(&tmS0);
+        tma_prefetch_desc(&tmS1);
+      }
+      const uint64_t pol_w = policy_evict_first();
+      const uint64_t pol_a = policy_evict_last();
+      long long cur_item = -1;
+      ItemInfo inf{};
+      long long issued = 0;
+      for (long long s = s_begin; s < s_end; ++s, ++issued) {
+        const long long it = s / KB;
+        const int kb = (int)(s % KB);
+        if (it != cur_item) {
+          cur_item = it;
+          inf = decode_item(it, rtiles, s_cpre, nA, p, NT);
+          if (p.phase == 1)
+            for (int j = 0; j < inf.nvalid; ++j) s_tok[j] = __ldg(p.sorted + inf.arow0 + j) / p.k;
+        }
+        const int slot = (int)(issued % S);
+        const uint32_t round = (uint32_t)(issued / S);
+        if (!mbar_wait_bounded(&empty_bar[slot], (round & 1u) ^ 1u, p.wait_ns, &s_abort)) {
+          set_status(p.status, timeout_bit);
+          s_abort = 1;
+          break;
+        }
+        if (p.test_stall && issued == 0) continue;  // test hook: this stage never arrives
+        unsigned char* st = smem + (size_t)slot * G::BYTES;
+        const int npad = (inf.nvalid + 7) & ~7;
+        uint32_t bytes = 2u * kRowsHalf * kRowBytes + 2u * kRowsHalf * FmtTraits<FMT>::SBYTES;
+        bytes += (p.phase == 1) ? (uint32_t)inf.nvalid * G::BROW : (uint32_t)npad * G::BROW;
+        mbar_arrive_expect_tx(&full_bar[slot], bytes);
+        int rowA0, rowA1;
+        if (p.phase == 1) {
+          rowA0 = inf.e * N + inf.rt * kRowsHalf;
+          rowA1 = rowA0;
+        } else {
+          rowA0 = inf.e * N + inf.rt * 2 * kRowsHalf;
+          rowA1 = rowA0 + kRowsHalf;
+        }
+        tma_load_2d(st + G::A0, &tmA0, &full_bar[slot], kb * kRowBytes, rowA0, pol_w);
+        tma_load_2d(st + G::A1, &tmA1, &full_bar[slot], kb * kRowBytes, rowA1, pol_w);
+        if (FMT == 2) {
+          tma_load_2d(st + G::S0, &tmS0, &full_bar[slot], kb * 16, rowA0, pol_w);
+          tma_load_2d(st + G::S1, &tmS1, &full_bar[slot], kb * 16, rowA1, pol_w);
+        }
+        if (p.phase == 1) {
+          for (int j = 0; j < inf.nvalid; ++j)
+            tma_load_2d(st + G::B + j * G::BROW, &tmB, &full_bar[slot], kb * KEL, s_tok[j], pol_a);
+        } else {
+          for (int r8 = 0; r8 < npad; r8 += 8)
+            tma_load_2d(st + G::B + r8 * G::BROW, &tmB, &full_bar[slot], kb * KEL, inf.arow0 + r8,
+                        pol_a);
+        }
+      }
+      // Let every copy this CTA issued land before the CTA exits.
+      const long long first = issued > S ? issued - S : 0;
+      for (long long j = first; j < issued; ++j) {
+        if (p.test_stall && j == 0) continue;
+        mbar_wait_bounded(&full_bar[j % S], (uint32_t)((j / S) & 1), p.wait_ns, nullptr);
+      }
+    }
+    return;
+  }
+
+  // ---------------------------------------------------------------- consumers
+  const int g = lane >> 2, t = lane & 3;
+  // MMA row m of this warp's 16-row tile lives in shared row 16*warp + rho(m);
+  // the order makes the two row groups of each quarter-warp differ in bit 2,
+  // so the 128B-swizzled reads of a quarter-warp never share a bank.
+  const int rho_g = ((g & 1) << 2) | (g >> 1);
+  const int ra = 16 * warp + rho_g, rb = ra + 8;
+
+  float acc0[NTILE][4], acc1[NTILE][4];
+  long long cur_item = -1;
+  ItemInfo inf{};
+  int done_in_item = 0;
+  // per-item column data
+  float colscale[NTILE][2];
+  int colrow[NTILE][2];   // flush destination row (assignment row or token)
+  float colgate[NTILE][2];
+
+  auto zero_acc = [&]() {
+#pragma unroll
+    for (int n = 0; n < NTILE; ++n)
+#pragma unroll
+      for (int i = 0; i < 4; ++i) acc0[n][i] = acc1[n][i] = 0.f;
+  };
+
+  auto load_item_cols = [&]() {
+#pragma unroll
+    for (int n = 0; n < NTILE; ++n)
+#pragma unroll
+      for (int c = 0; c < 2; ++c) {
+        const int j = n * 8 + 2 * t + c;
+        colscale[n][c] = 0.f;
+        colrow[n][c] = -1;
+        colgate[n][c] = 0.f;
+        if (j < inf.nvalid) {
+          const int arow = inf.arow0 + j;
+          const int a = __ldg(p.sorted + arow);
+          if (p.phase == 1) {
+            colscale[n][c] = __ldg(p.xinv + a / p.k);
+            colrow[n][c] = arow;
+          } else {
+            colscale[n][c] = __ldcg(p.xinv + arow);  // hinv, written by the previous kernel
+            if (p.fused) {
+              colrow[n][c] = a / p.k;
+              colgate[n][c] = __ldg(p.gates + a);
+            } else {
+              colrow[n][c] = arow;
+              colgate[n][c] = 1.f;
+            }
+          }
+        }
+      }
+  };
+
+  // Adds the item's partial sums to the global accumulators, then takes the
+  // item's ticket; the CTA completing an expert (phase 1) or a row tile
+  // (phase 2) finishes it.
+  // `dead`: this warp stopped at an expired wait.  It still walks the item
+  // boundaries and joins both barriers so the consumer warps stay matched,
+  // but adds nothing and takes no ticket.
+  auto flush = [&](bool dead) {
+    float ts0 = 1.f, ts1 = 1.f;
+    if (FMT == 2) {
+      ts0 = __ldg(p.ts0 + inf.e);
+      ts1 = __ldg(p.ts1 + inf.e);
+    }
+#pragma unroll
+    for (int n = 0; n < NTILE; ++n)
+#pragma unroll
+      for (int c = 0; c < 2; ++c) {
+        if (dead || colrow[n][c] < 0) continue;
+        const float sc = colscale[n][c];
+        const int dst = colrow[n][c];
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+          const float v0 = acc0[n][c + 2 * half] * sc * ts0;
+          const float v1 = acc1[n][c + 2 * half] * sc * ts1;
+          const int mrow = 16 * warp + rho_g + 8 * half;  // row within the 128-row box
+          if (p.phase == 1) {
+            const int f = inf.rt * kRowsHalf + mrow;
+            float* base = p.gu + (size_t)dst * 2 * p.I;
+            red_add_f32(base + f, v0);
+            red_add_f32(base + p.I + f, v1);
+          } else {
+            const int hrow = inf.rt * 2 * kRowsHalf + mrow;
+            const float gw = colgate[n][c];
+            float* base = p.fused ? p.oacc + (size_t)dst * p.H : p.y_perm + (size_t)dst * p.H;
+            red_add_f32(base + hrow, gw * v0);
+            red_add_f32(base + hrow + kRowsHalf, gw * v1);
+          }
+        }
+      }
+    if (!(p.phase == 1 || p.fused)) return;
+    __threadfence();
+    asm volatile("bar.sync 1, %0;" ::"n"(kFfnConsumerWarps * 32) : "memory");
+    if (threadIdx.x == 0) {
+      s_last = 0;
+    }
+    if (threadIdx.x == 0 && !dead && !s_abort) {
+      unsigned key, need;
+      if (p.phase == 1) {
+        key = (unsigned)inf.slot;
+        need = (unsigned)((s_cpre[inf.slot + 1] - s_cpre[inf.slot]) * rtiles * KB);
+      } else {
+        key = (unsigned)inf.rt;
+        need = (unsigned)((long long)s_cpre[nA] * KB);
+      }
+      const unsigned old = atomicAdd(p.cnt + key, (unsigned)done_in_item);
+      const int last = (old + (unsigned)done_in_item == need);
+      if (last) {
+        p.cnt[key] = 0;
+        __threadfence();
+      }
+      s_last = last;
+    }
+    asm volatile("bar.sync 1, %0;" ::"n"(kFfnConsumerWarps * 32) : "memory");
+    if (!s_last) return;
+    const int ct = threadIdx.x;  // 0..255
+    if (p.phase == 1) {
+      // SwiGLU of this expert's rows -> f16 rows (power-of-two scaled) for the down step.
+      const int e = inf.e;
+      const int r0 = __ldg(p.offsets + e), r1 = r0 + __ldg(p.counts + e);
+      for (int row = r0 + warp; row < r1; row += kFfnConsumerWarps) {
+        const float* gr = p.gu + (size_t)row * 2 * p.I;
+        float amax = 0.f;
+        for (int f = lane; f < p.I; f += 32) {
+          const float gv = __ldcg(gr + f), uv = __ldcg(gr + p.I + f);
+          const float hv = gv / (1.f + expf(-gv)) * uv;
+          amax = fmaxf(amax, fabsf(hv));
+        }
+        amax = warp_max(amax);
+        const float sc = pow2_scale_for(amax);
+        __half* hr = p.h16 + (size_t)row * p.I;
+        for (int f = lane; f < p.I; f += 32) {
+          const float gv = __ldcg(gr + f), uv = __ldcg(gr + p.I + f);
+          const float hv = gv / (1.f + expf(-gv)) * uv;
+          hr[act_pos<FMT>(f)] = __float2half_rn(hv * sc);
+        }
+        if (lane == 0) p.hinv[row] = 1.f / sc;
+      }
+    } else {
+      const int col = inf.rt * 2 * kRowsHalf + ct;
+      for (int tok = 0; tok < p.T; ++tok) {
+        float v = __ldcg(p.oacc + (size_t)tok * p.H + col);
+        if (p.residual) v += __bfloat162float(p.residual[(size_t)tok * p.H + col]);
+        p.out[(size_t)tok * p.H + col] = __float2bfloat16_rn(v);
+      }
+    }
+  };
+
+  zero_acc();
+  long long consumed = 0;
+  bool dead = false;
+  for (long long s = s_begin; s < s_end; ++s, ++consumed) {
+    const long long it = s / KB;
+    const int kb = (int)(s % KB);
+    if (it != cur_item) {
+      if (cur_item >= 0) {
+        flush(dead);
+        zero_acc();
+      }
+      cur_item = it;
+      inf = decode_item(it, rtiles, s_cpre, nA, p, NT);
+      load_item_cols();
+      done_in_item = 0;
+    }
+    if (dead) continue;
+    // FP8 block scales of this stage (one per 128x128 tile of each box)
+    float bs0 = 1.f, bs1 = 1.f;
+    if (FMT == 1) {
+      const int KB128 = K / 128;
+      if (p.phase == 1) {
+        const size_t tile = ((size_t)inf.e * (N / 128) + inf.rt) * KB128 + kb;
+        bs0 = __ldg(p.s0 + tile);
+        bs1 = __ldg(p.s1 + tile);
+      } else {
+        const size_t tile = ((size_t)inf.e * (N / 128) + 2 * inf.rt) * KB128 + kb;
+        bs0 = __ldg(p.s0 + tile);
+        bs1 = __ldg(p.s0 + tile + KB128);
+      }
+    }
+    const int slot = (int)(consumed % S);
+    const uint32_t round = (uint32_t)(consumed / S);
+    if (!mbar_wait_bounded(&full_bar[slot], round & 1u, p.wait_ns, &s_abort)) {
+      set_status(p.status, timeout_bit);
+      s_abort = 1;
+      dead = true;
+      continue;
+    }
+    const uint32_t st = smem_u32(smem + (size_t)slot * G::BYTES);
+    const int ntiles = (inf.nvalid + 7) >> 3;
+
+    float tmp0[NTILE][4], tmp1[NTILE][4];
+#pragma unroll
+    for (int n = 0; n < NTILE; ++n)
+#pragma unroll
+      for (int i = 0; i < 4; ++i) tmp0[n][i] = tmp1[n][i] = 0.f;
+
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int c = 4 * h + t;  // 16-byte weight chunk of this thread
+      const uint4 qa0 = lds128(st + G::A0 + ra * kRowBytes + ((c ^ (ra & 7)) << 4));
+      const uint4 qb0 = lds128(st + G::A0 + rb * kRowBytes + ((c ^ (rb & 7)) << 4));
+      const uint4 qa1 = lds128(st + G::A1 + ra * kRowBytes + ((c ^ (ra & 7)) << 4));
+      const uint4 qb1 = lds128(st + G::A1 + rb * kRowBytes + ((c ^ (rb & 7)) << 4));
+      uint32_t sa0 = 0, sb0 = 0, sa1 = 0, sb1 = 0;  // NVFP4 scale pairs (f16x2)
+      if (FMT == 2) {
+        sa0 = e4m3x2_to_f16x2(lds16(st + G::S0 + ra * 16 + 2 * c));
+        sb0 = e4m3x2_to_f16x2(lds16(st + G::S0 + rb * 16 + 2 * c));
+        sa1 = e4m3x2_to_f16x2(lds16(st + G::S1 + ra * 16 + 2 * c));
+        sb1 = e4m3x2_to_f16x2(lds16(st + G::S1 + rb * 16 + 2 * c));
+      }
+      const uint32_t wa0[4] = {qa0.x, qa0.y, qa0.z, qa0.w};
+      const uint32_t wb0[4] = {qb0.x, qb0.y, qb0.z, qb0.w};
+      const uint32_t wa1[4] = {qa1.x, qa1.y, qa1.z, qa1.w};
+      const uint32_t wb1[4] = {qb1.x, qb1.y, qb1.z, qb1.w};
+      constexpr int NU = FmtTraits<FMT>::NU;
+#pragma unroll
+      for (int u = 0; u < NU; ++u) {
+        // activation fragments: 8 f16 = K positions P..P+7 of this thread
+        uint4 xb[NTILE];
+#pragma unroll
+        for (int n = 0; n < NTILE; ++n) {
+          if (n < ntiles) {
+            const int row = n * 8 + g;
+            const int U = c * NU + u;
+            xb[n] = lds128(st + G::B + row * G::BROW + (act_unit<FMT>(U) << 4));
+          }
+        }
+#pragma unroll
+        for (int ss = 0; ss < 2; ++ss) {
+          const int s_ = 2 * u + ss;  // k-step within the half
+          uint32_t A0r[4], A1r[4];
+          if (FMT == 1) {
+            const uint32_t xa0 = wa0[s_], xb0_ = wb0[s_], xa1 = wa1[s_], xb1_ = wb1[s_];
+            A0r[0] = e4m3x2_to_f16x2(xa0 & 0xFFFFu);
+            A0r[1] = e4m3x2_to_f16x2(xb0_ & 0xFFFFu);
+            A0r[2] = e4m3x2_to_f16x2(xa0 >> 16);
+            A0r[3] = e4m3x2_to_f16x2(xb0_ >> 16);
+            A1r[0] = e4m3x2_to_f16x2(xa1 & 0xFFFFu);
+            A1r[1] = e4m3x2_to_f16x2(xb1_ & 0xFFFFu);
+            A1r[2] = e4m3x2_to_f16x2(xa1 >> 16);
+            A1r[3] = e4m3x2_to_f16x2(xb1_ >> 16);
+          } else {
+            const int sh = 16 * (s_ & 1);
+            const int wi = s_ >> 1;
+            const uint32_t pa0 = (wa0[wi] >> sh), pb0 = (wb0[wi] >> sh);
+            const uint32_t pa1 = (wa1[wi] >> sh), pb1 = (wb1[wi] >> sh);
+            // scale of this k-step's 16-block: low half for s_ < 4, high half otherwise
+            const uint32_t sel = (s_ < 4) ? 0x1010u : 0x3232u;
+            const uint32_t ca0 = __byte_perm(sa0, 0, sel), cb0 = __byte_perm(sb0, 0, sel);
+            const uint32_t ca1 = __byte_perm(sa1, 0, sel), cb1 = __byte_perm(sb1, 0, sel);
+            A0r[0] = hmul2_u32(e2m1x2_to_f16x2(pa0 & 0xFFu), ca0);
+            A0r[1] = hmul2_u32(e2m1x2_to_f16x2(pb0 & 0xFFu), cb0);
+            A0r[2] = hmul2_u32(e2m1x2_to_f16x2((pa0 >> 8) & 0xFFu), ca0);
+            A0r[3] = hmul2_u32(e2m1x2_to_f16x2((pb0 >> 8) & 0xFFu), cb0);
+            A1r[0] = hmul2_u32(e2m1x2_to_f16x2(pa1 & 0xFFu), ca1);
+            A1r[1] = hmul2_u32(e2m1x2_to_f16x2(pb1 & 0xFFu), cb1);
+            A1r[2] = hmul2_u32(e2m1x2_to_f16x2((pa1 >> 8) & 0xFFu), ca1);
+            A1r[3] = hmul2_u32(e2m1x2_to_f16x2((pb1 >> 8) & 0xFFu), cb1);
+          }
+#pragma unroll
+          for (int n = 0; n < NTILE; ++n) {
+            if (n < ntiles) {
+              const uint32_t b0 = ss ? xb[n].z : xb[n].x;
+              const uint32_t b1 = ss ? xb[n].w : xb[n].y;
+              mma_f16(tmp0[n], A0r[0], A0r[1], A0r[2], A0r[3], b0, b1);
+              mma_f16(tmp1[n], A1r[0], A1r[1], A1r[2], A1r[3], b0, b1);
+            }
+          }
+        }
+      }
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&empty_bar[slot]);
+#pragma unroll
+    for (int n = 0; n < NTILE; ++n)
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        acc0[n][i] = fmaf(bs0, tmp0[n][i], acc0[n][i]);
+        acc1[n][i] = fmaf(bs1, tmp1[n][i], acc1[n][i]);
+      }
+    ++done_in_item;
+  }
+  if (cur_item >= 0) flush(dead);
+}
+
+}  // namespace moe

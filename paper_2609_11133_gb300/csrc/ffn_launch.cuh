@@ -1,0 +1,62 @@
+// Host-side launchers of the expert FFN kernels (one translation unit per
+// weight format keeps compile times short).
+#pragma once
+
+#include "ffn.cuh"
+
+namespace moe {
+
+struct FfnMaps {
+  CUtensorMap a0, a1, s0, s1, b;
+};
+
+// Instantiated in ffn_fp8.cu (FMT = 1) and ffn_nvfp4.cu (FMT = 2).
+template <int FMT>
+cudaError_t launch_ffn(int nt, int grid, const FfnMaps& maps, const FfnParams& p,
+                       cudaStream_t st, bool pdl);
+
+template <int FMT>
+int ffn_smem_bytes(int nt);
+
+#define MOE_DEFINE_FFN_LAUNCH(FMTV)                                                            \
+  template <int NT>                                                                             \
+  static cudaError_t launch_ffn_nt_##FMTV(int grid, const FfnMaps& m, const FfnParams& p,      \
+                                          cudaStream_t st, bool pdl) {                          \
+    auto kern = ffn_kernel<FMTV, NT>;                                                           \
+    const int smem = StageGeom<FMTV, NT>::SMEM;                                                 \
+    cudaError_t err =                                                                           \
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);          \
+    if (err != cudaSuccess) return err;                                                         \
+    cudaLaunchConfig_t cfg = {};                                                                \
+    cfg.gridDim = dim3(grid);                                                                   \
+    cfg.blockDim = dim3(kFfnThreads);                                                           \
+    cfg.dynamicSmemBytes = smem;                                                                \
+    cfg.stream = st;                                                                            \
+    cudaLaunchAttribute attr[1];                                                                \
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;                            \
+    attr[0].val.programmaticStreamSerializationAllowed = 1;                                     \
+    cfg.attrs = attr;                                                                           \
+    cfg.numAttrs = pdl ? 1 : 0;                                                                 \
+    return cudaLaunchKernelEx(&cfg, kern, m.a0, m.a1, m.s0, m.s1, m.b, p);                      \
+  }                                                                                             \
+  template <>                                                                                   \
+  cudaError_t launch_ffn<FMTV>(int nt, int grid, const FfnMaps& m, const FfnParams& p,         \
+                               cudaStream_t st, bool pdl) {                                     \
+    switch (nt) {                                                                               \
+      case 8:                                                                                   \
+        return launch_ffn_nt_##FMTV<8>(grid, m, p, st, pdl);                                    \
+      case 16:                                                                                  \
+        return launch_ffn_nt_##FMTV<16>(grid, m, p, st, pdl);                                   \
+      case 32:                                                                                  \
+        return launch_ffn_nt_##FMTV<32>(grid, m, p, st, pdl);                                   \
+      default:                                                                                  \
+        return cudaErrorInvalidValue;                                                           \
+    }                                                                                           \
+  }                                                                                             \
+  template <>                                                                                   \
+  int ffn_smem_bytes<FMTV>(int nt) {                                                            \
+    return nt == 8 ? StageGeom<FMTV, 8>::SMEM                                                   \
+                   : (nt == 16 ? StageGeom<FMTV, 16>::SMEM : StageGeom<FMTV, 32>::SMEM);        \
+  }
+
+}  // namespace moe

@@ -1,0 +1,468 @@
+// Router GEMV + top-k, permutation / work plan, and the small elementwise
+// kernels (activation conversion, combine) of the MoE decode layer.
+#include "ffn.cuh"
+#include "route.cuh"
+
+namespace moe {
+
+// ------------------------------------------------------------------ helpers
+
+// Scale one token row to f16 (power-of-two factor, exact for bf16 input) in
+// the unit order the expert kernels read (act_pos), and store 1/factor.
+template <int FMT>
+__device__ void convert_row_x16(const __nv_bfloat16* row, int H, __half* dst, float* inv,
+                                int lane) {
+  float amax = 0.f;
+  for (int h = lane * 8; h < H; h += 256) {
+    const uint4 v = *reinterpret_cast<const uint4*>(row + h);
+    const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 f = __bfloat1622float2(b[i]);
+      amax = fmaxf(amax, fmaxf(fabsf(f.x), fabsf(f.y)));
+    }
+  }
+  amax = warp_max(amax);
+  const float sc = pow2_scale_for(amax);
+  constexpr int UPB = FmtTraits<FMT>::KEL / 8;  // 16-byte units per stage block
+  for (int h = lane * 8; h < H; h += 256) {
+    const uint4 v = *reinterpret_cast<const uint4*>(row + h);
+    const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&v);
+    uint4 o;
+    __half2* oh = reinterpret_cast<__half2*>(&o);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 f = __bfloat1622float2(b[i]);
+      oh[i] = __floats2half2_rn(f.x * sc, f.y * sc);
+    }
+    const int U = h >> 3;
+    const int phys = (U / UPB) * UPB + act_unit<FMT>(U % UPB);
+    *reinterpret_cast<uint4*>(dst + (size_t)phys * 8) = o;
+  }
+  if (lane == 0) *inv = 1.f / sc;
+}
+
+__device__ __forceinline__ void convert_row_dispatch(int fmt, const __nv_bfloat16* row, int H,
+                                                     __half* dst, float* inv, int lane) {
+  if (fmt == 2)
+    convert_row_x16<2>(row, H, dst, inv, lane);
+  else
+    convert_row_x16<1>(row, H, dst, inv, lane);
+}
+
+__device__ __forceinline__ unsigned lanemask_lt() {
+  unsigned m;
+  asm("mov.u32 %0, %%lanemask_lt;" : "=r"(m));
+  return m;
+}
+
+// Token -> expert permutation and the expert kernels' work plan, by one CTA of
+// 256 threads.  Assignments are ranked within eight contiguous segments (one
+// warp each, match_any per 32), the per-segment counts are prefix-summed per
+// expert, and every assignment is placed at offsets[e] + its stable rank.
+// cw: shared scratch of 8*E + 2*(E+1) ints.
+__device__ void permute_plan(const int* ids, int T, int k, int E, int nt, int* counts,
+                             int* offsets, int* sorted, int* inv, int* active, int* cprefix,
+                             uint32_t* status, int* cw) {
+  const int A = T * k;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int seg = (A + 7) / 8;
+  int* s_off = cw + 8 * E;
+  int* s_bad = s_off + E + 1;
+  for (int i = threadIdx.x; i < 8 * E; i += blockDim.x) cw[i] = 0;
+  if (threadIdx.x == 0) *s_bad = 0;
+  __syncthreads();
+  {
+    const int a_lo = warp * seg, a_hi = min(A, (warp + 1) * seg);
+    for (int base = a_lo; base < a_hi; base += 32) {
+      const int a = base + lane;
+      int e = -1;
+      if (a < a_hi) {
+        e = __ldcg(ids + a);
+        if (e < 0 || e >= E) {
+          e = -1;
+          *s_bad = 1;
+        }
+      }
+      const int key = (e >= 0) ? e : -(lane + 2);
+      const unsigned peers = __match_any_sync(0xffffffffu, key);
+      int c = 0;
+      if (e >= 0) c = cw[warp * E + e];
+      __syncwarp();
+      if (e >= 0 && lane == __ffs(peers) - 1) cw[warp * E + e] = c + __popc(peers);
+      __syncwarp();
+      if (e >= 0) inv[a] = c + __popc(peers & lanemask_lt());
+    }
+  }
+  __syncthreads();
+  for (int e = threadIdx.x; e < E; e += blockDim.x) {
+    int run = 0;
+    for (int w = 0; w < 8; ++w) {
+      const int c = cw[w * E + e];
+      cw[w * E + e] = run;
+      run += c;
+    }
+    counts[e] = run;
+    s_off[e] = run;  // counts for now
+  }
+  __syncthreads();
+  if (warp == 0) {
+    const int per = (E + 31) / 32;
+    const int e0 = lane * per, e1 = min(E, e0 + per);
+    int sc = 0, sa = 0, sch = 0;
+    for (int e = e0; e < e1; ++e) {
+      const int c = s_off[e];
+      sc += c;
+      sa += (c > 0);
+      sch += (c + nt - 1) / nt;
+    }
+    int xc = sc, xa = sa, xch = sch;  // inclusive scans
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int yc = __shfl_up_sync(0xffffffffu, xc, o);
+      const int ya = __shfl_up_sync(0xffffffffu, xa, o);
+      const int ych = __shfl_up_sync(0xffffffffu, xch, o);
+      if (lane >= o) {
+        xc += yc;
+        xa += ya;
+        xch += ych;
+      }
+    }
+    int rc = xc - sc, ra = xa - sa, rch = xch - sch;  // exclusive
+    for (int e = e0; e < e1; ++e) {
+      const int c = s_off[e];
+      s_off[e] = rc;
+      offsets[e] = rc;
+      if (c > 0) {
+        active[1 + ra] = e;
+        cprefix[ra] = rch;
+        ++ra;
+        rch += (c + nt - 1) / nt;
+      }
+      rc += c;
+    }
+    if (lane == 31) {
+      offsets[E] = xc;
+      s_off[E] = xc;
+      active[0] = *s_bad ? -1 : xa;
+      cprefix[xa] = xch;
+    }
+  }
+  __syncthreads();
+  for (int a = threadIdx.x; a < A; a += blockDim.x) {
+    const int e = __ldcg(ids + a);
+    if (e < 0 || e >= E) continue;
+    const int w = a / seg;
+    const int pos = s_off[e] + cw[w * E + e] + inv[a];
+    sorted[pos] = a;
+    inv[a] = pos;
+  }
+  if (threadIdx.x == 0 && *s_bad) set_status(status, kStatusBadExpertId);
+}
+
+// ------------------------------------------------------------------ route kernel
+__global__ void __launch_bounds__(256) route_kernel(const RouteParams p) {
+  extern __shared__ __align__(16) unsigned char route_smem[];
+  __nv_bfloat16* xs = reinterpret_cast<__nv_bfloat16*>(route_smem);
+  __shared__ int s_flag;
+  __shared__ int s_sel[kRouteWarps][kMaxK];
+  __shared__ float s_selv[kRouteWarps][kMaxK];
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int chunk = blockIdx.y, eb = blockIdx.x;
+  const int t0 = chunk * kRouteTok;
+  const int nt = min(kRouteTok, p.T - t0);
+  const int H = p.H, E = p.E;
+
+  // accumulators and counters of the later kernels start from zero
+  if (p.fused) {
+    const size_t nthr = (size_t)gridDim.x * gridDim.y * blockDim.x;
+    const size_t tid = ((size_t)blockIdx.y * gridDim.x + blockIdx.x) * blockDim.x + threadIdx.x;
+    const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (size_t i = tid; i < p.zero_a_n4; i += nthr) p.zero_a[i] = z;
+    for (size_t i = tid; i < p.zero_b_n4; i += nthr) p.zero_b[i] = z;
+    for (size_t i = tid; i < (size_t)p.zero_c_n; i += nthr) p.zero_c[i] = 0u;
+    for (size_t i = tid; i < (size_t)p.zero_d_n; i += nthr) p.zero_d[i] = 0u;
+  }
+
+  // stage this chunk's token rows
+  {
+    const uint4* src = reinterpret_cast<const uint4*>(p.x + (size_t)t0 * H);
+    uint4* dst = reinterpret_cast<uint4*>(xs);
+    const int n16 = nt * H / 8;
+    for (int i = threadIdx.x; i < n16; i += blockDim.x) dst[i] = __ldg(src + i);
+  }
+  __syncthreads();
+  if (p.prenorm && warp < nt) {
+    // bf16(x / sqrt(mean(x^2) + eps)), unit weight
+    __nv_bfloat16* row = xs + (size_t)warp * H;
+    float ss = 0.f;
+    for (int h = lane; h < H; h += 32) {
+      const float v = __bfloat162float(row[h]);
+      ss = fmaf(v, v, ss);
+    }
+    ss = warp_sum(ss);
+    const float r = 1.f / sqrtf(ss / (float)H + 1e-6f);
+    __syncwarp();
+    for (int h = lane; h < H; h += 32) row[h] = __float2bfloat16_rn(__bfloat162float(row[h]) * r);
+  }
+  __syncthreads();
+  if (p.fused && eb == 0 && warp < nt) {
+    const int t = t0 + warp;
+    convert_row_dispatch(p.fmt, xs + (size_t)warp * H, H, p.x16 + (size_t)t * H, p.xinv + t,
+                         lane);
+  }
+
+  // router GEMV: warp -> expert row, lanes -> 4 consecutive h per 128
+  const int e = eb * kRouteWarps + warp;
+  if (e < E) {
+    float acc[kRouteTok];
+#pragma unroll
+    for (int t = 0; t < kRouteTok; ++t) acc[t] = 0.f;
+    const float* wrow = p.wr + (size_t)e * H;
+    for (int h = lane * 4; h < H; h += 128) {
+      const float4 w = __ldg(reinterpret_cast<const float4*>(wrow + h));
+#pragma unroll
+      for (int t = 0; t < kRouteTok; ++t) {
+        if (t < nt) {
+          const uint2 xv = *reinterpret_cast<const uint2*>(xs + (size_t)t * H + h);
+          const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&xv.x));
+          const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&xv.y));
+          float s = acc[t];
+          s = fmaf(a.x, w.x, s);
+          s = fmaf(a.y, w.y, s);
+          s = fmaf(b.x, w.z, s);
+          s = fmaf(b.y, w.w, s);
+          acc[t] = s;
+        }
+      }
+    }
+#pragma unroll
+    for (int t = 0; t < kRouteTok; ++t) acc[t] = warp_sum(acc[t]);
+    if (lane == 0) {
+      const float b = p.bias ? __ldg(p.bias + e) : 0.f;
+      for (int t = 0; t < nt; ++t) p.logits[(size_t)(t0 + t) * E + e] = acc[t] + b;
+    }
+  }
+
+  // chunk ticket: the last of this chunk's expert blocks does the top-k
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const unsigned old = atomicAdd(p.chunk_cnt + chunk, 1u);
+    s_flag = (old == gridDim.x - 1);
+    if (s_flag) p.chunk_cnt[chunk] = 0u;
+  }
+  __syncthreads();
+  if (!s_flag) return;
+  __threadfence();
+
+  if (warp < nt) {
+    const int t = t0 + warp;
+    constexpr int PER = kMaxE / 32;
+    float v[PER];
+#pragma unroll
+    for (int i = 0; i < PER; ++i) {
+      const int ee = lane + 32 * i;
+      v[i] = (ee < E) ? __ldcg(p.logits + (size_t)t * E + ee) : -INFINITY;
+    }
+    unsigned taken = 0u;
+    for (int j = 0; j < p.k; ++j) {
+      float bv = -INFINITY;
+      int bi = 0x7fffffff;
+#pragma unroll
+      for (int i = 0; i < PER; ++i) {
+        const int ee = lane + 32 * i;
+        if (ee < E && !((taken >> i) & 1u) && (v[i] > bv || (v[i] == bv && ee < bi))) {
+          bv = v[i];
+          bi = ee;
+        }
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
+        const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+        if (ov > bv || (ov == bv && oi < bi)) {
+          bv = ov;
+          bi = oi;
+        }
+      }
+      if ((bi & 31) == lane) taken |= 1u << (bi >> 5);
+      if (lane == 0) {
+        s_sel[warp][j] = bi;
+        s_selv[warp][j] = bv;
+      }
+    }
+    __syncwarp();
+    const float lmax = s_selv[warp][0];
+    float den = 0.f;
+    if (p.renorm) {
+      for (int j = 0; j < p.k; ++j) den += expf(s_selv[warp][j] - lmax);
+    } else {
+      float part = 0.f;
+#pragma unroll
+      for (int i = 0; i < PER; ++i)
+        if (lane + 32 * i < E) part += expf(v[i] - lmax);
+      den = warp_sum(part);
+    }
+    for (int j = lane; j < p.k; j += 32) {
+      const int id = s_sel[warp][j];
+      const float gw = expf(s_selv[warp][j] - lmax) / den;
+      p.ids[(size_t)t * p.k + j] = id;
+      p.gates[(size_t)t * p.k + j] = gw;
+      if (p.ids2) p.ids2[(size_t)t * p.k + j] = id;
+      if (p.gates2) p.gates2[(size_t)t * p.k + j] = gw;
+    }
+  }
+  if (!p.fused) return;
+
+  // chunk-completion ticket: the last chunk builds the permutation and plan
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const unsigned old = atomicAdd(p.done_cnt, 1u);
+    s_flag = (old == gridDim.y - 1);
+    if (s_flag) *p.done_cnt = 0u;
+  }
+  __syncthreads();
+  if (!s_flag) return;
+  __threadfence();
+  permute_plan(p.ids, p.T, p.k, E, p.nt, p.counts, p.offsets, p.sorted, p.inv, p.active,
+               p.cprefix, p.status, reinterpret_cast<int*>(route_smem));
+}
+
+__global__ void __launch_bounds__(256) permute_kernel(const int* ids, int T, int k, int E,
+                                                      int* counts, int* offsets, int* sorted,
+                                                      int* inv, int* active) {
+  extern __shared__ __align__(16) unsigned char route_smem[];
+  int* cw = reinterpret_cast<int*>(route_smem);
+  int* cprefix_scratch = cw + 8 * E + 2 * (E + 1);  // the standalone call has no plan output
+  permute_plan(ids, T, k, E, 32, counts, offsets, sorted, inv, active, cprefix_scratch, nullptr,
+               cw);
+}
+
+// Activation conversion, zeroing and work plan for the unfused expert FFN.
+__global__ void __launch_bounds__(256) prep_kernel(const PrepParams p) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  {
+    const size_t nthr = (size_t)gridDim.x * blockDim.x;
+    const size_t tid = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (size_t i = tid; i < p.zero_a_n4; i += nthr) p.zero_a[i] = z;
+    for (size_t i = tid; i < p.zero_b_n4; i += nthr) p.zero_b[i] = z;
+    for (size_t i = tid; i < (size_t)p.zero_c_n; i += nthr) p.zero_c[i] = 0u;
+  }
+  const int t = blockIdx.x * 8 + warp;
+  if (t < p.T)
+    convert_row_dispatch(p.fmt, p.x + (size_t)t * p.H, p.H, p.x16 + (size_t)t * p.H, p.xinv + t,
+                         lane);
+  if (blockIdx.x == 0) {
+    for (int e = threadIdx.x; e < p.E; e += blockDim.x)
+      p.counts[e] = __ldg(p.offsets + e + 1) - __ldg(p.offsets + e);
+    if (warp == 0) {
+      const int nA = max(0, __ldg(p.active));
+      const int per = (nA + 31) / 32;
+      const int a0 = lane * per, a1 = min(nA, a0 + per);
+      int sch = 0;
+      for (int a = a0; a < a1; ++a) {
+        const int e = __ldg(p.active + 1 + a);
+        const int c = __ldg(p.offsets + e + 1) - __ldg(p.offsets + e);
+        sch += (c + p.nt - 1) / p.nt;
+      }
+      int x = sch;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+      }
+      int r = x - sch;
+      for (int a = a0; a < a1; ++a) {
+        const int e = __ldg(p.active + 1 + a);
+        const int c = __ldg(p.offsets + e + 1) - __ldg(p.offsets + e);
+        p.cprefix[a] = r;
+        r += (c + p.nt - 1) / p.nt;
+      }
+      if (lane == 31) p.cprefix[nA] = x;
+    }
+  }
+}
+
+__global__ void __launch_bounds__(256) combine_kernel(const CombineParams p) {
+  const size_t n4 = (size_t)p.T * p.H / 4;
+  for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4;
+       i += (size_t)gridDim.x * blockDim.x) {
+    const size_t t = i * 4 / p.H;
+    const int h = (int)(i * 4 - t * p.H);
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int j = 0; j < p.k; ++j) {
+      const size_t a = t * p.k + j;
+      const float w = __ldg(p.topk_w + a);
+      const int row = __ldg(p.inv + a);
+      const float4 y = __ldg(reinterpret_cast<const float4*>(p.y_perm + (size_t)row * p.H + h));
+      acc.x = fmaf(w, y.x, acc.x);
+      acc.y = fmaf(w, y.y, acc.y);
+      acc.z = fmaf(w, y.z, acc.z);
+      acc.w = fmaf(w, y.w, acc.w);
+    }
+    if (p.residual) {
+      const uint2 r = *reinterpret_cast<const uint2*>(p.residual + t * p.H + h);
+      const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&r.x));
+      const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&r.y));
+      acc.x += a.x;
+      acc.y += a.y;
+      acc.z += b.x;
+      acc.w += b.y;
+    }
+    __nv_bfloat162 o0 = __floats2bfloat162_rn(acc.x, acc.y);
+    __nv_bfloat162 o1 = __floats2bfloat162_rn(acc.z, acc.w);
+    uint2 o;
+    o.x = *reinterpret_cast<uint32_t*>(&o0);
+    o.y = *reinterpret_cast<uint32_t*>(&o1);
+    *reinterpret_cast<uint2*>(p.out + t * p.H + h) = o;
+  }
+}
+
+// ------------------------------------------------------------------ launchers
+size_t route_smem_bytes(int H, int E) {
+  const size_t xs = (size_t)kRouteTok * H * 2;
+  const size_t perm = sizeof(int) * (size_t)(8 * E + 2 * (E + 1));
+  return xs > perm ? xs : perm;
+}
+
+cudaError_t launch_route(const RouteParams& p, cudaStream_t st) {
+  const size_t smem = route_smem_bytes(p.H, p.E);
+  cudaError_t err =
+      cudaFuncSetAttribute(route_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (err != cudaSuccess) return err;
+  dim3 grid((p.E + kRouteWarps - 1) / kRouteWarps, (p.T + kRouteTok - 1) / kRouteTok);
+  route_kernel<<<grid, 256, smem, st>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_permute_standalone(const int* ids, int T, int k, int E, int* counts,
+                                      int* offsets, int* sorted, int* inv, int* active,
+                                      cudaStream_t st) {
+  const size_t smem = sizeof(int) * (size_t)(8 * E + 3 * (E + 1));
+  cudaError_t err =
+      cudaFuncSetAttribute(permute_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (err != cudaSuccess) return err;
+  permute_kernel<<<1, 256, smem, st>>>(ids, T, k, E, counts, offsets, sorted, inv, active);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_prep(const PrepParams& p, cudaStream_t st) {
+  const int grid = (p.T + 7) / 8 > 0 ? (p.T + 7) / 8 : 1;
+  prep_kernel<<<grid < 64 ? 64 : grid, 256, 0, st>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_combine(const CombineParams& p, cudaStream_t st) {
+  const size_t n4 = (size_t)p.T * p.H / 4;
+  size_t blocks = (n4 + 255) / 256;
+  if (blocks > 4096) blocks = 4096;
+  if (blocks == 0) blocks = 1;
+  combine_kernel<<<(unsigned)blocks, 256, 0, st>>>(p);
+  return cudaGetLastError();
+}
+
+}  // namespace moe

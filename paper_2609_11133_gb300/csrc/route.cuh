@@ -1,0 +1,87 @@
+// Router, top-k, permutation and small elementwise kernels of the MoE decode
+// layer.
+//
+// route_kernel (grid = [ceil(E/8) expert blocks, ceil(T/8) token chunks]):
+//   every CTA stages 8 token rows of x in shared memory and computes the fp32
+//   logits of 8 experts (one warp per expert row of the router, float4 loads,
+//   shuffle reduction).  The CTA that arrives last at a chunk's ticket does
+//   the softmax/top-k of those 8 tokens (one warp per token, k rounds of a
+//   warp arg-max with ties to the lower index); in the fused layer the CTA
+//   that completes the last chunk builds the token->expert permutation and
+//   the work plan of the expert kernels.  Tickets are atomic counters reset
+//   by their last user; nothing waits on another CTA.
+#pragma once
+
+#include "common.cuh"
+
+namespace moe {
+
+constexpr int kMaxK = 32;
+
+struct RouteParams {
+  const __nv_bfloat16* x;
+  const float* wr;
+  const float* bias;
+  int T, H, E, k, renorm, prenorm, fmt, fused, nt;
+  float* logits;  // [T, E]
+  int* ids;       // [T, k]
+  float* gates;   // [T, k]
+  int* ids2;      // optional copies
+  float* gates2;
+  unsigned* chunk_cnt;
+  unsigned* done_cnt;
+  // fused layer only
+  __half* x16;
+  float* xinv;
+  float4* zero_a;
+  size_t zero_a_n4;
+  float4* zero_b;
+  size_t zero_b_n4;
+  unsigned* zero_c;
+  int zero_c_n;
+  unsigned* zero_d;
+  int zero_d_n;
+  int* counts;
+  int* offsets;
+  int* sorted;
+  int* inv;
+  int* active;
+  int* cprefix;
+  uint32_t* status;
+};
+
+struct PrepParams {
+  const __nv_bfloat16* x;
+  int T, H, E, k, fmt, nt;
+  __half* x16;
+  float* xinv;
+  const int* offsets;  // [E+1] from the permutation
+  const int* active;   // [E+1]
+  int* counts;         // [E] (derived here)
+  int* cprefix;        // [E+1]
+  float4* zero_a;
+  size_t zero_a_n4;
+  float4* zero_b;
+  size_t zero_b_n4;
+  unsigned* zero_c;
+  int zero_c_n;
+};
+
+struct CombineParams {
+  const float* y_perm;
+  const float* topk_w;
+  const int* inv;
+  int T, k, H;
+  const __nv_bfloat16* residual;
+  __nv_bfloat16* out;
+};
+
+cudaError_t launch_route(const RouteParams& p, cudaStream_t st);
+cudaError_t launch_permute_standalone(const int* ids, int T, int k, int E, int* counts,
+                                      int* offsets, int* sorted, int* inv, int* active,
+                                      cudaStream_t st);
+cudaError_t launch_prep(const PrepParams& p, cudaStream_t st);
+cudaError_t launch_combine(const CombineParams& p, cudaStream_t st);
+size_t route_smem_bytes(int H, int E);
+
+}  // namespace moe

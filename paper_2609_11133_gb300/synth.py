@@ -125,24 +125,30 @@ class LayerWeights:
 
 
 def make_weights(fmt: int, E: int, H: int, I: int, seed: int = 0, device="cpu",
-                 std: float = 0.02) -> LayerWeights:
-    """Quantised expert weights of one layer, drawn expert by expert."""
+                 std: float = 0.02, experts=None) -> LayerWeights:
+    """Quantised expert weights of one layer, drawn expert by expert.
+
+    ``experts``: optional subset of expert ids to draw (each expert has its own
+    seed, so a subset equals the same rows of the full layer); the others are
+    left zero.
+    """
     dev = torch.device(device)
+    todo = range(E) if experts is None else sorted(set(int(e) for e in experts))
 
     def one(which: int, N: int, K: int):
         if fmt == FMT_FP8:
-            codes = torch.empty((E, N, K), dtype=torch.uint8, device=dev)
-            scales = torch.empty((E, N // 128, K // 128), dtype=torch.float32, device=dev)
-            for e in range(E):
+            codes = torch.zeros((E, N, K), dtype=torch.uint8, device=dev)
+            scales = torch.ones((E, N // 128, K // 128), dtype=torch.float32, device=dev)
+            for e in todo:
                 w = _normal((N, K), std, dev, seed * 1_000_003 + which * 10_007 + e)
                 c, s = quantize_fp8_block(w)
                 codes[e].copy_(c)
                 scales[e].copy_(s)
             return codes, scales, None
-        codes = torch.empty((E, N, K // 2), dtype=torch.uint8, device=dev)
-        sf = torch.empty((E, N, K // 16), dtype=torch.uint8, device=dev)
-        ts = torch.empty((E,), dtype=torch.float32, device=dev)
-        for e in range(E):
+        codes = torch.zeros((E, N, K // 2), dtype=torch.uint8, device=dev)
+        sf = torch.zeros((E, N, K // 16), dtype=torch.uint8, device=dev)
+        ts = torch.ones((E,), dtype=torch.float32, device=dev)
+        for e in todo:
             w = _normal((N, K), std, dev, seed * 1_000_003 + which * 10_007 + e)
             c, s, t = quantize_nvfp4(w)
             codes[e].copy_(c)

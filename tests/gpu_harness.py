@@ -1,0 +1,84 @@
+"""Helpers of the GPU parity tests: build seeded inputs on the device, run the
+CUDA layer through the C ABI, and compute the float64 oracle on the host from
+the very same stored tensors."""
+import numpy as np
+import torch
+
+from oracle import oracle
+from paper_2609_11133_gb300 import binding, synth
+from tests.util_np import np_, oracle_weights
+
+REL_TOL = 2e-2  # max|gpu - ref| <= REL_TOL * max|ref| per layer output
+GATE_TOL = 1e-6
+
+
+class Case:
+    def __init__(self, fmt, T, H, E, k, I, seed=0, bias=None, residual=False, flags=0):
+        dev = "cuda"
+        self.fmt, self.T, self.H, self.E, self.k, self.I, self.flags = fmt, T, H, E, k, I, flags
+        self.w = synth.make_weights(fmt, E, H, I, seed=seed, device=dev)
+        self.x = synth.make_x(T, H, seed=seed, device=dev)
+        self.wr = synth.make_router(E, H, seed=seed, device=dev)
+        self.bias = None if bias is None else bias.to(dev)
+        self.residual = synth.make_x(T, H, seed=seed + 1000, device=dev) if residual else None
+
+    def run(self, out=None):
+        T, H, E, k = self.T, self.H, self.E, self.k
+        n = binding.moe_workspace_size(self.w, T, k)
+        self.ws = binding.alloc_workspace(n)
+        self.out = torch.empty((T, H), dtype=torch.bfloat16, device="cuda") if out is None else out
+        self.logits = torch.empty((T, E), dtype=torch.float32, device="cuda")
+        self.ids = torch.empty((T, k), dtype=torch.int32, device="cuda")
+        self.gates = torch.empty((T, k), dtype=torch.float32, device="cuda")
+        binding.moe_decode_layer_ex(self.x, self.wr, self.bias, self.w, k, self.out, self.ws,
+                                    flags=self.flags, residual=self.residual,
+                                    logits_out=self.logits, topk_ids_out=self.ids,
+                                    topk_w_out=self.gates)
+        torch.cuda.synchronize()
+        assert binding.moe_read_status(self.ws) == 0
+        return self
+
+    # ---- oracle side
+    def x_bits(self):
+        if self.flags & binding.MOE_FLAG_PRENORM_RMS:
+            return oracle.rmsnorm_bf16(np_(self.x), 1e-6)
+        return np_(self.x)
+
+    def check_routing(self):
+        xb = self.x_bits()
+        g_logits = self.logits.double().cpu().numpy()
+        g_ids = self.ids.cpu().numpy()
+        g_gates = self.gates.double().cpu().numpy()
+        renorm = not (self.flags & binding.MOE_FLAG_NO_RENORM)
+        # 1. bit-exact selection given the GPU's fp32 logits
+        o_ids, o_gates = oracle.topk(g_logits, self.k, renorm)
+        assert np.array_equal(o_ids, g_ids), "top-k differs on identical logits"
+        assert np.abs(o_gates - g_gates).max() <= GATE_TOL
+        assert np.abs(g_gates.sum(axis=1) - 1).max() <= GATE_TOL if renorm else True
+        # 2. the fp32 logits are within the fp32 dot-product bound of the float64 ones
+        bias = None if self.bias is None else self.bias.cpu().numpy()
+        ref = oracle.router_logits(xb, np_(self.wr), bias)
+        from tests import indep
+        xa = np.abs(indep.bf16_to_f64(xb))
+        bound = 4 * self.H * 2.0 ** -24 * (xa @ np.abs(np_(self.wr)).astype(np.float64).T) + 1e-6
+        if bias is not None:
+            bound += np.abs(bias) * 2.0 ** -23
+        assert (np.abs(g_logits - ref) <= bound).all()
+        return o_ids, o_gates
+
+    def reference(self, tokens=None):
+        ids, gates = self.check_routing()
+        ow = oracle_weights(self.w)
+        res = None if self.residual is None else np_(self.residual)
+        return oracle.moe_tokens(ow, self.x_bits(), ids, gates, tokens, res)
+
+    def check_output(self, tokens=None, tol=REL_TOL):
+        ref = self.reference(tokens)
+        got = self.out.float().cpu().numpy().astype(np.float64)
+        if tokens is not None:
+            got = got[np.asarray(tokens)]
+        err = np.abs(got - ref).max()
+        scale = np.abs(ref).max()
+        assert np.isfinite(got).all()
+        assert err <= tol * scale, f"max err {err:.3e} vs {tol} * {scale:.3e}"
+        return err / scale

@@ -1,0 +1,104 @@
+"""Host-side checks of the C ABI that need no GPU: the library loads, exports
+every function moe.h declares, and rejects bad arguments before any launch."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2609_11133_gb300 import binding, build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "moe.h")
+
+
+def declared_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?\w+\**\s+\**(moe_\w+)\s*\(", src, flags=re.M)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    return binding.load()
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for required in ("moe_route_topk", "moe_permute", "moe_expert_ffn", "moe_combine",
+                     "moe_decode_layer", "moe_workspace_size", "moe_status_string"):
+        assert required in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+
+
+def test_status_strings(lib):
+    assert binding.status_string(0) == "MOE_OK"
+    assert binding.status_string(-3) == "MOE_ERR_WORKSPACE_TOO_SMALL"
+    assert binding.status_string(12345) == "MOE_ERR_UNKNOWN"
+    assert binding.moe_version() >= 100
+
+
+def fake_weights(fmt=1, E=8, H=512, I=256, **over):
+    c = binding.ExpertWeightsC(fmt, E, H, I, *[ctypes.c_void_p(0x10000 * (i + 1))
+                                                for i in range(9)])
+    for k_, v in over.items():
+        setattr(c, k_, v)
+    return c
+
+
+def ws_size(lib, c, T, k):
+    n = ctypes.c_size_t(0)
+    rc = lib.moe_workspace_size(ctypes.byref(c), T, k, ctypes.byref(n))
+    return rc, n.value
+
+
+def test_workspace_size_and_shape_rules(lib):
+    rc, n = ws_size(lib, fake_weights(), 4, 2)
+    assert rc == 0 and n > 0
+    rc2, n2 = ws_size(lib, fake_weights(), 64, 2)
+    assert rc2 == 0 and n2 > n
+    assert ws_size(lib, fake_weights(H=500), 4, 2)[0] == -2       # H % 256
+    assert ws_size(lib, fake_weights(I=192), 4, 2)[0] == -2       # FP8 I % 128
+    assert ws_size(lib, fake_weights(fmt=2, I=384), 4, 2)[0] == -2  # NVFP4 I % 256
+    assert ws_size(lib, fake_weights(E=600), 4, 2)[0] == -2
+    assert ws_size(lib, fake_weights(), 4, 9)[0] == -2            # k > E
+    assert ws_size(lib, fake_weights(), 4, 0)[0] == -1
+    assert ws_size(lib, fake_weights(), -1, 2)[0] == -1
+    assert ws_size(lib, fake_weights(fmt=3), 4, 2)[0] == -1
+    assert ws_size(lib, fake_weights(w_up=None), 4, 2)[0] == -1
+    assert ws_size(lib, fake_weights(fmt=2, ts_down=None), 4, 2)[0] == -1
+    assert ws_size(lib, fake_weights(w_gate=ctypes.c_void_p(0x10008)), 4, 2)[0] == -1  # align
+
+
+def test_decode_layer_rejects_bad_arguments_before_launch(lib):
+    c = fake_weights()
+    _, n = ws_size(lib, c, 4, 2)
+    P = ctypes.c_void_p
+    x, wr, out, ws = P(0x100000), P(0x200000), P(0x300000), P(0x400000)
+    call = lambda **kw: lib.moe_decode_layer(
+        kw.get("x", x), kw.get("wr", wr), None, ctypes.byref(kw.get("c", c)), kw.get("T", 4),
+        kw.get("k", 2), kw.get("flags", 0), None, kw.get("out", out), kw.get("ws", ws),
+        kw.get("n", n), None)
+    assert call(x=None) == -1
+    assert call(out=None) == -1
+    assert call(out=x) == -1                     # out aliases x
+    assert call(flags=0x40) == -1                # unknown flag
+    assert call(n=n - 1) == -3                   # workspace too small
+    assert call(ws=P(0x400010)) == -1            # workspace alignment
+    assert call(k=3, c=fake_weights(E=2)) == -2
+    assert call(T=0) == 0                        # empty batch is a no-op
+
+
+def test_other_entry_points_validate(lib):
+    P = ctypes.c_void_p
+    assert lib.moe_permute(None, 4, 2, 8, P(1), P(1), P(1), P(1), P(1), None) == -1
+    assert lib.moe_permute(P(16), 4, 9, 8, P(16), P(16), P(16), P(16), P(16), None) == -2
+    assert lib.moe_combine(P(16), P(16), P(16), 4, 2, 6, None, P(16), None) == -1  # H % 4
+    n = ctypes.c_size_t(0)
+    assert lib.moe_route_workspace_size(4, 8, ctypes.byref(n)) == 0 and n.value > 0
+    assert lib.moe_route_topk(P(16), P(16), None, 4, 512, 8, 2, 1, P(16), P(16), None,
+                              P(256), n.value - 1, None) == -3
