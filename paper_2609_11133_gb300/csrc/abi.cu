@@ -290,10 +290,11 @@ int moe_read_status(void* ws, size_t ws_bytes, int* status, void* stream) {
 int moe_route_topk(const void* x, const float* router_w, const float* router_bias, int T, int H,
                    int E, int k, int renorm, int32_t* topk_ids, float* topk_w, float* logits_out,
                    void* ws, size_t ws_bytes, void* stream) {
-  if (!x || !router_w || !topk_ids || !topk_w || !ws) return MOE_ERR_INVALID_ARG;
   if (E < 1 || E > kMaxE) return MOE_ERR_UNSUPPORTED_SHAPE;
   int rc = check_tk(T, k, E);
   if (rc) return rc;
+  if (T == 0) return MOE_OK;
+  if (!x || !router_w || !topk_ids || !topk_w || !ws) return MOE_ERR_INVALID_ARG;
   if (H < 256 || H > 8192 || H % 256) return MOE_ERR_UNSUPPORTED_SHAPE;
   if (!aligned(x, 16) || !aligned(router_w, 16) || !aligned(ws, 256)) return MOE_ERR_INVALID_ARG;
   size_t need = 0;
@@ -325,11 +326,11 @@ int moe_route_topk(const void* x, const float* router_w, const float* router_bia
 
 int moe_permute(const int32_t* topk_ids, int T, int k, int E, int32_t* counts, int32_t* offsets,
                 int32_t* sorted_assign, int32_t* inv_perm, int32_t* active, void* stream) {
-  if (!topk_ids || !counts || !offsets || !sorted_assign || !inv_perm || !active)
-    return MOE_ERR_INVALID_ARG;
+  if (!counts || !offsets || !sorted_assign || !inv_perm || !active) return MOE_ERR_INVALID_ARG;
   if (E < 1 || E > kMaxE) return MOE_ERR_UNSUPPORTED_SHAPE;
   int rc = check_tk(T, k, E);
   if (rc) return rc;
+  if (T > 0 && !topk_ids) return MOE_ERR_INVALID_ARG;
   int sms = 0;
   rc = device_check(&sms);
   if (rc) return rc;
@@ -342,11 +343,12 @@ int moe_permute(const int32_t* topk_ids, int T, int k, int E, int32_t* counts, i
 int moe_expert_ffn(const void* x, const moe_expert_weights_t* w, const int32_t* offsets,
                    const int32_t* sorted_assign, const int32_t* active, int T, int k,
                    float* y_perm, void* ws, size_t ws_bytes, void* stream) {
-  if (!x || !offsets || !sorted_assign || !active || !y_perm || !ws) return MOE_ERR_INVALID_ARG;
   int rc = check_weights(w);
   if (rc) return rc;
   rc = check_tk(T, k, w->E);
   if (rc) return rc;
+  if (T == 0) return MOE_OK;
+  if (!x || !offsets || !sorted_assign || !active || !y_perm || !ws) return MOE_ERR_INVALID_ARG;
   if (!aligned(x, 16) || !aligned(y_perm, 16) || !aligned(ws, 256)) return MOE_ERR_INVALID_ARG;
   const WsLayout L = ws_layout(T, k, w->E, w->H, w->I);
   if (ws_bytes < L.total) return MOE_ERR_WORKSPACE_TOO_SMALL;
@@ -396,8 +398,9 @@ int moe_expert_ffn(const void* x, const moe_expert_weights_t* w, const int32_t* 
 
 int moe_combine(const float* y_perm, const float* topk_w, const int32_t* inv_perm, int T, int k,
                 int H, const void* residual, void* out, void* stream) {
-  if (!y_perm || !topk_w || !inv_perm || !out) return MOE_ERR_INVALID_ARG;
   if (T < 0 || k < 1 || H < 4 || H % 4) return MOE_ERR_INVALID_ARG;
+  if (T == 0) return MOE_OK;
+  if (!y_perm || !topk_w || !inv_perm || !out) return MOE_ERR_INVALID_ARG;
   if (!aligned(y_perm, 16) || !aligned(out, 8) || (residual && !aligned(residual, 8)))
     return MOE_ERR_INVALID_ARG;
   if (T == 0) return MOE_OK;
@@ -411,13 +414,14 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
                         const void* residual, void* out, void* ws, size_t ws_bytes,
                         float* logits_out, int32_t* topk_ids_out, float* topk_w_out,
                         void* const* events, void* stream) {
-  if (!x || !router_w || !out || !ws) return MOE_ERR_INVALID_ARG;
   if (flags & ~(MOE_FLAG_NO_RENORM | MOE_FLAG_PRENORM_RMS | kFlagTestStall))
     return MOE_ERR_INVALID_ARG;
   int rc = check_weights(w);
   if (rc) return rc;
   rc = check_tk(T, k, w->E);
   if (rc) return rc;
+  if (T == 0) return MOE_OK;  // an empty batch may come with null row pointers
+  if (!x || !router_w || !out || !ws) return MOE_ERR_INVALID_ARG;
   if (!aligned(x, 16) || !aligned(router_w, 16) || !aligned(ws, 256) || !aligned(out, 2) ||
       (residual && !aligned(residual, 2)))
     return MOE_ERR_INVALID_ARG;

@@ -467,12 +467,23 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
       const uint4 qb0 = lds128(st + G::A0 + rb * kRowBytes + ((c ^ (rb & 7)) << 4));
       const uint4 qa1 = lds128(st + G::A1 + ra * kRowBytes + ((c ^ (ra & 7)) << 4));
       const uint4 qb1 = lds128(st + G::A1 + rb * kRowBytes + ((c ^ (rb & 7)) << 4));
-      uint32_t sa0 = 0, sb0 = 0, sa1 = 0, sb1 = 0;  // NVFP4 scale pairs (f16x2)
+      // NVFP4: the two 16-element scales of this chunk per row, as f16x2
+      // broadcasts {s, s} of the lower (k-steps 0-3) and upper (4-7) block
+      uint32_t sa0lo = 0, sa0hi = 0, sb0lo = 0, sb0hi = 0;
+      uint32_t sa1lo = 0, sa1hi = 0, sb1lo = 0, sb1hi = 0;
       if (FMT == 2) {
-        sa0 = e4m3x2_to_f16x2(lds16(st + G::S0 + ra * 16 + 2 * c));
-        sb0 = e4m3x2_to_f16x2(lds16(st + G::S0 + rb * 16 + 2 * c));
-        sa1 = e4m3x2_to_f16x2(lds16(st + G::S1 + ra * 16 + 2 * c));
-        sb1 = e4m3x2_to_f16x2(lds16(st + G::S1 + rb * 16 + 2 * c));
+        const uint32_t sa0 = e4m3x2_to_f16x2(lds16(st + G::S0 + ra * 16 + 2 * c));
+        const uint32_t sb0 = e4m3x2_to_f16x2(lds16(st + G::S0 + rb * 16 + 2 * c));
+        const uint32_t sa1 = e4m3x2_to_f16x2(lds16(st + G::S1 + ra * 16 + 2 * c));
+        const uint32_t sb1 = e4m3x2_to_f16x2(lds16(st + G::S1 + rb * 16 + 2 * c));
+        sa0lo = __byte_perm(sa0, 0, 0x1010);
+        sa0hi = __byte_perm(sa0, 0, 0x3232);
+        sb0lo = __byte_perm(sb0, 0, 0x1010);
+        sb0hi = __byte_perm(sb0, 0, 0x3232);
+        sa1lo = __byte_perm(sa1, 0, 0x1010);
+        sa1hi = __byte_perm(sa1, 0, 0x3232);
+        sb1lo = __byte_perm(sb1, 0, 0x1010);
+        sb1hi = __byte_perm(sb1, 0, 0x3232);
       }
       const uint32_t wa0[4] = {qa0.x, qa0.y, qa0.z, qa0.w};
       const uint32_t wb0[4] = {qb0.x, qb0.y, qb0.z, qb0.w};
@@ -491,38 +502,44 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
             xb[n] = lds128(st + G::B + row * G::BROW + (act_unit<FMT>(U) << 4));
           }
         }
+        // weights of the two k-steps of this unit: FP8 uses one 32-bit word
+        // (4 codes) per row per k-step, NVFP4 one word (8 codes) per row per 2 k-steps
+        uint32_t dA0[2][4], dA1[2][4];  // [k-step][a-reg]
+        if (FMT == 1) {
+#pragma unroll
+          for (int ss = 0; ss < 2; ++ss) {
+            const int s_ = 2 * u + ss;
+            e4m3x4_to_f16x4(wa0[s_], dA0[ss][0], dA0[ss][2]);
+            e4m3x4_to_f16x4(wb0[s_], dA0[ss][1], dA0[ss][3]);
+            e4m3x4_to_f16x4(wa1[s_], dA1[ss][0], dA1[ss][2]);
+            e4m3x4_to_f16x4(wb1[s_], dA1[ss][1], dA1[ss][3]);
+          }
+        } else {
+          // word u holds k-steps 2u (bytes 0,1) and 2u+1 (bytes 2,3); the
+          // 16-element scale block of k-step s_ is 2c + (s_ >> 2)
+          const uint32_t ca0 = (u < 2) ? sa0lo : sa0hi, cb0 = (u < 2) ? sb0lo : sb0hi;
+          const uint32_t ca1 = (u < 2) ? sa1lo : sa1hi, cb1 = (u < 2) ? sb1lo : sb1hi;
+          uint32_t qa[4], qb[4], qc[4], qd[4];
+          e2m1x8_to_f16x8(wa0[u], qa);
+          e2m1x8_to_f16x8(wb0[u], qb);
+          e2m1x8_to_f16x8(wa1[u], qc);
+          e2m1x8_to_f16x8(wb1[u], qd);
+#pragma unroll
+          for (int ss = 0; ss < 2; ++ss) {
+            dA0[ss][0] = hmul2_u32(qa[2 * ss], ca0);
+            dA0[ss][2] = hmul2_u32(qa[2 * ss + 1], ca0);
+            dA0[ss][1] = hmul2_u32(qb[2 * ss], cb0);
+            dA0[ss][3] = hmul2_u32(qb[2 * ss + 1], cb0);
+            dA1[ss][0] = hmul2_u32(qc[2 * ss], ca1);
+            dA1[ss][2] = hmul2_u32(qc[2 * ss + 1], ca1);
+            dA1[ss][1] = hmul2_u32(qd[2 * ss], cb1);
+            dA1[ss][3] = hmul2_u32(qd[2 * ss + 1], cb1);
+          }
+        }
 #pragma unroll
         for (int ss = 0; ss < 2; ++ss) {
-          const int s_ = 2 * u + ss;  // k-step within the half
-          uint32_t A0r[4], A1r[4];
-          if (FMT == 1) {
-            const uint32_t xa0 = wa0[s_], xb0_ = wb0[s_], xa1 = wa1[s_], xb1_ = wb1[s_];
-            A0r[0] = e4m3x2_to_f16x2(xa0 & 0xFFFFu);
-            A0r[1] = e4m3x2_to_f16x2(xb0_ & 0xFFFFu);
-            A0r[2] = e4m3x2_to_f16x2(xa0 >> 16);
-            A0r[3] = e4m3x2_to_f16x2(xb0_ >> 16);
-            A1r[0] = e4m3x2_to_f16x2(xa1 & 0xFFFFu);
-            A1r[1] = e4m3x2_to_f16x2(xb1_ & 0xFFFFu);
-            A1r[2] = e4m3x2_to_f16x2(xa1 >> 16);
-            A1r[3] = e4m3x2_to_f16x2(xb1_ >> 16);
-          } else {
-            const int sh = 16 * (s_ & 1);
-            const int wi = s_ >> 1;
-            const uint32_t pa0 = (wa0[wi] >> sh), pb0 = (wb0[wi] >> sh);
-            const uint32_t pa1 = (wa1[wi] >> sh), pb1 = (wb1[wi] >> sh);
-            // scale of this k-step's 16-block: low half for s_ < 4, high half otherwise
-            const uint32_t sel = (s_ < 4) ? 0x1010u : 0x3232u;
-            const uint32_t ca0 = __byte_perm(sa0, 0, sel), cb0 = __byte_perm(sb0, 0, sel);
-            const uint32_t ca1 = __byte_perm(sa1, 0, sel), cb1 = __byte_perm(sb1, 0, sel);
-            A0r[0] = hmul2_u32(e2m1x2_to_f16x2(pa0 & 0xFFu), ca0);
-            A0r[1] = hmul2_u32(e2m1x2_to_f16x2(pb0 & 0xFFu), cb0);
-            A0r[2] = hmul2_u32(e2m1x2_to_f16x2((pa0 >> 8) & 0xFFu), ca0);
-            A0r[3] = hmul2_u32(e2m1x2_to_f16x2((pb0 >> 8) & 0xFFu), cb0);
-            A1r[0] = hmul2_u32(e2m1x2_to_f16x2(pa1 & 0xFFu), ca1);
-            A1r[1] = hmul2_u32(e2m1x2_to_f16x2(pb1 & 0xFFu), cb1);
-            A1r[2] = hmul2_u32(e2m1x2_to_f16x2((pa1 >> 8) & 0xFFu), ca1);
-            A1r[3] = hmul2_u32(e2m1x2_to_f16x2((pb1 >> 8) & 0xFFu), cb1);
-          }
+          const uint32_t* A0r = dA0[ss];
+          const uint32_t* A1r = dA1[ss];
 #pragma unroll
           for (int n = 0; n < NTILE; ++n) {
             if (n < ntiles) {

@@ -174,23 +174,26 @@ __global__ void __launch_bounds__(256) route_kernel(const RouteParams p) {
   const int nt = min(kRouteTok, p.T - t0);
   const int H = p.H, E = p.E;
 
-  // accumulators and counters of the later kernels start from zero
-  if (p.fused) {
-    const size_t nthr = (size_t)gridDim.x * gridDim.y * blockDim.x;
-    const size_t tid = ((size_t)blockIdx.y * gridDim.x + blockIdx.x) * blockDim.x + threadIdx.x;
-    const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (size_t i = tid; i < p.zero_a_n4; i += nthr) p.zero_a[i] = z;
-    for (size_t i = tid; i < p.zero_b_n4; i += nthr) p.zero_b[i] = z;
-    for (size_t i = tid; i < (size_t)p.zero_c_n; i += nthr) p.zero_c[i] = 0u;
-    for (size_t i = tid; i < (size_t)p.zero_d_n; i += nthr) p.zero_d[i] = 0u;
-  }
-
-  // stage this chunk's token rows
+  // stage this chunk's token rows: every thread issues all of its 16-byte
+  // loads before storing any of them (one memory latency, not one per load)
   {
     const uint4* src = reinterpret_cast<const uint4*>(p.x + (size_t)t0 * H);
     uint4* dst = reinterpret_cast<uint4*>(xs);
     const int n16 = nt * H / 8;
-    for (int i = threadIdx.x; i < n16; i += blockDim.x) dst[i] = __ldg(src + i);
+    constexpr int BATCH = 16;
+    for (int base = 0; base < n16; base += BATCH * 256) {
+      uint4 v[BATCH];
+#pragma unroll
+      for (int q = 0; q < BATCH; ++q) {
+        const int i = base + q * 256 + threadIdx.x;
+        if (i < n16) v[q] = __ldg(src + i);
+      }
+#pragma unroll
+      for (int q = 0; q < BATCH; ++q) {
+        const int i = base + q * 256 + threadIdx.x;
+        if (i < n16) dst[i] = v[q];
+      }
+    }
   }
   __syncthreads();
   if (p.prenorm && warp < nt) {
@@ -220,20 +223,31 @@ __global__ void __launch_bounds__(256) route_kernel(const RouteParams p) {
 #pragma unroll
     for (int t = 0; t < kRouteTok; ++t) acc[t] = 0.f;
     const float* wrow = p.wr + (size_t)e * H;
-    for (int h = lane * 4; h < H; h += 128) {
-      const float4 w = __ldg(reinterpret_cast<const float4*>(wrow + h));
+    // 16 router loads in flight per lane before any is used
+    constexpr int DEPTH = 16;
+    for (int h0 = lane * 4; h0 < H; h0 += 128 * DEPTH) {
+      float4 w[DEPTH];
 #pragma unroll
-      for (int t = 0; t < kRouteTok; ++t) {
-        if (t < nt) {
-          const uint2 xv = *reinterpret_cast<const uint2*>(xs + (size_t)t * H + h);
-          const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&xv.x));
-          const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&xv.y));
-          float s = acc[t];
-          s = fmaf(a.x, w.x, s);
-          s = fmaf(a.y, w.y, s);
-          s = fmaf(b.x, w.z, s);
-          s = fmaf(b.y, w.w, s);
-          acc[t] = s;
+      for (int q = 0; q < DEPTH; ++q)
+        w[q] = (h0 + 128 * q < H) ? __ldg(reinterpret_cast<const float4*>(wrow + h0 + 128 * q))
+                                  : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+      for (int q = 0; q < DEPTH; ++q) {
+        const int h = h0 + 128 * q;
+        if (h >= H) break;
+#pragma unroll
+        for (int t = 0; t < kRouteTok; ++t) {
+          if (t < nt) {
+            const uint2 xv = *reinterpret_cast<const uint2*>(xs + (size_t)t * H + h);
+            const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&xv.x));
+            const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&xv.y));
+            float s = acc[t];
+            s = fmaf(a.x, w[q].x, s);
+            s = fmaf(a.y, w[q].y, s);
+            s = fmaf(b.x, w[q].z, s);
+            s = fmaf(b.y, w[q].w, s);
+            acc[t] = s;
+          }
         }
       }
     }
@@ -243,6 +257,17 @@ __global__ void __launch_bounds__(256) route_kernel(const RouteParams p) {
       const float b = p.bias ? __ldg(p.bias + e) : 0.f;
       for (int t = 0; t < nt; ++t) p.logits[(size_t)(t0 + t) * E + e] = acc[t] + b;
     }
+  }
+
+  // accumulators and counters of the later kernels start from zero
+  if (p.fused) {
+    const size_t nthr = (size_t)gridDim.x * gridDim.y * blockDim.x;
+    const size_t tid = ((size_t)blockIdx.y * gridDim.x + blockIdx.x) * blockDim.x + threadIdx.x;
+    const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (size_t i = tid; i < p.zero_a_n4; i += nthr) p.zero_a[i] = z;
+    for (size_t i = tid; i < p.zero_b_n4; i += nthr) p.zero_b[i] = z;
+    for (size_t i = tid; i < (size_t)p.zero_c_n; i += nthr) p.zero_c[i] = 0u;
+    for (size_t i = tid; i < (size_t)p.zero_d_n; i += nthr) p.zero_d[i] = 0u;
   }
 
   // chunk ticket: the last of this chunk's expert blocks does the top-k

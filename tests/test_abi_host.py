@@ -91,11 +91,13 @@ def test_decode_layer_rejects_bad_arguments_before_launch(lib):
     assert call(ws=P(0x400010)) == -1            # workspace alignment
     assert call(k=3, c=fake_weights(E=2)) == -2
     assert call(T=0) == 0                        # empty batch is a no-op
+    assert call(T=0, x=None, out=None) == 0      # ... even with null row pointers
 
 
 def test_other_entry_points_validate(lib):
     P = ctypes.c_void_p
-    assert lib.moe_permute(None, 4, 2, 8, P(1), P(1), P(1), P(1), P(1), None) == -1
+    assert lib.moe_permute(None, 4, 2, 8, P(16), P(16), P(16), P(16), P(16), None) == -1
+    assert lib.moe_permute(P(16), 4, 2, 8, None, P(16), P(16), P(16), P(16), None) == -1
     assert lib.moe_permute(P(16), 4, 9, 8, P(16), P(16), P(16), P(16), P(16), None) == -2
     assert lib.moe_combine(P(16), P(16), P(16), 4, 2, 6, None, P(16), None) == -1  # H % 4
     n = ctypes.c_size_t(0)
