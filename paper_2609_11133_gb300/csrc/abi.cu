@@ -101,7 +101,26 @@ bool map_sf(CUtensorMap* m, const void* sf, int E, int N, int K) {
 
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
-int nt_for(int T) { return T <= 8 ? 8 : (T <= 16 ? 16 : 32); }
+// Expert engine: tcgen05 (default) or the warp-MMA engine (MOE_ENGINE=mma).
+bool use_tc_engine() {
+  static int v = -1;
+  if (v < 0) {
+    const char* s = std::getenv("MOE_ENGINE");
+    v = (s && std::strcmp(s, "mma") == 0) ? 0 : 1;
+  }
+  return v == 1;
+}
+
+// Token-chunk size of the expert kernels (the N side of the MMA).
+// MOE_NT=8|16|32 overrides the choice (for measurements).
+int nt_for(int T) {
+  if (const char* s = std::getenv("MOE_NT")) {
+    const int v = std::atoi(s);
+    if (v == 16 || v == 32 || (v == 8 && !use_tc_engine())) return v;
+  }
+  if (use_tc_engine()) return T <= 16 ? 16 : 32;
+  return T <= 8 ? 8 : (T <= 16 ? 16 : 32);
+}
 
 // ------------------------------------------------------------------ validation
 int check_weights(const moe_expert_weights_t* w) {
@@ -166,10 +185,14 @@ int run_experts(const ExpertRun& r, cudaStream_t st, cudaEvent_t ev_mid) {
   }
   __half* x16 = ws_ptr<__half>(r.ws, r.L.x16);
   __half* h16 = ws_ptr<__half>(r.ws, r.L.h16);
+  const bool tc = use_tc_engine();
+  // token rows: tcgen05 reads 64-element 128B-swizzled K atoms, warp MMA whole K-stages
+  const uint32_t bcols = tc ? 64u : (uint32_t)KEL;
+  const CUtensorMapSwizzle bsw = tc ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE;
   ok = ok && map_2d(&m1.b, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, x16, (uint64_t)H, (uint64_t)r.T,
-                    (uint64_t)H * 2, KEL, 1, CU_TENSOR_MAP_SWIZZLE_NONE);
+                    (uint64_t)H * 2, bcols, 1, bsw);
   ok = ok && map_2d(&m2.b, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, h16, (uint64_t)I,
-                    (uint64_t)r.T * r.k, (uint64_t)I * 2, KEL, 8, CU_TENSOR_MAP_SWIZZLE_NONE);
+                    (uint64_t)r.T * r.k, (uint64_t)I * 2, bcols, 8, bsw);
   if (!ok) return MOE_ERR_CUDA;
 
   FfnParams p{};
@@ -214,12 +237,16 @@ int run_experts(const ExpertRun& r, cudaStream_t st, cudaEvent_t ev_mid) {
   p2.residual = r.residual;
   p2.cnt = ws_ptr<unsigned>(r.ws, r.L.dn_cnt);
 
-  cudaError_t err = fp4 ? launch_ffn<2>(r.nt, r.sms, m1, p1, st, false)
-                        : launch_ffn<1>(r.nt, r.sms, m1, p1, st, false);
+  auto launch = [&](const FfnMaps& m, const FfnParams& pp) {
+    if (tc)
+      return fp4 ? launch_ffn_tc<2>(r.nt, r.sms, m, pp, st) : launch_ffn_tc<1>(r.nt, r.sms, m, pp, st);
+    return fp4 ? launch_ffn<2>(r.nt, r.sms, m, pp, st, false)
+               : launch_ffn<1>(r.nt, r.sms, m, pp, st, false);
+  };
+  cudaError_t err = launch(m1, p1);
   if (err != cudaSuccess) return MOE_ERR_CUDA;
   if (ev_mid && cudaEventRecord(ev_mid, st) != cudaSuccess) return MOE_ERR_CUDA;
-  err = fp4 ? launch_ffn<2>(r.nt, r.sms, m2, p2, st, false)
-            : launch_ffn<1>(r.nt, r.sms, m2, p2, st, false);
+  err = launch(m2, p2);
   return err == cudaSuccess ? MOE_OK : MOE_ERR_CUDA;
 }
 
@@ -366,6 +393,7 @@ int moe_expert_ffn(const void* x, const moe_expert_weights_t* w, const int32_t* 
   pp.k = k;
   pp.fmt = w->fmt;
   pp.nt = nt;
+  pp.unit_perm = (!use_tc_engine() && w->fmt == MOE_FMT_NVFP4) ? 1 : 0;
   pp.x16 = ws_ptr<__half>(ws, L.x16);
   pp.xinv = ws_ptr<float>(ws, L.xinv);
   pp.offsets = offsets;
@@ -452,6 +480,7 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
   p.fmt = w->fmt;
   p.fused = 1;
   p.nt = nt;
+  p.unit_perm = (!use_tc_engine() && w->fmt == MOE_FMT_NVFP4) ? 1 : 0;
   p.logits = logits_out ? logits_out : ws_ptr<float>(ws, L.logits);
   p.ids = ws_ptr<int>(ws, L.ids);
   p.gates = ws_ptr<float>(ws, L.gates);

@@ -3,4 +3,5 @@
 
 namespace moe {
 MOE_DEFINE_FFN_LAUNCH(1)
+MOE_DEFINE_FFN_TC_LAUNCH(1)
 }  // namespace moe

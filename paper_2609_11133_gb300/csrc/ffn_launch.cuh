@@ -3,6 +3,7 @@
 #pragma once
 
 #include "ffn.cuh"
+#include "ffn_tc.cuh"
 
 namespace moe {
 
@@ -17,6 +18,12 @@ cudaError_t launch_ffn(int nt, int grid, const FfnMaps& maps, const FfnParams& p
 
 template <int FMT>
 int ffn_smem_bytes(int nt);
+
+// The tcgen05 engine (ffn_tc.cuh); nt in {16, 32}.
+template <int FMT>
+cudaError_t launch_ffn_tc(int nt, int grid, const FfnMaps& maps, const FfnParams& p,
+                          cudaStream_t st);
+
 
 #define MOE_DEFINE_FFN_LAUNCH(FMTV)                                                            \
   template <int NT>                                                                             \
@@ -57,6 +64,31 @@ int ffn_smem_bytes(int nt);
   int ffn_smem_bytes<FMTV>(int nt) {                                                            \
     return nt == 8 ? StageGeom<FMTV, 8>::SMEM                                                   \
                    : (nt == 16 ? StageGeom<FMTV, 16>::SMEM : StageGeom<FMTV, 32>::SMEM);        \
+  }
+
+#define MOE_DEFINE_FFN_TC_LAUNCH(FMTV)                                                         \
+  template <int NT>                                                                             \
+  static cudaError_t launch_ffn_tc_nt_##FMTV(int grid, const FfnMaps& m, const FfnParams& p,   \
+                                             cudaStream_t st) {                                 \
+    auto kern = ffn_tc_kernel<FMTV, NT>;                                                        \
+    const int smem = TcGeom<FMTV, NT>::SMEM;                                                    \
+    cudaError_t err =                                                                           \
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);          \
+    if (err != cudaSuccess) return err;                                                         \
+    kern<<<grid, kTcThreads, smem, st>>>(m.a0, m.a1, m.s0, m.s1, m.b, p);                       \
+    return cudaGetLastError();                                                                  \
+  }                                                                                             \
+  template <>                                                                                   \
+  cudaError_t launch_ffn_tc<FMTV>(int nt, int grid, const FfnMaps& m, const FfnParams& p,      \
+                                  cudaStream_t st) {                                            \
+    switch (nt) {                                                                               \
+      case 16:                                                                                  \
+        return launch_ffn_tc_nt_##FMTV<16>(grid, m, p, st);                                     \
+      case 32:                                                                                  \
+        return launch_ffn_tc_nt_##FMTV<32>(grid, m, p, st);                                     \
+      default:                                                                                  \
+        return cudaErrorInvalidValue;                                                           \
+    }                                                                                           \
   }
 
 }  // namespace moe

@@ -11,7 +11,7 @@ namespace moe {
 // the unit order the expert kernels read (act_pos), and store 1/factor.
 template <int FMT>
 __device__ void convert_row_x16(const __nv_bfloat16* row, int H, __half* dst, float* inv,
-                                int lane) {
+                                int lane, bool perm) {
   float amax = 0.f;
   for (int h = lane * 8; h < H; h += 256) {
     const uint4 v = *reinterpret_cast<const uint4*>(row + h);
@@ -36,18 +36,21 @@ __device__ void convert_row_x16(const __nv_bfloat16* row, int H, __half* dst, fl
       oh[i] = __floats2half2_rn(f.x * sc, f.y * sc);
     }
     const int U = h >> 3;
-    const int phys = (U / UPB) * UPB + act_unit<FMT>(U % UPB);
+    const int phys = perm ? (U / UPB) * UPB + act_unit<FMT>(U % UPB) : U;
     *reinterpret_cast<uint4*>(dst + (size_t)phys * 8) = o;
   }
   if (lane == 0) *inv = 1.f / sc;
 }
 
+// perm: store the 16-byte units in the order of the warp-MMA engine (ffn.cuh);
+// the tcgen05 engine reads rows in natural order.
 __device__ __forceinline__ void convert_row_dispatch(int fmt, const __nv_bfloat16* row, int H,
-                                                     __half* dst, float* inv, int lane) {
+                                                     __half* dst, float* inv, int lane,
+                                                     bool perm) {
   if (fmt == 2)
-    convert_row_x16<2>(row, H, dst, inv, lane);
+    convert_row_x16<2>(row, H, dst, inv, lane, perm);
   else
-    convert_row_x16<1>(row, H, dst, inv, lane);
+    convert_row_x16<1>(row, H, dst, inv, lane, perm);
 }
 
 __device__ __forceinline__ unsigned lanemask_lt() {
@@ -213,7 +216,7 @@ __global__ void __launch_bounds__(256) route_kernel(const RouteParams p) {
   if (p.fused && eb == 0 && warp < nt) {
     const int t = t0 + warp;
     convert_row_dispatch(p.fmt, xs + (size_t)warp * H, H, p.x16 + (size_t)t * H, p.xinv + t,
-                         lane);
+                         lane, p.unit_perm != 0);
   }
 
   // router GEMV: warp -> expert row, lanes -> 4 consecutive h per 128
@@ -380,7 +383,7 @@ __global__ void __launch_bounds__(256) prep_kernel(const PrepParams p) {
   const int t = blockIdx.x * 8 + warp;
   if (t < p.T)
     convert_row_dispatch(p.fmt, p.x + (size_t)t * p.H, p.H, p.x16 + (size_t)t * p.H, p.xinv + t,
-                         lane);
+                         lane, p.unit_perm != 0);
   if (blockIdx.x == 0) {
     for (int e = threadIdx.x; e < p.E; e += blockDim.x)
       p.counts[e] = __ldg(p.offsets + e + 1) - __ldg(p.offsets + e);

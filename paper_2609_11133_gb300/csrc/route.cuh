@@ -23,6 +23,7 @@ struct RouteParams {
   const float* wr;
   const float* bias;
   int T, H, E, k, renorm, prenorm, fmt, fused, nt;
+  int unit_perm;  // x16 rows in the warp-MMA engine's unit order
   float* logits;  // [T, E]
   int* ids;       // [T, k]
   float* gates;   // [T, k]
@@ -53,6 +54,7 @@ struct RouteParams {
 struct PrepParams {
   const __nv_bfloat16* x;
   int T, H, E, k, fmt, nt;
+  int unit_perm;
   __half* x16;
   float* xinv;
   const int* offsets;  // [E+1] from the permutation
