@@ -152,6 +152,7 @@ int moe_combine(const float* y_perm, const float* topk_w, const int32_t* inv_per
  *   w: expert weights (w->H must equal the row length of x and router_w);
  *   flags: MOE_FLAG_*; residual [T, H] bf16 or NULL (may alias out);
  *   out [T, H] bf16, must not alias x;
+ *   alignment: x and router_w 16 bytes, out and residual 8 bytes, ws 256 bytes;
  *   ws: at least moe_workspace_size(w, T, k) bytes, zeroed once before
  *   first use (moe_workspace_init). */
 int moe_decode_layer(const void* x, const float* router_w, const float* router_bias,

@@ -101,12 +101,12 @@ bool map_sf(CUtensorMap* m, const void* sf, int E, int N, int K) {
 
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
-// Expert engine: tcgen05 (default) or the warp-MMA engine (MOE_ENGINE=mma).
+// Expert engine: warp MMA (default) or tcgen05 (MOE_ENGINE=tc).
 bool use_tc_engine() {
   static int v = -1;
   if (v < 0) {
     const char* s = std::getenv("MOE_ENGINE");
-    v = (s && std::strcmp(s, "mma") == 0) ? 0 : 1;
+    v = (s && std::strcmp(s, "tc") == 0) ? 1 : 0;
   }
   return v == 1;
 }
@@ -119,7 +119,9 @@ int nt_for(int T) {
     if (v == 16 || v == 32 || (v == 8 && !use_tc_engine())) return v;
   }
   if (use_tc_engine()) return T <= 16 ? 16 : 32;
-  return T <= 8 ? 8 : (T <= 16 ? 16 : 32);
+  // 16-token chunks keep five stages in flight; an expert with more tokens
+  // is processed in several chunks
+  return T <= 8 ? 8 : 16;
 }
 
 // ------------------------------------------------------------------ validation
@@ -220,7 +222,6 @@ int run_experts(const ExpertRun& r, cudaStream_t st, cudaEvent_t ev_mid) {
   p1.gu = ws_ptr<float>(r.ws, r.L.gu);
   p1.h16 = h16;
   p1.hinv = ws_ptr<float>(r.ws, r.L.hinv);
-  p1.cnt = ws_ptr<unsigned>(r.ws, r.L.gu_cnt);
   p1.test_stall = r.test_stall;
 
   FfnParams p2 = p;
@@ -235,7 +236,6 @@ int run_experts(const ExpertRun& r, cudaStream_t st, cudaEvent_t ev_mid) {
   p2.y_perm = r.y_perm;
   p2.out = r.out;
   p2.residual = r.residual;
-  p2.cnt = ws_ptr<unsigned>(r.ws, r.L.dn_cnt);
 
   auto launch = [&](const FfnMaps& m, const FfnParams& pp) {
     if (tc)
@@ -246,7 +246,13 @@ int run_experts(const ExpertRun& r, cudaStream_t st, cudaEvent_t ev_mid) {
   cudaError_t err = launch(m1, p1);
   if (err != cudaSuccess) return MOE_ERR_CUDA;
   if (ev_mid && cudaEventRecord(ev_mid, st) != cudaSuccess) return MOE_ERR_CUDA;
+  const bool perm = !tc && fp4;  // h16 unit order of the warp-MMA NVFP4 engine
+  err = fp4 ? launch_swiglu<2>(r.T * r.k, r.sms, p1, perm, st)
+            : launch_swiglu<1>(r.T * r.k, r.sms, p1, perm, st);
+  if (err != cudaSuccess) return MOE_ERR_CUDA;
   err = launch(m2, p2);
+  if (err != cudaSuccess) return MOE_ERR_CUDA;
+  if (r.fused) err = launch_finalize(r.sms, p2, st);
   return err == cudaSuccess ? MOE_OK : MOE_ERR_CUDA;
 }
 
@@ -404,8 +410,6 @@ int moe_expert_ffn(const void* x, const moe_expert_weights_t* w, const int32_t* 
   pp.zero_a_n4 = (size_t)T * k * w->H / 4;
   pp.zero_b = ws_ptr<float4>(ws, L.gu);
   pp.zero_b_n4 = (size_t)T * k * 2 * w->I / 4;
-  pp.zero_c = ws_ptr<unsigned>(ws, L.gu_cnt);
-  pp.zero_c_n = w->E;
   if (launch_prep(pp, st) != cudaSuccess) return MOE_ERR_CUDA;
   ExpertRun r{};
   r.w = w;
@@ -450,8 +454,8 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
   if (rc) return rc;
   if (T == 0) return MOE_OK;  // an empty batch may come with null row pointers
   if (!x || !router_w || !out || !ws) return MOE_ERR_INVALID_ARG;
-  if (!aligned(x, 16) || !aligned(router_w, 16) || !aligned(ws, 256) || !aligned(out, 2) ||
-      (residual && !aligned(residual, 2)))
+  if (!aligned(x, 16) || !aligned(router_w, 16) || !aligned(ws, 256) || !aligned(out, 8) ||
+      (residual && !aligned(residual, 8)))
     return MOE_ERR_INVALID_ARG;
   if (out == x) return MOE_ERR_INVALID_ARG;
   const int E = w->E, H = w->H, I = w->I;
@@ -494,10 +498,6 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
   p.zero_a_n4 = (size_t)T * k * 2 * I / 4;
   p.zero_b = ws_ptr<float4>(ws, L.oacc);
   p.zero_b_n4 = (size_t)T * H / 4;
-  p.zero_c = ws_ptr<unsigned>(ws, L.gu_cnt);
-  p.zero_c_n = E;
-  p.zero_d = ws_ptr<unsigned>(ws, L.dn_cnt);
-  p.zero_d_n = H / 256;
   p.counts = ws_ptr<int>(ws, L.counts);
   p.offsets = ws_ptr<int>(ws, L.offsets);
   p.sorted = ws_ptr<int>(ws, L.sorted);

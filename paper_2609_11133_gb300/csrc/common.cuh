@@ -35,8 +35,6 @@ struct WsLayout {
   size_t status;       // u32 device status word
   size_t route_chunk;  // u32 [nChunks] per-token-chunk arrival tickets
   size_t route_done;   // u32 chunk-completion ticket
-  size_t gu_cnt;       // u32 [E] per-active-expert stage counters (gate/up)
-  size_t dn_cnt;       // u32 [H/256] per-row-tile stage counters (down)
   // routing
   size_t logits;   // f32 [T, E]
   size_t ids;      // i32 [T, k]
@@ -73,8 +71,6 @@ inline WsLayout ws_layout(int T, int k, int E, int H, int I) {
   L.status = take(4);
   L.route_chunk = take(4 * (size_t)(L.nChunks > 0 ? L.nChunks : 1));
   L.route_done = take(4);
-  L.gu_cnt = take(4 * (size_t)E);
-  L.dn_cnt = take(4 * (size_t)(H / 256 > 0 ? H / 256 : 1));
   L.logits = take(4 * (size_t)T * E);
   L.ids = take(4 * TK);
   L.gates = take(4 * TK);

@@ -24,13 +24,11 @@
 //   The tensor pipe (mma m16n8k16, fp32 accumulate) does the multiply-adds
 //   with the tokens as the n=8 side; FP8 block scales and NVFP4 tensor
 //   scales are applied to the fp32 accumulators.
-// * Fusion.  The gate/up step writes fp32 pre-activations; the CTA that
-//   completes an expert's last stage (a ticket counter) applies SwiGLU and
-//   writes the f16 input of the down step.  The down step multiplies by the
-//   gate weight and adds straight into a [T, H] fp32 accumulator (the
-//   scatter-combine); the CTA that completes a row tile's last stage
-//   converts those columns to bf16 (+ residual).  No wait depends on
-//   another CTA: every cross-CTA handoff is a ticket, never a spin.
+// * Fusion.  The gate/up step adds fp32 pre-activations into [T*k, 2I]
+//   accumulators; swiglu_kernel turns them into the f16 input of the down
+//   step.  The down step multiplies by the gate weight and adds straight into
+//   a [T, H] fp32 accumulator (the scatter-combine); finalize_kernel writes
+//   bf16 (+ residual).  No wait depends on another CTA.
 #pragma once
 
 #include "common.cuh"
@@ -114,7 +112,6 @@ struct FfnParams {
   float* y_perm;       // phase 2 unfused output [T*k, H]
   __nv_bfloat16* out;  // phase 2 fused output
   const __nv_bfloat16* residual;
-  unsigned* cnt;       // ticket counters (phase 1: [E] by slot, phase 2: [H/256])
   uint32_t* status;
   uint64_t wait_ns;
   int test_stall;      // test hook: producer withholds its first stage
@@ -145,6 +142,96 @@ __device__ __forceinline__ ItemInfo decode_item(long long it, int rtiles, const 
   return r;
 }
 
+// ------------------------------------------------------------------ between and after the phases
+// SwiGLU of every assignment row: h = silu(g) * u from the fp32 gate|up
+// accumulators, scaled per row by a power of two into f16 (in the unit order
+// of the warp-MMA NVFP4 layout when `perm`).  One warp per row; every lane
+// issues its 16-byte loads in batches of four before using them.
+template <int FMT>
+__global__ void __launch_bounds__(256) swiglu_kernel(const FfnParams p, int rows, int perm) {
+  const int lane = threadIdx.x & 31;
+  const int gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int nw = (gridDim.x * blockDim.x) >> 5;
+  pdl_wait();
+  const int n4 = p.I / 4;
+  constexpr int D = 4;
+  for (int row = gw; row < rows; row += nw) {
+    const float4* g4 = reinterpret_cast<const float4*>(p.gu + (size_t)row * 2 * p.I);
+    const float4* u4 = reinterpret_cast<const float4*>(p.gu + (size_t)row * 2 * p.I + p.I);
+    float amax = 0.f;
+    for (int base = lane; base < n4; base += 32 * D) {
+      float4 gv[D], uv[D];
+#pragma unroll
+      for (int q = 0; q < D; ++q)
+        if (base + 32 * q < n4) {
+          gv[q] = __ldcg(g4 + base + 32 * q);
+          uv[q] = __ldcg(u4 + base + 32 * q);
+        }
+#pragma unroll
+      for (int q = 0; q < D; ++q)
+        if (base + 32 * q < n4) {
+          amax = fmaxf(amax, fabsf(gv[q].x / (1.f + expf(-gv[q].x)) * uv[q].x));
+          amax = fmaxf(amax, fabsf(gv[q].y / (1.f + expf(-gv[q].y)) * uv[q].y));
+          amax = fmaxf(amax, fabsf(gv[q].z / (1.f + expf(-gv[q].z)) * uv[q].z));
+          amax = fmaxf(amax, fabsf(gv[q].w / (1.f + expf(-gv[q].w)) * uv[q].w));
+        }
+    }
+    amax = warp_max(amax);
+    const float sc = pow2_scale_for(amax);
+    __half* hr = p.h16 + (size_t)row * p.I;
+    for (int base = lane; base < n4; base += 32 * D) {
+      float4 gv[D], uv[D];
+#pragma unroll
+      for (int q = 0; q < D; ++q)
+        if (base + 32 * q < n4) {
+          gv[q] = __ldcg(g4 + base + 32 * q);
+          uv[q] = __ldcg(u4 + base + 32 * q);
+        }
+#pragma unroll
+      for (int q = 0; q < D; ++q) {
+        const int i = base + 32 * q;
+        if (i < n4) {
+          const __half2 lo = __floats2half2_rn(gv[q].x / (1.f + expf(-gv[q].x)) * uv[q].x * sc,
+                                               gv[q].y / (1.f + expf(-gv[q].y)) * uv[q].y * sc);
+          const __half2 hi = __floats2half2_rn(gv[q].z / (1.f + expf(-gv[q].z)) * uv[q].z * sc,
+                                               gv[q].w / (1.f + expf(-gv[q].w)) * uv[q].w * sc);
+          uint2 o;
+          o.x = *reinterpret_cast<const uint32_t*>(&lo);
+          o.y = *reinterpret_cast<const uint32_t*>(&hi);
+          const int f = 4 * i;  // 4 consecutive columns stay inside one 16-byte unit
+          *reinterpret_cast<uint2*>(hr + (perm ? act_pos<FMT>(f) : f)) = o;
+        }
+      }
+    }
+    if (lane == 0) p.hinv[row] = 1.f / sc;
+  }
+}
+
+// out = bf16(oacc + residual), four columns per thread.
+static __global__ void __launch_bounds__(256) finalize_kernel(const FfnParams p) {
+  pdl_wait();
+  const size_t n4 = (size_t)p.T * p.H / 4;
+  for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4;
+       i += (size_t)gridDim.x * blockDim.x) {
+    float4 a = __ldcg(reinterpret_cast<const float4*>(p.oacc) + i);
+    if (p.residual) {
+      const uint2 r = *(reinterpret_cast<const uint2*>(p.residual) + i);
+      const float2 r0 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&r.x));
+      const float2 r1 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&r.y));
+      a.x += r0.x;
+      a.y += r0.y;
+      a.z += r1.x;
+      a.w += r1.y;
+    }
+    const __nv_bfloat162 o0 = __floats2bfloat162_rn(a.x, a.y);
+    const __nv_bfloat162 o1 = __floats2bfloat162_rn(a.z, a.w);
+    uint2 o;
+    o.x = *reinterpret_cast<const uint32_t*>(&o0);
+    o.y = *reinterpret_cast<const uint32_t*>(&o1);
+    *(reinterpret_cast<uint2*>(p.out) + i) = o;
+  }
+}
+
 // ------------------------------------------------------------------ the kernel
 template <int FMT, int NT>
 __global__ void __launch_bounds__(kFfnThreads, 1)
@@ -165,7 +252,6 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
   __shared__ int s_cpre[kMaxE + 1];
   __shared__ int s_tok[NT];
   __shared__ volatile int s_abort;
-  __shared__ int s_last;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const bool is_producer = (warp == kFfnConsumerWarps);
@@ -274,7 +360,6 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
   float acc0[NTILE][4], acc1[NTILE][4];
   long long cur_item = -1;
   ItemInfo inf{};
-  int done_in_item = 0;
   // per-item column data
   float colscale[NTILE][2];
   int colrow[NTILE][2];   // flush destination row (assignment row or token)
@@ -319,9 +404,7 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
   // Adds the item's partial sums to the global accumulators, then takes the
   // item's ticket; the CTA completing an expert (phase 1) or a row tile
   // (phase 2) finishes it.
-  // `dead`: this warp stopped at an expired wait.  It still walks the item
-  // boundaries and joins both barriers so the consumer warps stay matched,
-  // but adds nothing and takes no ticket.
+  // `dead`: this warp stopped at an expired wait; it adds nothing.
   auto flush = [&](bool dead) {
     float ts0 = 1.f, ts1 = 1.f;
     if (FMT == 2) {
@@ -354,62 +437,6 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
           }
         }
       }
-    if (!(p.phase == 1 || p.fused)) return;
-    __threadfence();
-    asm volatile("bar.sync 1, %0;" ::"n"(kFfnConsumerWarps * 32) : "memory");
-    if (threadIdx.x == 0) {
-      s_last = 0;
-    }
-    if (threadIdx.x == 0 && !dead && !s_abort) {
-      unsigned key, need;
-      if (p.phase == 1) {
-        key = (unsigned)inf.slot;
-        need = (unsigned)((s_cpre[inf.slot + 1] - s_cpre[inf.slot]) * rtiles * KB);
-      } else {
-        key = (unsigned)inf.rt;
-        need = (unsigned)((long long)s_cpre[nA] * KB);
-      }
-      const unsigned old = atomicAdd(p.cnt + key, (unsigned)done_in_item);
-      const int last = (old + (unsigned)done_in_item == need);
-      if (last) {
-        p.cnt[key] = 0;
-        __threadfence();
-      }
-      s_last = last;
-    }
-    asm volatile("bar.sync 1, %0;" ::"n"(kFfnConsumerWarps * 32) : "memory");
-    if (!s_last) return;
-    const int ct = threadIdx.x;  // 0..255
-    if (p.phase == 1) {
-      // SwiGLU of this expert's rows -> f16 rows (power-of-two scaled) for the down step.
-      const int e = inf.e;
-      const int r0 = __ldg(p.offsets + e), r1 = r0 + __ldg(p.counts + e);
-      for (int row = r0 + warp; row < r1; row += kFfnConsumerWarps) {
-        const float* gr = p.gu + (size_t)row * 2 * p.I;
-        float amax = 0.f;
-        for (int f = lane; f < p.I; f += 32) {
-          const float gv = __ldcg(gr + f), uv = __ldcg(gr + p.I + f);
-          const float hv = gv / (1.f + expf(-gv)) * uv;
-          amax = fmaxf(amax, fabsf(hv));
-        }
-        amax = warp_max(amax);
-        const float sc = pow2_scale_for(amax);
-        __half* hr = p.h16 + (size_t)row * p.I;
-        for (int f = lane; f < p.I; f += 32) {
-          const float gv = __ldcg(gr + f), uv = __ldcg(gr + p.I + f);
-          const float hv = gv / (1.f + expf(-gv)) * uv;
-          hr[act_pos<FMT>(f)] = __float2half_rn(hv * sc);
-        }
-        if (lane == 0) p.hinv[row] = 1.f / sc;
-      }
-    } else {
-      const int col = inf.rt * 2 * kRowsHalf + ct;
-      for (int tok = 0; tok < p.T; ++tok) {
-        float v = __ldcg(p.oacc + (size_t)tok * p.H + col);
-        if (p.residual) v += __bfloat162float(p.residual[(size_t)tok * p.H + col]);
-        p.out[(size_t)tok * p.H + col] = __float2bfloat16_rn(v);
-      }
-    }
   };
 
   zero_acc();
@@ -426,7 +453,6 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
       cur_item = it;
       inf = decode_item(it, rtiles, s_cpre, nA, p, NT);
       load_item_cols();
-      done_in_item = 0;
     }
     if (dead) continue;
     // FP8 block scales of this stage (one per 128x128 tile of each box)
@@ -561,7 +587,6 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
         acc0[n][i] = fmaf(bs0, tmp0[n][i], acc0[n][i]);
         acc1[n][i] = fmaf(bs1, tmp1[n][i], acc1[n][i]);
       }
-    ++done_in_item;
   }
   if (cur_item >= 0) flush(dead);
 }

@@ -19,6 +19,11 @@ cudaError_t launch_ffn(int nt, int grid, const FfnMaps& maps, const FfnParams& p
 template <int FMT>
 int ffn_smem_bytes(int nt);
 
+// SwiGLU between the phases and the bf16 conversion after them.
+template <int FMT>
+cudaError_t launch_swiglu(int rows, int sms, const FfnParams& p, bool perm, cudaStream_t st);
+cudaError_t launch_finalize(int sms, const FfnParams& p, cudaStream_t st);
+
 // The tcgen05 engine (ffn_tc.cuh); nt in {16, 32}.
 template <int FMT>
 cudaError_t launch_ffn_tc(int nt, int grid, const FfnMaps& maps, const FfnParams& p,
@@ -64,6 +69,17 @@ cudaError_t launch_ffn_tc(int nt, int grid, const FfnMaps& maps, const FfnParams
   int ffn_smem_bytes<FMTV>(int nt) {                                                            \
     return nt == 8 ? StageGeom<FMTV, 8>::SMEM                                                   \
                    : (nt == 16 ? StageGeom<FMTV, 16>::SMEM : StageGeom<FMTV, 32>::SMEM);        \
+  }
+
+#define MOE_DEFINE_SWIGLU_LAUNCH(FMTV)                                                         \
+  template <>                                                                                   \
+  cudaError_t launch_swiglu<FMTV>(int rows, int sms, const FfnParams& p, bool perm,            \
+                                  cudaStream_t st) {                                            \
+    int blocks = (rows + 7) / 8;                                                                \
+    if (blocks > 4 * sms) blocks = 4 * sms;                                                     \
+    if (blocks < 1) blocks = 1;                                                                 \
+    swiglu_kernel<FMTV><<<blocks, 256, 0, st>>>(p, rows, perm ? 1 : 0);                         \
+    return cudaGetLastError();                                                                  \
   }
 
 #define MOE_DEFINE_FFN_TC_LAUNCH(FMTV)                                                         \

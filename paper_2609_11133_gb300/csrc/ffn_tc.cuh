@@ -15,8 +15,8 @@
 //   applied to it.
 // * Epilogue warps 8-11 read each stage's accumulator back (tcgen05.ld),
 //   apply the scale, keep the item's sums in registers, and flush them with
-//   red.global.add at the item's end, as ffn.cuh does; they also take the
-//   tickets.  Decoding never waits for an accumulator read.
+//   red.global.add at the item's end, as ffn.cuh does.  Decoding never waits
+//   for an accumulator read.
 // * Warp 12 (one thread) is the TMA producer.
 // Every mbarrier wait is bounded; TMEM is always released before exit.
 #pragma once
@@ -84,7 +84,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   __shared__ int s_tok[NT];
   __shared__ uint32_t s_tmem;
   __shared__ volatile int s_abort;
-  __shared__ int s_last;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
@@ -376,7 +375,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   for (int j = 0; j < NT; ++j) acc0[j] = acc1[j] = 0.f;
   bool dead = false;
 
-  auto flush = [&](const ItemInfo& fi, int done, bool is_dead) {
+  auto flush = [&](const ItemInfo& fi, bool is_dead) {
     float ts0 = 1.f, ts1 = 1.f;
     if (FMT == 2) {
       ts0 = __ldg(p.ts0 + fi.e);
@@ -412,64 +411,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
 #pragma unroll
     for (int j = 0; j < NT; ++j) acc0[j] = acc1[j] = 0.f;
-    if (!(p.phase == 1 || p.fused)) return;
-    __threadfence();
-    asm volatile("bar.sync 1, %0;" ::"n"(kEpiThreads) : "memory");
-    if (et == 0) s_last = 0;
-    if (et == 0 && !is_dead && !s_abort) {
-      unsigned key, need;
-      if (p.phase == 1) {
-        key = (unsigned)fi.slot;
-        need = (unsigned)((s_cpre[fi.slot + 1] - s_cpre[fi.slot]) * rtiles * KB);
-      } else {
-        key = (unsigned)fi.rt;
-        need = (unsigned)((long long)s_cpre[nA] * KB);
-      }
-      const unsigned old = atomicAdd(p.cnt + key, (unsigned)done);
-      const int last = (old + (unsigned)done == need);
-      if (last) {
-        p.cnt[key] = 0;
-        __threadfence();
-      }
-      s_last = last;
-    }
-    asm volatile("bar.sync 1, %0;" ::"n"(kEpiThreads) : "memory");
-    if (!s_last) return;
-    if (p.phase == 1) {
-      // SwiGLU of this expert's rows -> power-of-two scaled f16 rows for the down step
-      const int e = fi.e;
-      const int r0 = __ldg(p.offsets + e), r1 = r0 + __ldg(p.counts + e);
-      for (int rr = r0 + quad; rr < r1; rr += kTcEpiWarps) {
-        const float* gr = p.gu + (size_t)rr * 2 * p.I;
-        float amax = 0.f;
-        for (int f = lane; f < p.I; f += 32) {
-          const float gv = __ldcg(gr + f), uv = __ldcg(gr + p.I + f);
-          amax = fmaxf(amax, fabsf(gv / (1.f + expf(-gv)) * uv));
-        }
-        amax = warp_max(amax);
-        const float sc = pow2_scale_for(amax);
-        __half* hr = p.h16 + (size_t)rr * p.I;
-        for (int f = lane; f < p.I; f += 32) {
-          const float gv = __ldcg(gr + f), uv = __ldcg(gr + p.I + f);
-          hr[f] = __float2half_rn(gv / (1.f + expf(-gv)) * uv * sc);
-        }
-        if (lane == 0) p.hinv[rr] = 1.f / sc;
-      }
-    } else {
-      for (int c = et; c < 2 * kRowsHalf; c += kEpiThreads) {
-        const int col = fi.rt * 2 * kRowsHalf + c;
-        for (int tok = 0; tok < p.T; ++tok) {
-          float v = __ldcg(p.oacc + (size_t)tok * p.H + col);
-          if (p.residual) v += __bfloat162float(p.residual[(size_t)tok * p.H + col]);
-          p.out[(size_t)tok * p.H + col] = __float2bfloat16_rn(v);
-        }
-      }
-    }
   };
 
   long long cur_item = -1;
   ItemInfo inf{};
-  int done_in_item = 0;
   for (long long i = 0; i < nst; ++i) {
     const long long s = s_begin + i;
     const long long it = s / KB;
@@ -477,9 +422,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     if (it != cur_item) {
       cur_item = it;
       inf = decode_item(it, rtiles, s_cpre, nA, p, NT);
-      done_in_item = 0;
     }
-    ++done_in_item;
     float bs0 = 1.f, bs1 = 1.f;
     if (FMT == 1) {  // the FP8 block scales of this stage's two boxes
       const int KB128 = K / 128;
@@ -526,7 +469,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       }
     }
     const bool closes = (i + 1 == nst) || ((s + 1) / KB != it);
-    if (closes) flush(inf, done_in_item, dead);
+    if (closes) flush(inf, dead);
   }
   tc_fence_before();
   asm volatile("bar.sync 2, %0;" ::"n"(kTeardown) : "memory");

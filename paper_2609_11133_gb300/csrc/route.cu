@@ -269,8 +269,6 @@ __global__ void __launch_bounds__(256) route_kernel(const RouteParams p) {
     const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
     for (size_t i = tid; i < p.zero_a_n4; i += nthr) p.zero_a[i] = z;
     for (size_t i = tid; i < p.zero_b_n4; i += nthr) p.zero_b[i] = z;
-    for (size_t i = tid; i < (size_t)p.zero_c_n; i += nthr) p.zero_c[i] = 0u;
-    for (size_t i = tid; i < (size_t)p.zero_d_n; i += nthr) p.zero_d[i] = 0u;
   }
 
   // chunk ticket: the last of this chunk's expert blocks does the top-k
@@ -378,7 +376,6 @@ __global__ void __launch_bounds__(256) prep_kernel(const PrepParams p) {
     const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
     for (size_t i = tid; i < p.zero_a_n4; i += nthr) p.zero_a[i] = z;
     for (size_t i = tid; i < p.zero_b_n4; i += nthr) p.zero_b[i] = z;
-    for (size_t i = tid; i < (size_t)p.zero_c_n; i += nthr) p.zero_c[i] = 0u;
   }
   const int t = blockIdx.x * 8 + warp;
   if (t < p.T)

@@ -38,10 +38,6 @@ struct RouteParams {
   size_t zero_a_n4;
   float4* zero_b;
   size_t zero_b_n4;
-  unsigned* zero_c;
-  int zero_c_n;
-  unsigned* zero_d;
-  int zero_d_n;
   int* counts;
   int* offsets;
   int* sorted;
@@ -65,8 +61,6 @@ struct PrepParams {
   size_t zero_a_n4;
   float4* zero_b;
   size_t zero_b_n4;
-  unsigned* zero_c;
-  int zero_c_n;
 };
 
 struct CombineParams {
