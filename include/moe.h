@@ -171,6 +171,27 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
                         float* logits_out, int32_t* topk_ids_out, float* topk_w_out,
                         void* const* events, void* stream);
 
+/* moe_decode_layer without a caller-provided workspace, for callers that must
+ * not allocate device memory when they run the layer (for example an
+ * inference engine's plugin enqueue path, which gets a stream and its tensors
+ * but no allocator, or a serving loop that cannot afford a cudaMalloc that may
+ * synchronise the device).  The paper has no counterpart of this call.
+ *   Arguments as moe_decode_layer, minus ws / ws_bytes.
+ *   Scratch: a 16 MiB device array inside libmoe.so; every GPU that loads the
+ *     library holds it until the process exits.  Shapes whose
+ *     moe_workspace_size() exceeds 16 MiB return MOE_ERR_WORKSPACE_TOO_SMALL
+ *     (e.g. the 235B-shaped NVFP4 layer fits up to T = 113 tokens).
+ *   The first call on a device looks up the array's device address; make
+ *     that first call before capturing the stream into a CUDA graph.
+ *   Every call shares the one array and clears its control words itself;
+ *     calls that overlap on the GPU (two streams, or two host threads) race
+ *     and must be serialised by the caller.  Device-side error status is not
+ *     reported by this call.
+ *   Allocates nothing: no cudaMalloc, no cudaFree. */
+int moe_decode_layer_noalloc(const void* x, const float* router_w, const float* router_bias,
+                             const moe_expert_weights_t* w, int T, int k, int flags,
+                             const void* residual, void* out, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

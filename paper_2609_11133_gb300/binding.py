@@ -63,6 +63,8 @@ _SIGS = {
     "moe_combine": [_P, _P, _P, _I, _I, _I, _P, _P, _P],
     "moe_decode_layer": [_P, _P, _P, ctypes.POINTER(ExpertWeightsC), _I, _I, _I, _P, _P, _P,
                          _SZ, _P],
+    "moe_decode_layer_noalloc": [_P, _P, _P, ctypes.POINTER(ExpertWeightsC), _I, _I, _I, _P, _P,
+                                 _P],
     "moe_decode_layer_ex": [_P, _P, _P, ctypes.POINTER(ExpertWeightsC), _I, _I, _I, _P, _P, _P,
                             _SZ, _P, _P, _P, ctypes.POINTER(_P), _P],
 }
@@ -214,3 +216,15 @@ def moe_decode_layer_ex(x, router_w, router_bias, w, k: int, out, ws, flags: int
                                       _ptr(ws), ws.numel(), _ptr(logits_out), _ptr(topk_ids_out),
                                       _ptr(topk_w_out), ev, _stream(stream)),
            "moe_decode_layer_ex")
+
+
+def moe_decode_layer_noalloc(x, router_w, router_bias, w, k: int, out, flags: int = 0,
+                             residual=None, stream=None):
+    """The fused layer on the library's own 16 MiB scratch array (no workspace
+    argument, no allocation); for callers that may not allocate device memory."""
+    T = x.shape[0]
+    c = weights_struct(w)
+    _check(load().moe_decode_layer_noalloc(_ptr(x), _ptr(router_w), _ptr(router_bias),
+                                           ctypes.byref(c), T, k, flags, _ptr(residual),
+                                           _ptr(out), _stream(stream)),
+           "moe_decode_layer_noalloc")
