@@ -119,9 +119,10 @@ int nt_for(int T) {
     if (v == 16 || v == 32 || (v == 8 && !use_tc_engine())) return v;
   }
   if (use_tc_engine()) return T <= 16 ? 16 : 32;
-  // 16-token chunks keep five stages in flight; an expert with more tokens
-  // is processed in several chunks
-  return T <= 8 ? 8 : 16;
+  // 8-token chunks let the consumer warps hold a whole stage in registers and
+  // release it at once; at T <= 64 few experts get more than 8 tokens (those
+  // are processed in several chunks).  Larger batches use 32-token chunks.
+  return T <= 64 ? 8 : 32;
 }
 
 // ------------------------------------------------------------------ validation

@@ -17,7 +17,8 @@ constexpr int kMaxE = 512;          // experts per layer
 constexpr int kMaxTK = 65536;       // T * k
 constexpr int kMaxHI = 32768;       // H and I
 constexpr int kRouteTok = 8;        // tokens per router CTA
-constexpr int kRouteWarps = 8;      // warps per router CTA (one expert row each)
+constexpr int kRouteWarps = 8;      // warps per router CTA
+constexpr int kRouteEPB = 4;        // expert rows per router CTA (two warps each)
 
 // Device status bits (the first error wins; see moe_read_status).
 constexpr uint32_t kStatusTimeoutGateUp = 1u;

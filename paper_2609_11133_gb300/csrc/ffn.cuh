@@ -35,8 +35,11 @@
 
 namespace moe {
 
-constexpr int kFfnConsumerWarps = 8;
-constexpr int kFfnThreads = (kFfnConsumerWarps + 1) * 32;
+constexpr int kFfnMTiles = 8;  // 16-row MMA tiles per 128-row weight box
+// Consumer warps = kFfnMTiles * KS: with KS = 2 the two halves of each stage's
+// K range go to different warps, which doubles the warps that hide latency.
+template <int KS>
+constexpr int ffn_threads() { return (kFfnMTiles * KS + 1) * 32; }
 constexpr int kRowsHalf = 128;  // rows of each of the two weight boxes of a stage
 constexpr int kRowBytes = 128;  // weight bytes per row per stage
 
@@ -233,8 +236,8 @@ static __global__ void __launch_bounds__(256) finalize_kernel(const FfnParams p)
 }
 
 // ------------------------------------------------------------------ the kernel
-template <int FMT, int NT>
-__global__ void __launch_bounds__(kFfnThreads, 1)
+template <int FMT, int NT, int KS>
+__global__ void __launch_bounds__(ffn_threads<KS>(), 1)
     ffn_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmA1,
                const __grid_constant__ CUtensorMap tmS0, const __grid_constant__ CUtensorMap tmS1,
                const __grid_constant__ CUtensorMap tmB, const FfnParams p) {
@@ -254,7 +257,8 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
   __shared__ volatile int s_abort;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const bool is_producer = (warp == kFfnConsumerWarps);
+  constexpr int CW = kFfnMTiles * KS;  // consumer warps
+  const bool is_producer = (warp == CW);
 
   pdl_wait();
 
@@ -264,7 +268,7 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
     s_abort = 0;
     for (int i = 0; i < S; ++i) {
       mbar_init(&full_bar[i], 1);
-      mbar_init(&empty_bar[i], kFfnConsumerWarps);
+      mbar_init(&empty_bar[i], CW);
     }
     fence_mbar_init();
   }
@@ -355,7 +359,9 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
   // the order makes the two row groups of each quarter-warp differ in bit 2,
   // so the 128B-swizzled reads of a quarter-warp never share a bank.
   const int rho_g = ((g & 1) << 2) | (g >> 1);
-  const int ra = 16 * warp + rho_g, rb = ra + 8;
+  const int mtile = warp % kFfnMTiles;
+  const int khalf = warp / kFfnMTiles;  // KS = 2: which half of the stage's K
+  const int ra = 16 * mtile + rho_g, rb = ra + 8;
 
   float acc0[NTILE][4], acc1[NTILE][4];
   long long cur_item = -1;
@@ -422,7 +428,7 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
         for (int half = 0; half < 2; ++half) {
           const float v0 = acc0[n][c + 2 * half] * sc * ts0;
           const float v1 = acc1[n][c + 2 * half] * sc * ts1;
-          const int mrow = 16 * warp + rho_g + 8 * half;  // row within the 128-row box
+          const int mrow = 16 * mtile + rho_g + 8 * half;  // row within the 128-row box
           if (p.phase == 1) {
             const int f = inf.rt * kRowsHalf + mrow;
             float* base = p.gu + (size_t)dst * 2 * p.I;
@@ -486,47 +492,77 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
 #pragma unroll
       for (int i = 0; i < 4; ++i) tmp0[n][i] = tmp1[n][i] = 0.f;
 
+    // Load phase: this warp's share of the stage (weights, scales, token
+    // fragments) into registers.  With EARLY the slot is released right after,
+    // so the producer can refill it while the warp computes.
+    constexpr int HH = 2 / KS;                  // halves of the stage's K per warp
+    constexpr int NU = FmtTraits<FMT>::NU;
+    constexpr bool EARLY = (KS == 2 && NT == 8);
+    uint4 qa0[HH], qb0[HH], qa1[HH], qb1[HH];
+    uint32_t sa0[HH], sb0[HH], sa1[HH], sb1[HH];  // NVFP4 scale pairs (f16x2)
+    uint4 xb[HH][NU][NTILE];
 #pragma unroll
-    for (int h = 0; h < 2; ++h) {
+    for (int hh = 0; hh < HH; ++hh) {
+      const int h = (KS == 2) ? khalf : hh;
       const int c = 4 * h + t;  // 16-byte weight chunk of this thread
-      const uint4 qa0 = lds128(st + G::A0 + ra * kRowBytes + ((c ^ (ra & 7)) << 4));
-      const uint4 qb0 = lds128(st + G::A0 + rb * kRowBytes + ((c ^ (rb & 7)) << 4));
-      const uint4 qa1 = lds128(st + G::A1 + ra * kRowBytes + ((c ^ (ra & 7)) << 4));
-      const uint4 qb1 = lds128(st + G::A1 + rb * kRowBytes + ((c ^ (rb & 7)) << 4));
+      qa0[hh] = lds128(st + G::A0 + ra * kRowBytes + ((c ^ (ra & 7)) << 4));
+      qb0[hh] = lds128(st + G::A0 + rb * kRowBytes + ((c ^ (rb & 7)) << 4));
+      qa1[hh] = lds128(st + G::A1 + ra * kRowBytes + ((c ^ (ra & 7)) << 4));
+      qb1[hh] = lds128(st + G::A1 + rb * kRowBytes + ((c ^ (rb & 7)) << 4));
+      if (FMT == 2) {
+        sa0[hh] = lds16(st + G::S0 + ra * 16 + 2 * c);
+        sb0[hh] = lds16(st + G::S0 + rb * 16 + 2 * c);
+        sa1[hh] = lds16(st + G::S1 + ra * 16 + 2 * c);
+        sb1[hh] = lds16(st + G::S1 + rb * 16 + 2 * c);
+      }
+      if (EARLY) {
+#pragma unroll
+        for (int u = 0; u < NU; ++u)
+#pragma unroll
+          for (int n = 0; n < NTILE; ++n)
+            if (n < ntiles)
+              xb[hh][u][n] =
+                  lds128(st + G::B + (n * 8 + g) * G::BROW + (act_unit<FMT>(c * NU + u) << 4));
+      }
+    }
+    if (EARLY) {
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty_bar[slot]);
+    }
+
+#pragma unroll
+    for (int hh = 0; hh < HH; ++hh) {
+      const int c = 4 * ((KS == 2) ? khalf : hh) + t;
       // NVFP4: the two 16-element scales of this chunk per row, as f16x2
       // broadcasts {s, s} of the lower (k-steps 0-3) and upper (4-7) block
       uint32_t sa0lo = 0, sa0hi = 0, sb0lo = 0, sb0hi = 0;
       uint32_t sa1lo = 0, sa1hi = 0, sb1lo = 0, sb1hi = 0;
       if (FMT == 2) {
-        const uint32_t sa0 = e4m3x2_to_f16x2(lds16(st + G::S0 + ra * 16 + 2 * c));
-        const uint32_t sb0 = e4m3x2_to_f16x2(lds16(st + G::S0 + rb * 16 + 2 * c));
-        const uint32_t sa1 = e4m3x2_to_f16x2(lds16(st + G::S1 + ra * 16 + 2 * c));
-        const uint32_t sb1 = e4m3x2_to_f16x2(lds16(st + G::S1 + rb * 16 + 2 * c));
-        sa0lo = __byte_perm(sa0, 0, 0x1010);
-        sa0hi = __byte_perm(sa0, 0, 0x3232);
-        sb0lo = __byte_perm(sb0, 0, 0x1010);
-        sb0hi = __byte_perm(sb0, 0, 0x3232);
-        sa1lo = __byte_perm(sa1, 0, 0x1010);
-        sa1hi = __byte_perm(sa1, 0, 0x3232);
-        sb1lo = __byte_perm(sb1, 0, 0x1010);
-        sb1hi = __byte_perm(sb1, 0, 0x3232);
+        const uint32_t fa0 = e4m3x2_to_f16x2(sa0[hh]), fb0 = e4m3x2_to_f16x2(sb0[hh]);
+        const uint32_t fa1 = e4m3x2_to_f16x2(sa1[hh]), fb1 = e4m3x2_to_f16x2(sb1[hh]);
+        sa0lo = __byte_perm(fa0, 0, 0x1010);
+        sa0hi = __byte_perm(fa0, 0, 0x3232);
+        sb0lo = __byte_perm(fb0, 0, 0x1010);
+        sb0hi = __byte_perm(fb0, 0, 0x3232);
+        sa1lo = __byte_perm(fa1, 0, 0x1010);
+        sa1hi = __byte_perm(fa1, 0, 0x3232);
+        sb1lo = __byte_perm(fb1, 0, 0x1010);
+        sb1hi = __byte_perm(fb1, 0, 0x3232);
       }
-      const uint32_t wa0[4] = {qa0.x, qa0.y, qa0.z, qa0.w};
-      const uint32_t wb0[4] = {qb0.x, qb0.y, qb0.z, qb0.w};
-      const uint32_t wa1[4] = {qa1.x, qa1.y, qa1.z, qa1.w};
-      const uint32_t wb1[4] = {qb1.x, qb1.y, qb1.z, qb1.w};
-      constexpr int NU = FmtTraits<FMT>::NU;
+      const uint32_t wa0[4] = {qa0[hh].x, qa0[hh].y, qa0[hh].z, qa0[hh].w};
+      const uint32_t wb0[4] = {qb0[hh].x, qb0[hh].y, qb0[hh].z, qb0[hh].w};
+      const uint32_t wa1[4] = {qa1[hh].x, qa1[hh].y, qa1[hh].z, qa1[hh].w};
+      const uint32_t wb1[4] = {qb1[hh].x, qb1[hh].y, qb1[hh].z, qb1[hh].w};
 #pragma unroll
       for (int u = 0; u < NU; ++u) {
-        // activation fragments: 8 f16 = K positions P..P+7 of this thread
-        uint4 xb[NTILE];
+        // token fragments of this unit: 8 f16 = K positions P..P+7 of this thread
+        uint4 xu[NTILE];
 #pragma unroll
         for (int n = 0; n < NTILE; ++n) {
-          if (n < ntiles) {
-            const int row = n * 8 + g;
-            const int U = c * NU + u;
-            xb[n] = lds128(st + G::B + row * G::BROW + (act_unit<FMT>(U) << 4));
-          }
+          if (n < ntiles)
+            xu[n] = EARLY ? xb[hh][u][n]
+                          : lds128(st + G::B + (n * 8 + g) * G::BROW +
+                                   (act_unit<FMT>(c * NU + u) << 4));
         }
         // weights of the two k-steps of this unit: FP8 uses one 32-bit word
         // (4 codes) per row per k-step, NVFP4 one word (8 codes) per row per 2 k-steps
@@ -569,8 +605,8 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
 #pragma unroll
           for (int n = 0; n < NTILE; ++n) {
             if (n < ntiles) {
-              const uint32_t b0 = ss ? xb[n].z : xb[n].x;
-              const uint32_t b1 = ss ? xb[n].w : xb[n].y;
+              const uint32_t b0 = ss ? xu[n].z : xu[n].x;
+              const uint32_t b1 = ss ? xu[n].w : xu[n].y;
               mma_f16(tmp0[n], A0r[0], A0r[1], A0r[2], A0r[3], b0, b1);
               mma_f16(tmp1[n], A1r[0], A1r[1], A1r[2], A1r[3], b0, b1);
             }
@@ -578,8 +614,10 @@ __global__ void __launch_bounds__(kFfnThreads, 1)
         }
       }
     }
-    __syncwarp();
-    if (lane == 0) mbar_arrive(&empty_bar[slot]);
+    if (!EARLY) {
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty_bar[slot]);
+    }
 #pragma unroll
     for (int n = 0; n < NTILE; ++n)
 #pragma unroll

@@ -34,14 +34,15 @@ cudaError_t launch_ffn_tc(int nt, int grid, const FfnMaps& maps, const FfnParams
   template <int NT>                                                                             \
   static cudaError_t launch_ffn_nt_##FMTV(int grid, const FfnMaps& m, const FfnParams& p,      \
                                           cudaStream_t st, bool pdl) {                          \
-    auto kern = ffn_kernel<FMTV, NT>;                                                           \
+    constexpr int KS = (NT == 32) ? 1 : 2;                                                      \
+    auto kern = ffn_kernel<FMTV, NT, KS>;                                                       \
     const int smem = StageGeom<FMTV, NT>::SMEM;                                                 \
     cudaError_t err =                                                                           \
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);          \
     if (err != cudaSuccess) return err;                                                         \
     cudaLaunchConfig_t cfg = {};                                                                \
     cfg.gridDim = dim3(grid);                                                                   \
-    cfg.blockDim = dim3(kFfnThreads);                                                           \
+    cfg.blockDim = dim3(ffn_threads<KS>());                                                     \
     cfg.dynamicSmemBytes = smem;                                                                \
     cfg.stream = st;                                                                            \
     cudaLaunchAttribute attr[1];                                                                \

@@ -219,8 +219,12 @@ __global__ void __launch_bounds__(256) route_kernel(const RouteParams p) {
                          lane, p.unit_perm != 0);
   }
 
-  // router GEMV: warp -> expert row, lanes -> 4 consecutive h per 128
-  const int e = eb * kRouteWarps + warp;
+  // router GEMV: two warps per expert row (one half of H each), lanes -> 4
+  // consecutive h per 128; the halves meet in shared memory
+  __shared__ float s_part[kRouteWarps][kRouteTok];
+  const int e = eb * kRouteEPB + (warp >> 1);
+  const int hhalf = H / 2;
+  const int hbeg = (warp & 1) * hhalf;
   if (e < E) {
     float acc[kRouteTok];
 #pragma unroll
@@ -228,38 +232,42 @@ __global__ void __launch_bounds__(256) route_kernel(const RouteParams p) {
     const float* wrow = p.wr + (size_t)e * H;
     // 16 router loads in flight per lane before any is used
     constexpr int DEPTH = 16;
-    for (int h0 = lane * 4; h0 < H; h0 += 128 * DEPTH) {
+    for (int h0 = hbeg + lane * 4; h0 < hbeg + hhalf; h0 += 128 * DEPTH) {
       float4 w[DEPTH];
 #pragma unroll
       for (int q = 0; q < DEPTH; ++q)
-        w[q] = (h0 + 128 * q < H) ? __ldg(reinterpret_cast<const float4*>(wrow + h0 + 128 * q))
-                                  : make_float4(0.f, 0.f, 0.f, 0.f);
+        w[q] = (h0 + 128 * q < hbeg + hhalf)
+                   ? __ldg(reinterpret_cast<const float4*>(wrow + h0 + 128 * q))
+                   : make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
       for (int q = 0; q < DEPTH; ++q) {
         const int h = h0 + 128 * q;
-        if (h >= H) break;
+        if (h >= hbeg + hhalf) break;
 #pragma unroll
         for (int t = 0; t < kRouteTok; ++t) {
           if (t < nt) {
             const uint2 xv = *reinterpret_cast<const uint2*>(xs + (size_t)t * H + h);
             const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&xv.x));
             const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&xv.y));
-            float s = acc[t];
-            s = fmaf(a.x, w[q].x, s);
-            s = fmaf(a.y, w[q].y, s);
-            s = fmaf(b.x, w[q].z, s);
-            s = fmaf(b.y, w[q].w, s);
-            acc[t] = s;
+            float sacc = acc[t];
+            sacc = fmaf(a.x, w[q].x, sacc);
+            sacc = fmaf(a.y, w[q].y, sacc);
+            sacc = fmaf(b.x, w[q].z, sacc);
+            sacc = fmaf(b.y, w[q].w, sacc);
+            acc[t] = sacc;
           }
         }
       }
     }
 #pragma unroll
     for (int t = 0; t < kRouteTok; ++t) acc[t] = warp_sum(acc[t]);
-    if (lane == 0) {
-      const float b = p.bias ? __ldg(p.bias + e) : 0.f;
-      for (int t = 0; t < nt; ++t) p.logits[(size_t)(t0 + t) * E + e] = acc[t] + b;
-    }
+    if (lane == 0)
+      for (int t = 0; t < kRouteTok; ++t) s_part[warp][t] = acc[t];
+  }
+  __syncthreads();
+  if (e < E && (warp & 1) == 0 && lane < nt) {
+    const float b = p.bias ? __ldg(p.bias + e) : 0.f;
+    p.logits[(size_t)(t0 + lane) * E + e] = (s_part[warp][lane] + s_part[warp + 1][lane]) + b;
   }
 
   // accumulators and counters of the later kernels start from zero
@@ -459,7 +467,7 @@ cudaError_t launch_route(const RouteParams& p, cudaStream_t st) {
   cudaError_t err =
       cudaFuncSetAttribute(route_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (err != cudaSuccess) return err;
-  dim3 grid((p.E + kRouteWarps - 1) / kRouteWarps, (p.T + kRouteTok - 1) / kRouteTok);
+  dim3 grid((p.E + kRouteEPB - 1) / kRouteEPB, (p.T + kRouteTok - 1) / kRouteTok);
   route_kernel<<<grid, 256, smem, st>>>(p);
   return cudaGetLastError();
 }

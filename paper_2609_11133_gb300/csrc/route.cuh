@@ -1,10 +1,10 @@
 // Router, top-k, permutation and small elementwise kernels of the MoE decode
 // layer.
 //
-// route_kernel (grid = [ceil(E/8) expert blocks, ceil(T/8) token chunks]):
+// route_kernel (grid = [ceil(E/4) expert blocks, ceil(T/8) token chunks]):
 //   every CTA stages 8 token rows of x in shared memory and computes the fp32
-//   logits of 8 experts (one warp per expert row of the router, float4 loads,
-//   shuffle reduction).  The CTA that arrives last at a chunk's ticket does
+//   logits of 4 experts (two warps per expert row of the router, one half of
+//   H each, float4 loads, shuffle reduction).  The CTA that arrives last at a chunk's ticket does
 //   the softmax/top-k of those 8 tokens (one warp per token, k rounds of a
 //   warp arg-max with ties to the lower index); in the fused layer the CTA
 //   that completes the last chunk builds the token->expert permutation and
