@@ -241,8 +241,8 @@ int run_experts(const ExpertRun& r, cudaStream_t st, cudaEvent_t ev_mid) {
   auto launch = [&](const FfnMaps& m, const FfnParams& pp) {
     if (tc)
       return fp4 ? launch_ffn_tc<2>(r.nt, r.sms, m, pp, st) : launch_ffn_tc<1>(r.nt, r.sms, m, pp, st);
-    return fp4 ? launch_ffn<2>(r.nt, r.sms, m, pp, st, false)
-               : launch_ffn<1>(r.nt, r.sms, m, pp, st, false);
+    return fp4 ? launch_ffn<2>(r.nt, r.sms, m, pp, st, true)
+               : launch_ffn<1>(r.nt, r.sms, m, pp, st, true);
   };
   cudaError_t err = launch(m1, p1);
   if (err != cudaSuccess) return MOE_ERR_CUDA;

@@ -156,6 +156,7 @@ __global__ void __launch_bounds__(256) swiglu_kernel(const FfnParams p, int rows
   const int gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int nw = (gridDim.x * blockDim.x) >> 5;
   pdl_wait();
+  pdl_launch_dependents();
   const int n4 = p.I / 4;
   constexpr int D = 4;
   for (int row = gw; row < rows; row += nw) {
@@ -260,10 +261,6 @@ __global__ void __launch_bounds__(ffn_threads<KS>(), 1)
   constexpr int CW = kFfnMTiles * KS;  // consumer warps
   const bool is_producer = (warp == CW);
 
-  pdl_wait();
-
-  const int nA = __ldg(p.active);
-  for (int i = threadIdx.x; i <= nA; i += blockDim.x) s_cpre[i] = __ldg(p.cprefix + i);
   if (threadIdx.x == 0) {
     s_abort = 0;
     for (int i = 0; i < S; ++i) {
@@ -272,6 +269,12 @@ __global__ void __launch_bounds__(ffn_threads<KS>(), 1)
     }
     fence_mbar_init();
   }
+  // Launched as a programmatic dependent: everything above overlapped the
+  // previous kernel; from here on its outputs are read.
+  pdl_wait();
+  pdl_launch_dependents();
+  const int nA = __ldg(p.active);
+  for (int i = threadIdx.x; i <= nA; i += blockDim.x) s_cpre[i] = __ldg(p.cprefix + i);
   __syncthreads();
 
   const int N = (p.phase == 1) ? p.I : p.H;       // rows of one expert matrix

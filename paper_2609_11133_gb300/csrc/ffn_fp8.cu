@@ -9,7 +9,6 @@ cudaError_t launch_finalize(int sms, const FfnParams& p, cudaStream_t st) {
   size_t blocks = ((size_t)p.T * p.H / 4 + 255) / 256;
   if (blocks > (size_t)(4 * sms)) blocks = 4 * sms;
   if (blocks < 1) blocks = 1;
-  finalize_kernel<<<(unsigned)blocks, 256, 0, st>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(finalize_kernel, dim3((unsigned)blocks), dim3(256), 0, st, p);
 }
 }  // namespace moe

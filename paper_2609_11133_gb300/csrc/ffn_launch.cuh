@@ -7,6 +7,25 @@
 
 namespace moe {
 
+// Launch `kern` as a programmatic dependent of the previous kernel on the
+// stream (its blocks may start while that kernel finishes; the kernel calls
+// griddepcontrol.wait before reading what the previous kernel wrote).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t st, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
 struct FfnMaps {
   CUtensorMap a0, a1, s0, s1, b;
 };
@@ -79,8 +98,8 @@ cudaError_t launch_ffn_tc(int nt, int grid, const FfnMaps& maps, const FfnParams
     int blocks = (rows + 7) / 8;                                                                \
     if (blocks > 4 * sms) blocks = 4 * sms;                                                     \
     if (blocks < 1) blocks = 1;                                                                 \
-    swiglu_kernel<FMTV><<<blocks, 256, 0, st>>>(p, rows, perm ? 1 : 0);                         \
-    return cudaGetLastError();                                                                  \
+    return launch_pdl(swiglu_kernel<FMTV>, dim3(blocks), dim3(256), 0, st, p, rows,            \
+                      perm ? 1 : 0);                                                            \
   }
 
 #define MOE_DEFINE_FFN_TC_LAUNCH(FMTV)                                                         \
@@ -92,8 +111,8 @@ cudaError_t launch_ffn_tc(int nt, int grid, const FfnMaps& maps, const FfnParams
     cudaError_t err =                                                                           \
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);          \
     if (err != cudaSuccess) return err;                                                         \
-    kern<<<grid, kTcThreads, smem, st>>>(m.a0, m.a1, m.s0, m.s1, m.b, p);                       \
-    return cudaGetLastError();                                                                  \
+    return launch_pdl(kern, dim3(grid), dim3(kTcThreads), smem, st, m.a0, m.a1, m.s0, m.s1,   \
+                      m.b, p);                                                                  \
   }                                                                                             \
   template <>                                                                                   \
   cudaError_t launch_ffn_tc<FMTV>(int nt, int grid, const FfnMaps& m, const FfnParams& p,      \

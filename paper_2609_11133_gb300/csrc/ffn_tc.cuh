@@ -87,10 +87,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-  pdl_wait();
-
-  const int nA = __ldg(p.active);
-  for (int i = threadIdx.x; i <= nA; i += blockDim.x) s_cpre[i] = __ldg(p.cprefix + i);
   if (threadIdx.x == 0) {
     s_abort = 0;
     for (int i = 0; i < S; ++i) {
@@ -112,6 +108,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     tmem_alloc(&s_tmem, kTmemCols);
     tmem_relinquish();
   }
+  // Launched as a programmatic dependent: everything above overlapped the
+  // previous kernel; from here on its outputs are read.
+  pdl_wait();
+  pdl_launch_dependents();
+  const int nA = __ldg(p.active);
+  for (int i = threadIdx.x; i <= nA; i += blockDim.x) s_cpre[i] = __ldg(p.cprefix + i);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();

@@ -173,6 +173,7 @@ __global__ void __launch_bounds__(256) route_kernel(const RouteParams p) {
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int chunk = blockIdx.y, eb = blockIdx.x;
+  pdl_launch_dependents();  // the expert kernel may start its prologue now
   const int t0 = chunk * kRouteTok;
   const int nt = min(kRouteTok, p.T - t0);
   const int H = p.H, E = p.E;
@@ -294,24 +295,34 @@ __global__ void __launch_bounds__(256) route_kernel(const RouteParams p) {
   if (warp < nt) {
     const int t = t0 + warp;
     constexpr int PER = kMaxE / 32;
+    const int per = (E + 31) / 32;  // logits held by each lane
     float v[PER];
 #pragma unroll
     for (int i = 0; i < PER; ++i) {
       const int ee = lane + 32 * i;
-      v[i] = (ee < E) ? __ldcg(p.logits + (size_t)t * E + ee) : -INFINITY;
+      v[i] = (i < per && ee < E) ? __ldcg(p.logits + (size_t)t * E + ee) : -INFINITY;
     }
+    // Each lane keeps the best of its own untaken logits; a round takes the
+    // warp's best (value desc, index asc) and only the winning lane rescans.
     unsigned taken = 0u;
-    for (int j = 0; j < p.k; ++j) {
-      float bv = -INFINITY;
-      int bi = 0x7fffffff;
+    float lbv;
+    int lbi;
+    auto local_best = [&]() {
+      lbv = -INFINITY;
+      lbi = 0x7fffffff;
 #pragma unroll
       for (int i = 0; i < PER; ++i) {
         const int ee = lane + 32 * i;
-        if (ee < E && !((taken >> i) & 1u) && (v[i] > bv || (v[i] == bv && ee < bi))) {
-          bv = v[i];
-          bi = ee;
+        if (i < per && ee < E && !((taken >> i) & 1u) && (v[i] > lbv || (v[i] == lbv && ee < lbi))) {
+          lbv = v[i];
+          lbi = ee;
         }
       }
+    };
+    local_best();
+    for (int j = 0; j < p.k; ++j) {
+      float bv = lbv;
+      int bi = lbi;
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) {
         const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
@@ -321,7 +332,10 @@ __global__ void __launch_bounds__(256) route_kernel(const RouteParams p) {
           bi = oi;
         }
       }
-      if ((bi & 31) == lane) taken |= 1u << (bi >> 5);
+      if ((bi & 31) == lane) {
+        taken |= 1u << (bi >> 5);
+        local_best();
+      }
       if (lane == 0) {
         s_sel[warp][j] = bi;
         s_selv[warp][j] = bv;
@@ -378,6 +392,7 @@ __global__ void __launch_bounds__(256) permute_kernel(const int* ids, int T, int
 // Activation conversion, zeroing and work plan for the unfused expert FFN.
 __global__ void __launch_bounds__(256) prep_kernel(const PrepParams p) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  pdl_launch_dependents();
   {
     const size_t nthr = (size_t)gridDim.x * blockDim.x;
     const size_t tid = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
