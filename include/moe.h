@@ -43,7 +43,7 @@
  *   W = e2m1(code) * e4m3(scale) * ts.
  *
  * Supported shapes: H % 256 == 0; I % 128 == 0 (FP8) or I % 256 == 0
- * (NVFP4); 1 <= k <= E <= 512; 0 <= T; T*k <= 65536; H, I <= 32768.
+ * (NVFP4); 1 <= k <= min(E, 32); E <= 512; 0 <= T; T*k <= 65536; H, I <= 8192.
  * T == 0 is a no-op.  Anything else returns MOE_ERR_UNSUPPORTED_SHAPE.
  */
 #ifndef MOE_H_

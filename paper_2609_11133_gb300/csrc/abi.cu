@@ -136,7 +136,7 @@ int check_weights(const moe_expert_weights_t* w) {
   if (w->E < 1 || w->E > kMaxE) return MOE_ERR_UNSUPPORTED_SHAPE;
   if (w->H < 256 || w->H > 8192 || w->H % 256) return MOE_ERR_UNSUPPORTED_SHAPE;
   const int imod = (w->fmt == MOE_FMT_FP8_B128) ? 128 : 256;
-  if (w->I < imod || w->I > 16384 || w->I % imod) return MOE_ERR_UNSUPPORTED_SHAPE;
+  if (w->I < imod || w->I > 8192 || w->I % imod) return MOE_ERR_UNSUPPORTED_SHAPE;
   if (!aligned(w->w_gate, 16) || !aligned(w->w_up, 16) || !aligned(w->w_down, 16))
     return MOE_ERR_INVALID_ARG;
   const size_t sa = (w->fmt == MOE_FMT_NVFP4) ? 16 : 4;

@@ -10,6 +10,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+
 namespace moe {
 
 // ------------------------------------------------------------------ limits
@@ -89,6 +91,21 @@ inline WsLayout ws_layout(int T, int k, int E, int H, int I) {
   L.oacc = take(4 * (size_t)T * H);
   L.total = o;
   return L;
+}
+
+// Raise a kernel's dynamic shared-memory limit once per device (the call is a
+// host-side attribute change; doing it once keeps it out of graph captures
+// and off the per-call path).  `mask` is one bit per device, per kernel.
+template <typename K>
+inline cudaError_t set_smem_once(K kern, int bytes, std::atomic<unsigned long long>& mask) {
+  int dev = 0;
+  cudaError_t err = cudaGetDevice(&dev);
+  if (err != cudaSuccess) return err;
+  const unsigned long long bit = 1ull << (dev & 63);
+  if (mask.load(std::memory_order_acquire) & bit) return cudaSuccess;
+  err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (err == cudaSuccess) mask.fetch_or(bit, std::memory_order_acq_rel);
+  return err;
 }
 
 template <typename Ty>

@@ -148,66 +148,59 @@ __device__ __forceinline__ ItemInfo decode_item(long long it, int rtiles, const 
 // ------------------------------------------------------------------ between and after the phases
 // SwiGLU of every assignment row: h = silu(g) * u from the fp32 gate|up
 // accumulators, scaled per row by a power of two into f16 (in the unit order
-// of the warp-MMA NVFP4 layout when `perm`).  One warp per row; every lane
-// issues its 16-byte loads in batches of four before using them.
+// of the warp-MMA NVFP4 layout when `perm`).  One CTA per row: every thread
+// loads its share of the row once (up to 8 groups of 4 columns, I <= 8192),
+// the row maximum comes from a shared-memory reduction, and the scaled values
+// are written from registers - two memory latencies per row.
 template <int FMT>
 __global__ void __launch_bounds__(256) swiglu_kernel(const FfnParams p, int rows, int perm) {
-  const int lane = threadIdx.x & 31;
-  const int gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int nw = (gridDim.x * blockDim.x) >> 5;
+  constexpr int G = 8;  // float4 groups per thread
+  __shared__ float s_max[8];
   pdl_wait();
   pdl_launch_dependents();
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int n4 = p.I / 4;
-  constexpr int D = 4;
-  for (int row = gw; row < rows; row += nw) {
+  for (int row = blockIdx.x; row < rows; row += gridDim.x) {
     const float4* g4 = reinterpret_cast<const float4*>(p.gu + (size_t)row * 2 * p.I);
     const float4* u4 = reinterpret_cast<const float4*>(p.gu + (size_t)row * 2 * p.I + p.I);
+    float4 hv[G];
     float amax = 0.f;
-    for (int base = lane; base < n4; base += 32 * D) {
-      float4 gv[D], uv[D];
 #pragma unroll
-      for (int q = 0; q < D; ++q)
-        if (base + 32 * q < n4) {
-          gv[q] = __ldcg(g4 + base + 32 * q);
-          uv[q] = __ldcg(u4 + base + 32 * q);
-        }
-#pragma unroll
-      for (int q = 0; q < D; ++q)
-        if (base + 32 * q < n4) {
-          amax = fmaxf(amax, fabsf(gv[q].x / (1.f + expf(-gv[q].x)) * uv[q].x));
-          amax = fmaxf(amax, fabsf(gv[q].y / (1.f + expf(-gv[q].y)) * uv[q].y));
-          amax = fmaxf(amax, fabsf(gv[q].z / (1.f + expf(-gv[q].z)) * uv[q].z));
-          amax = fmaxf(amax, fabsf(gv[q].w / (1.f + expf(-gv[q].w)) * uv[q].w));
-        }
-    }
-    amax = warp_max(amax);
-    const float sc = pow2_scale_for(amax);
-    __half* hr = p.h16 + (size_t)row * p.I;
-    for (int base = lane; base < n4; base += 32 * D) {
-      float4 gv[D], uv[D];
-#pragma unroll
-      for (int q = 0; q < D; ++q)
-        if (base + 32 * q < n4) {
-          gv[q] = __ldcg(g4 + base + 32 * q);
-          uv[q] = __ldcg(u4 + base + 32 * q);
-        }
-#pragma unroll
-      for (int q = 0; q < D; ++q) {
-        const int i = base + 32 * q;
-        if (i < n4) {
-          const __half2 lo = __floats2half2_rn(gv[q].x / (1.f + expf(-gv[q].x)) * uv[q].x * sc,
-                                               gv[q].y / (1.f + expf(-gv[q].y)) * uv[q].y * sc);
-          const __half2 hi = __floats2half2_rn(gv[q].z / (1.f + expf(-gv[q].z)) * uv[q].z * sc,
-                                               gv[q].w / (1.f + expf(-gv[q].w)) * uv[q].w * sc);
-          uint2 o;
-          o.x = *reinterpret_cast<const uint32_t*>(&lo);
-          o.y = *reinterpret_cast<const uint32_t*>(&hi);
-          const int f = 4 * i;  // 4 consecutive columns stay inside one 16-byte unit
-          *reinterpret_cast<uint2*>(hr + (perm ? act_pos<FMT>(f) : f)) = o;
-        }
+    for (int q = 0; q < G; ++q) {
+      const int i = threadIdx.x + 256 * q;
+      if (i < n4) {
+        const float4 gv = __ldcg(g4 + i), uv = __ldcg(u4 + i);
+        hv[q].x = gv.x / (1.f + expf(-gv.x)) * uv.x;
+        hv[q].y = gv.y / (1.f + expf(-gv.y)) * uv.y;
+        hv[q].z = gv.z / (1.f + expf(-gv.z)) * uv.z;
+        hv[q].w = gv.w / (1.f + expf(-gv.w)) * uv.w;
+        amax = fmaxf(amax, fmaxf(fmaxf(fabsf(hv[q].x), fabsf(hv[q].y)),
+                                 fmaxf(fabsf(hv[q].z), fabsf(hv[q].w))));
       }
     }
-    if (lane == 0) p.hinv[row] = 1.f / sc;
+    amax = warp_max(amax);
+    if (lane == 0) s_max[warp] = amax;
+    __syncthreads();
+    amax = s_max[0];
+#pragma unroll
+    for (int w = 1; w < 8; ++w) amax = fmaxf(amax, s_max[w]);
+    const float sc = pow2_scale_for(amax);
+    __half* hr = p.h16 + (size_t)row * p.I;
+#pragma unroll
+    for (int q = 0; q < G; ++q) {
+      const int i = threadIdx.x + 256 * q;
+      if (i < n4) {
+        const __half2 lo = __floats2half2_rn(hv[q].x * sc, hv[q].y * sc);
+        const __half2 hi = __floats2half2_rn(hv[q].z * sc, hv[q].w * sc);
+        uint2 o;
+        o.x = *reinterpret_cast<const uint32_t*>(&lo);
+        o.y = *reinterpret_cast<const uint32_t*>(&hi);
+        const int f = 4 * i;  // 4 consecutive columns stay inside one 16-byte unit
+        *reinterpret_cast<uint2*>(hr + (perm ? act_pos<FMT>(f) : f)) = o;
+      }
+    }
+    if (threadIdx.x == 0) p.hinv[row] = 1.f / sc;
+    __syncthreads();  // s_max is reused by the next row
   }
 }
 

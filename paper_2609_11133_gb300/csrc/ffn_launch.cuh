@@ -56,8 +56,8 @@ cudaError_t launch_ffn_tc(int nt, int grid, const FfnMaps& maps, const FfnParams
     constexpr int KS = (NT == 32) ? 1 : 2;                                                      \
     auto kern = ffn_kernel<FMTV, NT, KS>;                                                       \
     const int smem = StageGeom<FMTV, NT>::SMEM;                                                 \
-    cudaError_t err =                                                                           \
-        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);          \
+    static std::atomic<unsigned long long> done{0};                                             \
+    cudaError_t err = set_smem_once(kern, smem, done);                                          \
     if (err != cudaSuccess) return err;                                                         \
     cudaLaunchConfig_t cfg = {};                                                                \
     cfg.gridDim = dim3(grid);                                                                   \
@@ -95,8 +95,8 @@ cudaError_t launch_ffn_tc(int nt, int grid, const FfnMaps& maps, const FfnParams
   template <>                                                                                   \
   cudaError_t launch_swiglu<FMTV>(int rows, int sms, const FfnParams& p, bool perm,            \
                                   cudaStream_t st) {                                            \
-    int blocks = (rows + 7) / 8;                                                                \
-    if (blocks > 4 * sms) blocks = 4 * sms;                                                     \
+    int blocks = rows;                                                                          \
+    if (blocks > 8 * sms) blocks = 8 * sms;                                                     \
     if (blocks < 1) blocks = 1;                                                                 \
     return launch_pdl(swiglu_kernel<FMTV>, dim3(blocks), dim3(256), 0, st, p, rows,            \
                       perm ? 1 : 0);                                                            \
@@ -108,8 +108,8 @@ cudaError_t launch_ffn_tc(int nt, int grid, const FfnMaps& maps, const FfnParams
                                              cudaStream_t st) {                                 \
     auto kern = ffn_tc_kernel<FMTV, NT>;                                                        \
     const int smem = TcGeom<FMTV, NT>::SMEM;                                                    \
-    cudaError_t err =                                                                           \
-        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);          \
+    static std::atomic<unsigned long long> done{0};                                             \
+    cudaError_t err = set_smem_once(kern, smem, done);                                          \
     if (err != cudaSuccess) return err;                                                         \
     return launch_pdl(kern, dim3(grid), dim3(kTcThreads), smem, st, m.a0, m.a1, m.s0, m.s1,   \
                       m.b, p);                                                                  \

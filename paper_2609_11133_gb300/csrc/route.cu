@@ -64,6 +64,12 @@ __device__ __forceinline__ unsigned lanemask_lt() {
 // warp each, match_any per 32), the per-segment counts are prefix-summed per
 // expert, and every assignment is placed at offsets[e] + its stable rank.
 // cw: shared scratch of 8*E + 2*(E+1) ints.
+template <bool IDS_SHARED>
+__device__ __forceinline__ int load_id(const int* ids, int a) {
+  return IDS_SHARED ? ids[a] : __ldcg(ids + a);
+}
+
+template <bool IDS_SHARED>
 __device__ void permute_plan(const int* ids, int T, int k, int E, int nt, int* counts,
                              int* offsets, int* sorted, int* inv, int* active, int* cprefix,
                              uint32_t* status, int* cw) {
@@ -81,7 +87,7 @@ __device__ void permute_plan(const int* ids, int T, int k, int E, int nt, int* c
       const int a = base + lane;
       int e = -1;
       if (a < a_hi) {
-        e = __ldcg(ids + a);
+        e = load_id<IDS_SHARED>(ids, a);
         if (e < 0 || e >= E) {
           e = -1;
           *s_bad = 1;
@@ -153,7 +159,7 @@ __device__ void permute_plan(const int* ids, int T, int k, int E, int nt, int* c
   }
   __syncthreads();
   for (int a = threadIdx.x; a < A; a += blockDim.x) {
-    const int e = __ldcg(ids + a);
+    const int e = load_id<IDS_SHARED>(ids, a);
     if (e < 0 || e >= E) continue;
     const int w = a / seg;
     const int pos = s_off[e] + cw[w * E + e] + inv[a];
@@ -168,7 +174,7 @@ __global__ void __launch_bounds__(256) route_kernel(const RouteParams p) {
   extern __shared__ __align__(16) unsigned char route_smem[];
   __nv_bfloat16* xs = reinterpret_cast<__nv_bfloat16*>(route_smem);
   __shared__ int s_flag;
-  __shared__ int s_sel[kRouteWarps][kMaxK];
+  __shared__ int s_sel[kRouteWarps][kMaxK];  // top-k of the chunk's tokens, by warp
   __shared__ float s_selv[kRouteWarps][kMaxK];
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -363,6 +369,17 @@ __global__ void __launch_bounds__(256) route_kernel(const RouteParams p) {
     }
   }
   if (!p.fused) return;
+  if (gridDim.y == 1) {
+    // a single token chunk: this CTA already holds every id (s_sel, warp t =
+    // token t) and builds the permutation without another ticket
+    __syncthreads();
+    int* s_ids = reinterpret_cast<int*>(route_smem);  // [T*k], ahead of the scratch
+    for (int a = threadIdx.x; a < p.T * p.k; a += blockDim.x) s_ids[a] = s_sel[a / p.k][a % p.k];
+    __syncthreads();
+    permute_plan<true>(s_ids, p.T, p.k, E, p.nt, p.counts, p.offsets, p.sorted, p.inv, p.active,
+                       p.cprefix, p.status, s_ids + kRouteTok * kMaxK);
+    return;
+  }
 
   // chunk-completion ticket: the last chunk builds the permutation and plan
   __threadfence();
@@ -375,8 +392,8 @@ __global__ void __launch_bounds__(256) route_kernel(const RouteParams p) {
   __syncthreads();
   if (!s_flag) return;
   __threadfence();
-  permute_plan(p.ids, p.T, p.k, E, p.nt, p.counts, p.offsets, p.sorted, p.inv, p.active,
-               p.cprefix, p.status, reinterpret_cast<int*>(route_smem));
+  permute_plan<false>(p.ids, p.T, p.k, E, p.nt, p.counts, p.offsets, p.sorted, p.inv, p.active,
+                      p.cprefix, p.status, reinterpret_cast<int*>(route_smem));
 }
 
 __global__ void __launch_bounds__(256) permute_kernel(const int* ids, int T, int k, int E,
@@ -385,8 +402,8 @@ __global__ void __launch_bounds__(256) permute_kernel(const int* ids, int T, int
   extern __shared__ __align__(16) unsigned char route_smem[];
   int* cw = reinterpret_cast<int*>(route_smem);
   int* cprefix_scratch = cw + 8 * E + 2 * (E + 1);  // the standalone call has no plan output
-  permute_plan(ids, T, k, E, 32, counts, offsets, sorted, inv, active, cprefix_scratch, nullptr,
-               cw);
+  permute_plan<false>(ids, T, k, E, 32, counts, offsets, sorted, inv, active, cprefix_scratch,
+                      nullptr, cw);
 }
 
 // Activation conversion, zeroing and work plan for the unfused expert FFN.
@@ -473,14 +490,15 @@ __global__ void __launch_bounds__(256) combine_kernel(const CombineParams p) {
 // ------------------------------------------------------------------ launchers
 size_t route_smem_bytes(int H, int E) {
   const size_t xs = (size_t)kRouteTok * H * 2;
-  const size_t perm = sizeof(int) * (size_t)(8 * E + 2 * (E + 1));
+  const size_t perm = sizeof(int) * (size_t)(kRouteTok * kMaxK + 8 * E + 2 * (E + 1));
   return xs > perm ? xs : perm;
 }
 
 cudaError_t launch_route(const RouteParams& p, cudaStream_t st) {
+  // the largest dynamic size any call can ask for (H <= 8192, E <= 512)
+  static std::atomic<unsigned long long> done{0};
   const size_t smem = route_smem_bytes(p.H, p.E);
-  cudaError_t err =
-      cudaFuncSetAttribute(route_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  cudaError_t err = set_smem_once(route_kernel, (int)route_smem_bytes(8192, kMaxE), done);
   if (err != cudaSuccess) return err;
   dim3 grid((p.E + kRouteEPB - 1) / kRouteEPB, (p.T + kRouteTok - 1) / kRouteTok);
   route_kernel<<<grid, 256, smem, st>>>(p);
@@ -490,9 +508,10 @@ cudaError_t launch_route(const RouteParams& p, cudaStream_t st) {
 cudaError_t launch_permute_standalone(const int* ids, int T, int k, int E, int* counts,
                                       int* offsets, int* sorted, int* inv, int* active,
                                       cudaStream_t st) {
+  static std::atomic<unsigned long long> done{0};
   const size_t smem = sizeof(int) * (size_t)(8 * E + 3 * (E + 1));
   cudaError_t err =
-      cudaFuncSetAttribute(permute_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      set_smem_once(permute_kernel, (int)(sizeof(int) * (size_t)(8 * kMaxE + 3 * (kMaxE + 1))), done);
   if (err != cudaSuccess) return err;
   permute_kernel<<<1, 256, smem, st>>>(ids, T, k, E, counts, offsets, sorted, inv, active);
   return cudaGetLastError();
