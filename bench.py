@@ -3,14 +3,26 @@
 python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
                 [--workload NAME] [--tokens T]
 
-One step = one decode layer (router GEMV + top-k + permute + gate/up SwiGLU
-+ down + combine) over a batch of T tokens, on synthetic seeded inputs shaped
-like the Qwen3-235B-A22B NVFP4 MoE layer (H=4096, E=128, top-8, I=1536) at
-T=64 by default.  The metric is decode-layer tokens/s; achieved HBM GB/s, the
-roofline fraction of the dominant kernel and J/token (NVML energy counter)
-are reported beside it.  Under torchrun each rank runs an independent replica
-on its own GPU (the layer does not shard across GPUs); the timed region is
-bracketed by a barrier and the slowest rank's time is reported.
+One step = one decode step (router GEMV + top-k + permute + gate/up SwiGLU
++ down + combine, for each layer of the workload) over a batch of T tokens,
+on synthetic seeded inputs.  Workloads:
+
+  qwen3_235b_nvfp4      Qwen3-235B-A22B-shaped NVFP4 layer (H=4096, E=128,
+                        top-8, I=1536), T=64 by default (the headline line)
+  qwen3_480b_fp8        Qwen3-Coder-480B-shaped FP8 layer (H=6144, E=160,
+                        top-8, I=2560), T=64
+  qwen3_480b_fp8_zipf   the 480B layer with a router bias that makes expert
+                        popularity follow Zipf(1.1); sweep --tokens
+  qwen3_235b_nvfp4_x94  94 235B-shaped NVFP4 layers with fresh weights per
+                        layer (~128 GB), RMS pre-norm and the residual stream
+                        threaded between them, T=128
+  tiny_fp8              H=512, E=8, top-2, I=256, T=4
+
+The metric is decode tokens/s; achieved HBM GB/s, the roofline fraction of
+the dominant kernel (gate/up) and J/token (NVML energy counter) are reported
+beside it.  Under torchrun each rank runs an independent replica on its own
+GPU (the layer does not shard across GPUs); the timed region is bracketed by
+a barrier and the slowest rank's time is reported.
 
 --impl reference times the float64 CPU oracle (the reference semantics) on
 the host cores on a bounded sample of the same workload.
@@ -32,21 +44,33 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 WORKLOADS = {
-    # name: (fmt, H, E, k, I)
-    "qwen3_235b_nvfp4": (2, 4096, 128, 8, 1536),
-    "qwen3_480b_fp8": (1, 6144, 160, 8, 2560),
-    "tiny_fp8": (1, 512, 8, 2, 256),
+    # name: format, shape, default tokens, layers, router bias, RMS pre-norm
+    "qwen3_235b_nvfp4": dict(fmt=2, H=4096, E=128, k=8, I=1536, T=64),
+    "qwen3_480b_fp8": dict(fmt=1, H=6144, E=160, k=8, I=2560, T=64),
+    "qwen3_480b_fp8_zipf": dict(fmt=1, H=6144, E=160, k=8, I=2560, T=64, zipf=1.1),
+    "qwen3_235b_nvfp4_x94": dict(fmt=2, H=4096, E=128, k=8, I=1536, T=128, layers=94,
+                                 prenorm=True),
+    "tiny_fp8": dict(fmt=1, H=512, E=8, k=2, I=256, T=4),
 }
+MOE_FLAG_PRENORM_RMS = 0x2
+
+
+def workload(args):
+    wl = dict(layers=1, zipf=None, prenorm=False)
+    wl.update(WORKLOADS[args.workload])
+    if args.tokens is not None:
+        wl["T"] = args.tokens
+    return wl
 
 
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="qwen3_235b_nvfp4", choices=sorted(WORKLOADS))
-    ap.add_argument("--tokens", type=int, default=64)
+    ap.add_argument("--tokens", type=int, default=None, help="batch size (default per workload)")
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-energy", action="store_true")
@@ -80,7 +104,8 @@ def barrier(world):
 
 # ---------------------------------------------------------------- clocks / energy
 class ClockSampler:
-    """nvidia-smi samples of SM clock and throttle reasons during a region."""
+    """nvidia-smi samples of SM clock and throttle reasons, each stamped with
+    the host time it arrived, so that a window of them can be kept."""
 
     Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
          "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -104,9 +129,12 @@ class ClockSampler:
 
     def _read(self):
         for line in self.proc.stdout:
-            self.lines.append(line.strip())
+            self.lines.append((time.perf_counter(), line.strip()))
 
-    def stop(self):
+    def running(self):
+        return self.proc is not None and self.proc.poll() is None
+
+    def stop(self, t0=None, t1=None):
         if self.proc is None:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
         self.proc.terminate()
@@ -114,22 +142,26 @@ class ClockSampler:
             self.proc.wait(timeout=5)
         except subprocess.TimeoutExpired:
             self.proc.kill()
-        sm, smax, reasons = [], None, set()
+        sm, smax, reasons, watts = [], None, set(), []
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for ln in self.lines:
+        for ts, ln in list(self.lines):
+            if (t0 is not None and ts < t0) or (t1 is not None and ts > t1):
+                continue
             f = [v.strip() for v in ln.split(",")]
             if len(f) < 9:
                 continue
             try:
                 sm.append(float(f[1]))
                 smax = float(f[2])
+                watts.append(float(f[3]))
             except ValueError:
                 continue
             for n, v in zip(names, f[5:9]):
                 if v.lower() == "active":
                     reasons.add(n)
         return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": smax,
-                "reasons": sorted(reasons), "samples": len(sm)}
+                "reasons": sorted(reasons), "samples": len(sm),
+                "power_w_median": statistics.median(watts) if watts else None}
 
 
 class Nvml:
@@ -155,6 +187,19 @@ class Nvml:
         return v.value
 
 
+# ---------------------------------------------------------------- synthetic workload
+def layer_seed(seed, layer):
+    """Seed of layer `layer`'s weights and router (fresh weights per layer)."""
+    return seed + 1009 * layer
+
+
+def zipf_bias(wl, seed, device):
+    from paper_2609_11133_gb300 import synth
+    if not wl["zipf"]:
+        return None
+    return synth.make_zipf_bias(wl["E"], wl["H"], s=wl["zipf"], seed=seed, device=device)
+
+
 # ---------------------------------------------------------------- CPU oracle
 def _oracle_weights(w):
     from oracle import oracle
@@ -165,33 +210,40 @@ def _oracle_weights(w):
 
 
 class OracleSample:
-    """The float64 oracle (router + top-k + experts + combine) on the first n
-    tokens of the workload batch, on the host cores.  n is chosen so that one
-    pass takes about `budget_s` seconds; only the experts those tokens route
-    to are generated (on the host, untimed) unless the full weights are given."""
+    """The float64 oracle (RMS pre-norm if the workload has it, router, top-k,
+    experts, combine) on the first n tokens of layer 0 of the workload, on the
+    host cores.  n is chosen so that one pass takes about `budget_s` seconds;
+    only the experts those tokens route to are generated (on the host,
+    untimed) unless the full weights are given."""
 
-    def __init__(self, fmt, H, E, k, I, T, seed, budget_s=10.0, w=None):
+    def __init__(self, wl, seed, budget_s=10.0, w=None):
         import numpy as np
         import torch
 
         from oracle import oracle
         from paper_2609_11133_gb300 import synth
+        fmt, H, E, k, I, T = (wl[n] for n in ("fmt", "H", "E", "k", "I", "T"))
         self.k = k
+        self.prenorm = wl["prenorm"]
         self.cores = len(os.sched_getaffinity(0))
         x = synth.make_x(T, H, seed=seed)
         self.xb = x.view(torch.int16).numpy().view(np.uint16)
-        self.wr = synth.make_router(E, H, seed=seed).numpy()
-        ids, _ = oracle.topk(oracle.router_logits(self.xb, self.wr), k)
+        s0 = layer_seed(seed, 0)
+        self.wr = synth.make_router(E, H, seed=s0).numpy()
+        b = zipf_bias(wl, seed, "cpu")
+        self.bias = None if b is None else b.numpy()
+        xr = oracle.rmsnorm_bf16(self.xb) if self.prenorm else self.xb
+        ids, _ = oracle.topk(oracle.router_logits(xr, self.wr, self.bias), k)
         # calibrate on one token
         if w is None:
-            w = synth.make_weights(fmt, E, H, I, seed=seed, experts=np.unique(ids[:1]))
+            w = synth.make_weights(fmt, E, H, I, seed=s0, experts=np.unique(ids[:1]))
         self.ow = _oracle_weights(w)
         self.n = 1
         dt = self.run()
         n = max(1, min(T, int(budget_s / max(dt, 1e-3))))
         self.n = n
         if n > 1 and not self._full(w, E):
-            w = synth.make_weights(fmt, E, H, I, seed=seed, experts=np.unique(ids[:n]))
+            w = synth.make_weights(fmt, E, H, I, seed=s0, experts=np.unique(ids[:n]))
             self.ow = _oracle_weights(w)
         self.experts = int(np.unique(ids[:n]).size)
 
@@ -203,22 +255,47 @@ class OracleSample:
         from oracle import oracle
         sub = self.xb[:self.n]
         t0 = time.perf_counter()
-        ids, gates = oracle.topk(oracle.router_logits(sub, self.wr), self.k)
-        oracle.moe_tokens(self.ow, sub, ids, gates)
+        xr = oracle.rmsnorm_bf16(sub) if self.prenorm else sub
+        ids, gates = oracle.topk(oracle.router_logits(xr, self.wr, self.bias), self.k)
+        oracle.moe_tokens(self.ow, xr, ids, gates, residual_bits=sub if self.prenorm else None)
         return time.perf_counter() - t0
 
 
-def cpu_oracle_sample(fmt, H, E, k, I, T, seed, w=None, budget_s=10.0):
-    s = OracleSample(fmt, H, E, k, I, T, seed, budget_s=budget_s, w=w)
+def cpu_oracle_sample(wl, seed, w=None, budget_s=10.0):
+    s = OracleSample(wl, seed, budget_s=budget_s, w=w)
     dt = s.run()
-    return {"value": s.n / dt, "unit": "tokens/s", "cores": s.cores, "kind": "oracle",
-            "sample": f"first {s.n} of {T} tokens ({s.experts} experts): router, top-k, "
-                      f"experts and combine in float64, {dt:.2f} s"}
+    L = wl["layers"]
+    per_layer = f", x{L} layers (layer 0 timed)" if L > 1 else ""
+    return {"value": s.n / (dt * L), "unit": "tokens/s", "cores": s.cores, "kind": "oracle",
+            "sample": f"first {s.n} of {wl['T']} tokens ({s.experts} experts): "
+                      f"{'RMS pre-norm, ' if wl['prenorm'] else ''}router, top-k, experts and "
+                      f"combine in float64, {dt:.2f} s{per_layer}"}
 
 
-def layer_bytes(fmt, H, E, k, I, T, n_active, w_expert_bytes, router_bytes):
-    act = 2 * T * H * 2  # x in, out
-    return router_bytes + n_active * w_expert_bytes + act
+def expert_bytes(w):
+    """(gate+up, down) stored bytes of one expert: codes + scales."""
+    gu = (w.w_gate[0].numel() + w.w_up[0].numel()) + \
+        (w.s_gate[0].numel() * w.s_gate.element_size() + w.s_up[0].numel() * w.s_up.element_size())
+    dn = w.w_down[0].numel() + w.s_down[0].numel() * w.s_down.element_size()
+    if w.fmt == 2:
+        gu += 8
+        dn += 4
+    return gu, dn
+
+
+def zipf_stats(ids, E):
+    """Realised expert popularity of a routed batch: counts, and the exponent
+    of a least-squares fit log n_e = c - s log rank over the experts used."""
+    import numpy as np
+    cnt = np.bincount(ids.reshape(-1), minlength=E)
+    srt = np.sort(cnt)[::-1]
+    nz = srt[srt > 0]
+    fit = None
+    if nz.size >= 3:
+        r = np.log(np.arange(1, nz.size + 1))
+        fit = float(-np.polyfit(r, np.log(nz), 1)[0])
+    return {"max_n_e": int(srt[0]), "top5_n_e": [int(v) for v in srt[:5]],
+            "fitted_s": fit}
 
 
 # ---------------------------------------------------------------- our arm
@@ -235,79 +312,125 @@ def run_ours(args):
         torch.cuda.set_device(0)
     from paper_2609_11133_gb300 import binding, synth
 
-    fmt, H, E, k, I = WORKLOADS[args.workload]
-    T = args.tokens
+    wl = workload(args)
+    fmt, H, E, k, I, T, L = (wl[n] for n in ("fmt", "H", "E", "k", "I", "T", "layers"))
+    flags = MOE_FLAG_PRENORM_RMS if wl["prenorm"] else 0
     dev = "cuda"
-    w = synth.make_weights(fmt, E, H, I, seed=args.seed, device=dev)
+    layers = []
+    for l in range(L):
+        sl = layer_seed(args.seed, l)
+        layers.append((synth.make_weights(fmt, E, H, I, seed=sl, device=dev),
+                       synth.make_router(E, H, seed=sl, device=dev)))
+    bias = zipf_bias(wl, args.seed, dev)
     x = synth.make_x(T, H, seed=args.seed + rank, device=dev)
-    wr = synth.make_router(E, H, seed=args.seed, device=dev)
-    out = torch.empty((T, H), dtype=torch.bfloat16, device=dev)
-    ws = binding.alloc_workspace(binding.moe_workspace_size(w, T, k))
-    ids = torch.empty((T, k), dtype=torch.int32, device=dev)
+    # the residual stream of a stack: layer l reads cur and writes nxt
+    bufs = [torch.empty((T, H), dtype=torch.bfloat16, device=dev) for _ in range(2)]
+    ws = binding.alloc_workspace(binding.moe_workspace_size(layers[0][0], T, k))
     stream = torch.cuda.current_stream()
 
-    # routing of this batch -> unique experts -> algorithmic bytes
-    binding.moe_decode_layer_ex(x, wr, None, w, k, out, ws, topk_ids_out=ids)
+    def io(l, x_in):
+        """(input, residual, output) of layer l."""
+        if L == 1:
+            return x_in, None, bufs[0]
+        cur = x_in if l == 0 else bufs[(l - 1) % 2]
+        return cur, cur, bufs[l % 2]
+
+    def run_layers(x_in, ev=None, ids=None):
+        for l, (w, wr) in enumerate(layers):
+            xi, res, out = io(l, x_in)
+            if ev is None and ids is None:
+                binding.moe_decode_layer(xi, wr, bias, w, k, out, ws, flags=flags, residual=res)
+            else:
+                binding.moe_decode_layer_ex(xi, wr, bias, w, k, out, ws, flags=flags,
+                                            residual=res, events=None if ev is None else ev[l],
+                                            topk_ids_out=None if ids is None else ids[l])
+        return io(L - 1, x_in)[2]
+
+    # routing of this batch -> unique experts per layer -> algorithmic bytes
+    ids = [torch.empty((T, k), dtype=torch.int32, device=dev) for _ in range(L)]
+    run_layers(x, ids=ids)
     torch.cuda.synchronize()
     assert binding.moe_read_status(ws) == 0
-    n_active = int(torch.unique(ids).numel())
-    per_expert = w.nbytes_expert()
-    gu_bytes = (w.w_gate[0].numel() + w.w_up[0].numel()) * 1 + \
-        (w.s_gate[0].numel() * w.s_gate.element_size() + w.s_up[0].numel() * w.s_up.element_size())
-    dn_bytes = w.w_down[0].numel() + w.s_down[0].numel() * w.s_down.element_size()
-    if fmt == 2:
-        gu_bytes += 8
-        dn_bytes += 4
+    n_active = [int(torch.unique(i).numel()) for i in ids]
+    w0 = layers[0][0]
+    per_expert = w0.nbytes_expert()
+    gu_bytes, dn_bytes = expert_bytes(w0)
     router_bytes = E * H * 4
-    B = layer_bytes(fmt, H, E, k, I, T, n_active, per_expert, router_bytes)
-
-    ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
-
-    def step(record):
-        binding.moe_decode_layer_ex(x, wr, None, w, k, out, ws, events=ev if record else None)
+    act_bytes = 2 * T * H * 2  # x in, out
+    B = sum(router_bytes + n * per_expert + act_bytes for n in n_active)
 
     for _ in range(max(3, args.warmup)):
-        step(False)
+        run_layers(x)
     torch.cuda.synchronize()
 
-    # One layer call captured in a CUDA graph: the timed loop replays it, so the
-    # host's launch work is not part of the measurement (the layer takes no
-    # host-side decisions between its kernels).
+    # The step's layer calls captured in one CUDA graph: the timed loop replays
+    # it, so the host's launch work is not part of the measurement (the layer
+    # takes no host-side decisions between its kernels).
     g_step = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g_step):
-        binding.moe_decode_layer(x, wr, None, w, k, out, ws)
+        out = run_layers(x)
     for _ in range(max(3, args.warmup)):
         g_step.replay()
     torch.cuda.synchronize()
     barrier(world)
 
-    # ---- timed region (device time, CUDA events on the launching stream)
+    # clock sampler: started before the timed region; the replays below keep
+    # the GPU busy until its first sample arrives (bounded), so that the
+    # samples kept cover the timed region and the energy window only
     clocks = ClockSampler(local)
     clocks.start()
+    t_wait = time.perf_counter()
+    while clocks.running() and not clocks.lines and time.perf_counter() - t_wait < 5.0:
+        g_step.replay()
+        torch.cuda.synchronize()
+
+    # ---- timed region (device time, CUDA events on the launching stream)
     t_beg = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
     torch.cuda.synchronize()
     barrier(world)
+    h_beg = time.perf_counter()
     t_beg.record(stream)
     for _ in range(args.steps):
         g_step.replay()
     t_end.record(stream)
     torch.cuda.synchronize()
+    h_end = time.perf_counter()
     ms_total = t_beg.elapsed_time(t_end)
-    clk = clocks.stop()
     ms_step = barrier_max(ms_total / args.steps, world)
     tok_s = world * T / (ms_step * 1e-3)
 
+    # ---- energy per token (NVML counter over >= 2 s of back-to-back steps)
+    energy = None
+    if not args.no_energy:
+        nv = Nvml(local)
+        if nv.ok:
+            n_rep = max(1, int(2.0 / (ms_step * 1e-3)))
+            torch.cuda.synchronize()
+            j0 = nv.energy_mj()
+            t0 = time.perf_counter()
+            for _ in range(n_rep):
+                g_step.replay()
+            torch.cuda.synchronize()
+            h_end = time.perf_counter()
+            dt = h_end - t0
+            j1 = nv.energy_mj()
+            energy = {"j_per_token": (j1 - j0) * 1e-3 / (n_rep * T), "avg_w": (j1 - j0) * 1e-3 / dt,
+                      "window_s": dt, "source": "nvmlDeviceGetTotalEnergyConsumption"}
+    clk = clocks.stop(h_beg, h_end)
+    clk["window"] = "timed region" + (" + energy window (same step replayed)" if energy else "")
+
     # per-kernel durations: eager calls with events between the kernels
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(L)]
     kern = [[], [], []]
-    for _ in range(min(args.steps, 20)):
-        step(True)
+    for _ in range(max(1, min(args.steps, 20 if L == 1 else 2))):
+        run_layers(x, ev=ev)
         torch.cuda.synchronize()
         for i in range(3):
-            kern[i].append(ev[i].elapsed_time(ev[i + 1]))
+            kern[i].append(sum(ev[l][i].elapsed_time(ev[l][i + 1]) for l in range(L)))
 
     # ---- end to end through the public API with host buffers: the input is
-    # copied from pinned host memory, the layer runs, the output is copied
+    # copied from pinned host memory, the step runs, the output is copied
     # back, every step (captured together in one graph)
     x_host = torch.empty((T, H), dtype=torch.bfloat16, pin_memory=True)
     x_host.copy_(x.cpu())
@@ -316,8 +439,8 @@ def run_ours(args):
     g_e2e = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g_e2e):
         x_dev.copy_(x_host, non_blocking=True)
-        binding.moe_decode_layer(x_dev, wr, None, w, k, out, ws)
-        out_host.copy_(out, non_blocking=True)
+        out_e2e = run_layers(x_dev)
+        out_host.copy_(out_e2e, non_blocking=True)
     for _ in range(3):
         g_e2e.replay()
     torch.cuda.synchronize()
@@ -330,48 +453,48 @@ def run_ours(args):
     e1.record(stream)
     torch.cuda.synchronize()
     ms_e2e = barrier_max(e0.elapsed_time(e1) / args.steps, world)
+    assert torch.isfinite(out_host.float()).all()
 
-    # ---- energy per token (NVML counter over >= 2 s of back-to-back layers)
-    energy = None
-    if not args.no_energy:
-        nv = Nvml(local)
-        if nv.ok:
-            n_rep = max(1, int(2.0 / (ms_step * 1e-3)))
-            torch.cuda.synchronize()
-            j0 = nv.energy_mj()
-            t0 = time.perf_counter()
-            for _ in range(n_rep):
-                g_step.replay()
-            torch.cuda.synchronize()
-            dt = time.perf_counter() - t0
-            j1 = nv.energy_mj()
-            energy = {"j_per_token": (j1 - j0) * 1e-3 / (n_rep * T), "avg_w": (j1 - j0) * 1e-3 / dt,
-                      "window_s": dt, "source": "nvmlDeviceGetTotalEnergyConsumption"}
-
-    # ---- roofline of the dominant kernel (gate/up) and of the whole layer
-    import json as _json
+    # ---- roofline of the dominant kernel (gate/up) and of the whole step
     peaks = {}
     pp = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(pp):
-        peaks = _json.load(open(pp))
+        peaks = json.load(open(pp))
     hbm = float(peaks.get("hbm_gbs", 6800.0))
     peak_src = "measured" if "hbm_gbs" in peaks else "fallback"
-    gu_ms = statistics.mean(kern[1])
-    dn_ms = statistics.mean(kern[2])
-    rt_ms = statistics.mean(kern[0])
-    gu_alg = n_active * gu_bytes
-    dn_alg = n_active * dn_bytes
+    gu_ms = statistics.mean(kern[1]) / L
+    dn_ms = statistics.mean(kern[2]) / L
+    rt_ms = statistics.mean(kern[0]) / L
+    gu_alg = statistics.mean(n_active) * gu_bytes  # per launch
     gu_gbs = gu_alg / (gu_ms * 1e-3) / 1e9
     layer_gbs = B / (ms_step * 1e-3) / 1e9
+    # DRAM bytes of one gate/up launch from a committed ncu capture, valid only
+    # while the kernel sources are the ones that capture was taken on
     traffic = None
     tp = os.path.join(ROOT, "profiles", "traffic.json")
     if os.path.exists(tp):
-        tj = _json.load(open(tp)).get(f"{args.workload}_T{T}")
+        import hashlib
+        tj = json.load(open(tp)).get(f"{args.workload}_T{T}")
         if tj:
-            traffic = tj.get("gateup_dram_bytes")
+            hsh = hashlib.sha256()
+            for f in ("ffn.cuh", "common.cuh"):
+                hsh.update(open(os.path.join(ROOT, "paper_2609_11133_gb300", "csrc", f), "rb").read())
+            if hsh.hexdigest() == tj.get("kernel_sources_sha256"):
+                traffic = tj.get("gateup_dram_bytes")
 
+    cfg = {"workload": f"{args.workload}_T{T}", "H": H, "E": E, "k": k, "I": I,
+           "tokens": T, "format": "nvfp4" if fmt == 2 else "fp8_block128",
+           "active_experts": n_active[0] if L == 1 else statistics.mean(n_active),
+           "l2": f"inputs larger than L2: {B / 1e9:.2f} GB of weights touched per step",
+           "parallelism": f"replicas x{world}"}
+    if L > 1:
+        cfg.update(layers=L, prenorm="rms, eps 1e-6, unit weight", residual="threaded",
+                   weights_gb=round(sum(w.nbytes_expert() * E for w, _ in layers) / 1e9, 1))
+    if wl["zipf"]:
+        cfg["router_bias"] = f"zipf s={wl['zipf']}"
+        cfg["popularity"] = zipf_stats(ids[0].cpu().numpy(), E)
     res = {
-        "metric": "MoE decode-layer tokens/s",
+        "metric": "MoE decode-layer tokens/s" if L == 1 else f"MoE {L}-layer decode-step tokens/s",
         "value": tok_s,
         "unit": "tokens/s",
         "n_gpus": world,
@@ -384,30 +507,28 @@ def run_ours(args):
         "dtype": "nvfp4 weights, f16 MMA with fp32 accumulate" if fmt == 2 else
                  "fp8 weights, f16 MMA with fp32 accumulate",
         "data": "synthetic (seeded N(0,1) activations, N(0,0.02) weights quantised)",
-        "config": {"workload": f"{args.workload}_T{T}", "H": H, "E": E, "k": k, "I": I,
-                   "tokens": T, "format": "nvfp4" if fmt == 2 else "fp8_block128",
-                   "active_experts": n_active,
-                   "l2": f"inputs larger than L2: {B / 1e9:.2f} GB of weights touched per step",
-                   "parallelism": f"replicas x{world}"},
+        "config": cfg,
         "hbm_gbs": layer_gbs,
         "hbm_frac_of_measured": layer_gbs / hbm,
         "hbm_frac_of_8tbs": layer_gbs / 8000.0,
         "algorithmic_bytes_per_step": B,
-        "kernel_ms": {"route": rt_ms, "gate_up": gu_ms, "down": dn_ms},
+        "kernel_ms": {"route": rt_ms, "gate_up": gu_ms, "down": dn_ms,
+                      "per": "layer" if L == 1 else f"layer, mean of {L}"},
         "roofline": {"bound": "hbm", "achieved": gu_gbs, "peak": hbm, "unit": "GB/s",
                      "frac": gu_gbs / hbm, "traffic": traffic, "kernel": "ffn gate/up",
                      "peak_source": peak_src},
         "e2e": {"value": world * T / (ms_e2e * 1e-3), "unit": "tokens/s",
                 "h2d_bytes_per_step": T * H * 2, "d2h_bytes_per_step": T * H * 2},
-        "gpu_launches": 5 * args.steps,
-        "timing": "CUDA-graph replay of one layer call per step",
+        "gpu_launches": 5 * L * args.steps,
+        "timing": "CUDA-graph replay of one step's layer calls per step",
         "clocks": clk,
         "energy": energy,
     }
     if energy:
         res["j_per_token"] = energy["j_per_token"]
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        res["cpu_baseline"] = cpu_oracle_sample(fmt, H, E, k, I, T, args.seed, w=w)
+        res["cpu_baseline"] = cpu_oracle_sample(wl, args.seed, w=w0 if L == 1 and not wl["zipf"]
+                                                else None)
     if rank == 0:
         print(json.dumps(res))
     if world > 1:
@@ -419,23 +540,26 @@ def run_reference(args):
     rank, world, _ = dist_env()
     if rank != 0:
         return
-    fmt, H, E, k, I = WORKLOADS[args.workload]
-    T = args.tokens
-    s = OracleSample(fmt, H, E, k, I, T, args.seed, budget_s=8.0)
-    warm = max(0, min(args.warmup, 1))
+    wl = workload(args)
+    T, L = wl["T"], wl["layers"]
+    steps, warm = max(1, args.steps), max(0, args.warmup)
+    # each step is a bounded token sample, sized so the whole run takes ~2 min
+    budget = min(8.0, max(0.3, 120.0 / (steps + warm)))
+    s = OracleSample(wl, args.seed, budget_s=budget)
     for _ in range(warm):
         s.run()
-    steps = max(1, min(args.steps, 5))
     dt = sum(s.run() for _ in range(steps)) / steps
-    v = s.n / dt
-    res = {"metric": "MoE decode-layer tokens/s", "value": v, "unit": "tokens/s", "n_gpus": world,
-           "steps": steps, "warmup": warm, "ms_per_step": dt * 1e3,
+    v = s.n / (dt * L)
+    res = {"metric": "MoE decode-layer tokens/s" if L == 1 else f"MoE {L}-layer decode-step tokens/s",
+           "value": v, "unit": "tokens/s", "n_gpus": world,
+           "steps": steps, "warmup": warm, "ms_per_step": dt * L * 1e3 * T / s.n,
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
            "data": "synthetic", "impl": "reference",
-           "config": {"workload": f"{args.workload}_T{T}", "H": H, "E": E, "k": k, "I": I,
-                      "tokens": T},
+           "config": {"workload": f"{args.workload}_T{T}", "H": wl["H"], "E": wl["E"],
+                      "k": wl["k"], "I": wl["I"], "tokens": T},
            "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": s.cores, "kind": "oracle",
-                            "sample": f"first {s.n} of {T} tokens per step ({s.experts} experts)"},
+                            "sample": f"first {s.n} of {T} tokens per step ({s.experts} experts)"
+                                      + (f", layer 0 of {L}" if L > 1 else "")},
            "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0,
                    "d2h_bytes_per_step": 0}}
     print(json.dumps(res))

@@ -78,9 +78,16 @@ def quantize_fp8_block(w: torch.Tensor):
 
 def quantize_nvfp4(w: torch.Tensor):
     """w [N, K] fp32 -> (codes uint8 [N, K/2], sf uint8 [N, K/16], ts float)."""
+    codes, sf, ts = _quantize_nvfp4(w)
+    return codes, sf, float(ts)
+
+
+def _quantize_nvfp4(w: torch.Tensor):
+    """quantize_nvfp4 with the tensor scale left as a 0-d fp32 tensor on w's
+    device (no host synchronisation)."""
     N, K = w.shape
     amax = w.abs().amax()
-    ts = (amax / (_E4M3_MAX * _E2M1_MAX)) if float(amax) > 0 else torch.ones((), device=w.device)
+    ts = torch.where(amax > 0, amax / (_E4M3_MAX * _E2M1_MAX), torch.ones_like(amax))
     blk = w.reshape(N, K // 16, 16)
     bmax = blk.abs().amax(dim=2)
     sf_code = encode_e4m3(bmax / (_E2M1_MAX * ts))
@@ -90,7 +97,7 @@ def quantize_nvfp4(w: torch.Tensor):
                     torch.zeros_like(blk))
     nib = encode_e2m1(q).reshape(N, K)
     codes = (nib[:, 0::2] | (nib[:, 1::2] << 4)).contiguous()
-    return codes, sf_code.contiguous(), float(ts)
+    return codes, sf_code.contiguous(), ts
 
 
 # ----------------------------------------------------------------- layer inputs
@@ -150,10 +157,10 @@ def make_weights(fmt: int, E: int, H: int, I: int, seed: int = 0, device="cpu",
         ts = torch.ones((E,), dtype=torch.float32, device=dev)
         for e in todo:
             w = _normal((N, K), std, dev, seed * 1_000_003 + which * 10_007 + e)
-            c, s, t = quantize_nvfp4(w)
+            c, s, t = _quantize_nvfp4(w)
             codes[e].copy_(c)
             sf[e].copy_(s)
-            ts[e] = t
+            ts[e].copy_(t)
         return codes, sf, ts
 
     wg, sg, tg = one(1, I, H)

@@ -13,14 +13,24 @@ GATE_TOL = 1e-6
 
 
 class Case:
-    def __init__(self, fmt, T, H, E, k, I, seed=0, bias=None, residual=False, flags=0):
+    """One layer call.  Weights, router, input and residual are drawn from
+    `seed` unless given (w, wr, x: device tensors; residual: True to draw one,
+    or a [T, H] bf16 device tensor); `ow` is the oracle's copy of w, if the
+    caller already made one."""
+
+    def __init__(self, fmt, T, H, E, k, I, seed=0, bias=None, residual=False, flags=0,
+                 w=None, wr=None, x=None, ow=None):
         dev = "cuda"
         self.fmt, self.T, self.H, self.E, self.k, self.I, self.flags = fmt, T, H, E, k, I, flags
-        self.w = synth.make_weights(fmt, E, H, I, seed=seed, device=dev)
-        self.x = synth.make_x(T, H, seed=seed, device=dev)
-        self.wr = synth.make_router(E, H, seed=seed, device=dev)
+        self.w = synth.make_weights(fmt, E, H, I, seed=seed, device=dev) if w is None else w
+        self.x = synth.make_x(T, H, seed=seed, device=dev) if x is None else x
+        self.wr = synth.make_router(E, H, seed=seed, device=dev) if wr is None else wr
         self.bias = None if bias is None else bias.to(dev)
-        self.residual = synth.make_x(T, H, seed=seed + 1000, device=dev) if residual else None
+        if isinstance(residual, torch.Tensor):
+            self.residual = residual
+        else:
+            self.residual = synth.make_x(T, H, seed=seed + 1000, device=dev) if residual else None
+        self.ow = ow
 
     def run(self, out=None):
         T, H, E, k = self.T, self.H, self.E, self.k
@@ -68,7 +78,7 @@ class Case:
 
     def reference(self, tokens=None):
         ids, gates = self.check_routing()
-        ow = oracle_weights(self.w)
+        ow = oracle_weights(self.w) if self.ow is None else self.ow
         res = None if self.residual is None else np_(self.residual)
         return oracle.moe_tokens(ow, self.x_bits(), ids, gates, tokens, res)
 
