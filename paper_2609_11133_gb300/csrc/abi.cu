@@ -8,6 +8,7 @@
 #include <mutex>
 
 #include "../../include/moe.h"
+#include "act_terms.cuh"
 #include "ffn_launch.cuh"
 #include "route.cuh"
 
@@ -101,27 +102,37 @@ bool map_sf(CUtensorMap* m, const void* sf, int E, int N, int K) {
 
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
-// Expert engine: warp MMA (default) or tcgen05 (MOE_ENGINE=tc).
-bool use_tc_engine() {
-  static int v = -1;
-  if (v < 0) {
+// Expert engines: the block-scaled tcgen05 engine (ffn_bs.cuh) for NVFP4, the
+// warp-MMA engine (ffn.cuh) for FP8.  MOE_ENGINE=mma runs NVFP4 on the
+// warp-MMA engine too (for comparisons).
+enum Engine { kEngMma = 0, kEngBs = 1 };
+
+int engine_for(int fmt) {
+  static int force_mma = -1;
+  if (force_mma < 0) {
     const char* s = std::getenv("MOE_ENGINE");
-    v = (s && std::strcmp(s, "tc") == 0) ? 1 : 0;
+    force_mma = (s && std::strcmp(s, "mma") == 0) ? 1 : 0;
   }
-  return v == 1;
+  return (fmt == MOE_FMT_NVFP4 && !force_mma) ? kEngBs : kEngMma;
 }
 
-// Token-chunk size of the expert kernels (the N side of the MMA).
-// MOE_NT=8|16|32 overrides the choice (for measurements).
-int nt_for(int T) {
+int act_for(int fmt, int eng) {
+  if (eng == kEngBs) return kActTerms;
+  return fmt == MOE_FMT_NVFP4 ? kActF16Perm : kActF16;
+}
+
+// Token-chunk size of the expert kernels (the N side of the MMA; the
+// block-scaled engine uses 4 rows of N per token).  MOE_NT overrides the
+// choice (for measurements).
+int nt_for(int T, int eng) {
   if (const char* s = std::getenv("MOE_NT")) {
     const int v = std::atoi(s);
-    if (v == 16 || v == 32 || (v == 8 && !use_tc_engine())) return v;
+    if (v == 8 || v == 16 || (v == 32 && eng == kEngMma)) return v;
   }
-  if (use_tc_engine()) return T <= 16 ? 16 : 32;
-  // 8-token chunks let the consumer warps hold a whole stage in registers and
-  // release it at once; at T <= 64 few experts get more than 8 tokens (those
-  // are processed in several chunks).  Larger batches use 32-token chunks.
+  // 8-token chunks: at T <= 64 few experts get more than 8 tokens (those are
+  // processed in several chunks); the warp-MMA consumers then hold a whole
+  // stage in registers and release it at once.
+  if (eng == kEngBs) return T <= 64 ? 8 : 16;
   return T <= 64 ? 8 : 32;
 }
 
@@ -188,14 +199,23 @@ int run_experts(const ExpertRun& r, cudaStream_t st, cudaEvent_t ev_mid) {
   }
   __half* x16 = ws_ptr<__half>(r.ws, r.L.x16);
   __half* h16 = ws_ptr<__half>(r.ws, r.L.h16);
-  const bool tc = use_tc_engine();
-  // token rows: tcgen05 reads 64-element 128B-swizzled K atoms, warp MMA whole K-stages
-  const uint32_t bcols = tc ? 64u : (uint32_t)KEL;
-  const CUtensorMapSwizzle bsw = tc ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE;
-  ok = ok && map_2d(&m1.b, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, x16, (uint64_t)H, (uint64_t)r.T,
-                    (uint64_t)H * 2, bcols, 1, bsw);
-  ok = ok && map_2d(&m2.b, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, h16, (uint64_t)I,
-                    (uint64_t)r.T * r.k, (uint64_t)I * 2, bcols, 8, bsw);
+  const int eng = engine_for(w->fmt);
+  if (eng == kEngBs) {
+    // activation terms: x rows 4t..4t+3 (one box per token), h rows of a
+    // chunk's assignments (one box of 4*nt rows)
+    ok = ok && map_2d(&m1.b, CU_TENSOR_MAP_DATA_TYPE_UINT8, ws_ptr<uint8_t>(r.ws, r.L.xq),
+                      (uint64_t)H / 2, (uint64_t)r.T * kTerms, (uint64_t)H / 2, kRowBytes, kTerms,
+                      CU_TENSOR_MAP_SWIZZLE_128B);
+    ok = ok && map_2d(&m2.b, CU_TENSOR_MAP_DATA_TYPE_UINT8, ws_ptr<uint8_t>(r.ws, r.L.hq),
+                      (uint64_t)I / 2, (uint64_t)hq_rows(r.T, r.k), (uint64_t)I / 2, kRowBytes,
+                      (uint32_t)(kTerms * r.nt), CU_TENSOR_MAP_SWIZZLE_128B);
+  } else {
+    ok = ok && map_2d(&m1.b, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, x16, (uint64_t)H, (uint64_t)r.T,
+                      (uint64_t)H * 2, (uint32_t)KEL, 1, CU_TENSOR_MAP_SWIZZLE_NONE);
+    ok = ok && map_2d(&m2.b, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, h16, (uint64_t)I,
+                      (uint64_t)r.T * r.k, (uint64_t)I * 2, (uint32_t)KEL, 8,
+                      CU_TENSOR_MAP_SWIZZLE_NONE);
+  }
   if (!ok) return MOE_ERR_CUDA;
 
   FfnParams p{};
@@ -223,6 +243,9 @@ int run_experts(const ExpertRun& r, cudaStream_t st, cudaEvent_t ev_mid) {
   p1.gu = ws_ptr<float>(r.ws, r.L.gu);
   p1.h16 = h16;
   p1.hinv = ws_ptr<float>(r.ws, r.L.hinv);
+  p1.bsf = ws_ptr<uint8_t>(r.ws, r.L.xsf);
+  p1.hq = ws_ptr<uint8_t>(r.ws, r.L.hq);
+  p1.hsf = ws_ptr<uint8_t>(r.ws, r.L.hsf);
   p1.test_stall = r.test_stall;
 
   FfnParams p2 = p;
@@ -237,19 +260,22 @@ int run_experts(const ExpertRun& r, cudaStream_t st, cudaEvent_t ev_mid) {
   p2.y_perm = r.y_perm;
   p2.out = r.out;
   p2.residual = r.residual;
+  p2.bsf = ws_ptr<uint8_t>(r.ws, r.L.hsf);
 
   auto launch = [&](const FfnMaps& m, const FfnParams& pp) {
-    if (tc)
-      return fp4 ? launch_ffn_tc<2>(r.nt, r.sms, m, pp, st) : launch_ffn_tc<1>(r.nt, r.sms, m, pp, st);
+    if (eng == kEngBs) return launch_ffn_bs(r.nt, r.sms, m, pp, st);
     return fp4 ? launch_ffn<2>(r.nt, r.sms, m, pp, st, true)
                : launch_ffn<1>(r.nt, r.sms, m, pp, st, true);
   };
   cudaError_t err = launch(m1, p1);
   if (err != cudaSuccess) return MOE_ERR_CUDA;
   if (ev_mid && cudaEventRecord(ev_mid, st) != cudaSuccess) return MOE_ERR_CUDA;
-  const bool perm = !tc && fp4;  // h16 unit order of the warp-MMA NVFP4 engine
-  err = fp4 ? launch_swiglu<2>(r.T * r.k, r.sms, p1, perm, st)
-            : launch_swiglu<1>(r.T * r.k, r.sms, p1, perm, st);
+  if (eng == kEngBs)
+    err = launch_swiglu_terms(r.T * r.k, r.sms, p1, st);
+  else if (fp4)
+    err = launch_swiglu<2>(r.T * r.k, r.sms, p1, true, st);  // h16 in the unit order
+  else
+    err = launch_swiglu<1>(r.T * r.k, r.sms, p1, false, st);
   if (err != cudaSuccess) return MOE_ERR_CUDA;
   err = launch(m2, p2);
   if (err != cudaSuccess) return MOE_ERR_CUDA;
@@ -284,7 +310,7 @@ int moe_workspace_size(const moe_expert_weights_t* w, int T, int k, size_t* byte
   if (rc) return rc;
   rc = check_tk(T, k, w->E);
   if (rc) return rc;
-  *bytes = ws_layout(T, k, w->E, w->H, w->I).total;
+  *bytes = ws_layout(T, k, w->E, w->H, w->I, w->fmt == MOE_FMT_NVFP4).total;
   return MOE_OK;
 }
 
@@ -384,14 +410,15 @@ int moe_expert_ffn(const void* x, const moe_expert_weights_t* w, const int32_t* 
   if (T == 0) return MOE_OK;
   if (!x || !offsets || !sorted_assign || !active || !y_perm || !ws) return MOE_ERR_INVALID_ARG;
   if (!aligned(x, 16) || !aligned(y_perm, 16) || !aligned(ws, 256)) return MOE_ERR_INVALID_ARG;
-  const WsLayout L = ws_layout(T, k, w->E, w->H, w->I);
+  const WsLayout L = ws_layout(T, k, w->E, w->H, w->I, w->fmt == MOE_FMT_NVFP4);
   if (ws_bytes < L.total) return MOE_ERR_WORKSPACE_TOO_SMALL;
   if (T == 0) return MOE_OK;
   int sms = 0;
   rc = device_check(&sms);
   if (rc) return rc;
   cudaStream_t st = (cudaStream_t)stream;
-  const int nt = nt_for(T);
+  const int eng = engine_for(w->fmt);
+  const int nt = nt_for(T, eng);
   PrepParams pp{};
   pp.x = static_cast<const __nv_bfloat16*>(x);
   pp.T = T;
@@ -400,8 +427,10 @@ int moe_expert_ffn(const void* x, const moe_expert_weights_t* w, const int32_t* 
   pp.k = k;
   pp.fmt = w->fmt;
   pp.nt = nt;
-  pp.unit_perm = (!use_tc_engine() && w->fmt == MOE_FMT_NVFP4) ? 1 : 0;
+  pp.act = act_for(w->fmt, eng);
   pp.x16 = ws_ptr<__half>(ws, L.x16);
+  pp.xq = ws_ptr<uint8_t>(ws, L.xq);
+  pp.xsf = ws_ptr<uint8_t>(ws, L.xsf);
   pp.xinv = ws_ptr<float>(ws, L.xinv);
   pp.offsets = offsets;
   pp.active = active;
@@ -460,7 +489,7 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
     return MOE_ERR_INVALID_ARG;
   if (out == x) return MOE_ERR_INVALID_ARG;
   const int E = w->E, H = w->H, I = w->I;
-  const WsLayout L = ws_layout(T, k, E, H, I);
+  const WsLayout L = ws_layout(T, k, E, H, I, w->fmt == MOE_FMT_NVFP4);
   if (ws_bytes < L.total) return MOE_ERR_WORKSPACE_TOO_SMALL;
   if (T == 0) return MOE_OK;
   int sms = 0;
@@ -470,7 +499,8 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
   cudaEvent_t ev[4] = {nullptr, nullptr, nullptr, nullptr};
   if (events)
     for (int i = 0; i < 4; ++i) ev[i] = static_cast<cudaEvent_t>(events[i]);
-  const int nt = nt_for(T);
+  const int eng = engine_for(w->fmt);
+  const int nt = nt_for(T, eng);
 
   RouteParams p{};
   p.x = static_cast<const __nv_bfloat16*>(x);
@@ -485,7 +515,7 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
   p.fmt = w->fmt;
   p.fused = 1;
   p.nt = nt;
-  p.unit_perm = (!use_tc_engine() && w->fmt == MOE_FMT_NVFP4) ? 1 : 0;
+  p.act = act_for(w->fmt, eng);
   p.logits = logits_out ? logits_out : ws_ptr<float>(ws, L.logits);
   p.ids = ws_ptr<int>(ws, L.ids);
   p.gates = ws_ptr<float>(ws, L.gates);
@@ -494,6 +524,8 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
   p.chunk_cnt = ws_ptr<unsigned>(ws, L.route_chunk);
   p.done_cnt = ws_ptr<unsigned>(ws, L.route_done);
   p.x16 = ws_ptr<__half>(ws, L.x16);
+  p.xq = ws_ptr<uint8_t>(ws, L.xq);
+  p.xsf = ws_ptr<uint8_t>(ws, L.xsf);
   p.xinv = ws_ptr<float>(ws, L.xinv);
   p.zero_a = ws_ptr<float4>(ws, L.gu);
   p.zero_a_n4 = (size_t)T * k * 2 * I / 4;

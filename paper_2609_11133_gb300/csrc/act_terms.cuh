@@ -1,0 +1,130 @@
+// Activations as sums of NVFP4-coded terms, the B operand of the block-scaled
+// tensor-core engine (ffn_bs.cuh).
+//
+// The tcgen05 kind::mxf4nvf4 MMA multiplies E2M1 codes with one UE4M3 scale
+// per 16 K elements on BOTH operands.  The weights are stored that way; the
+// activations (bf16 x, fp32 h) are not, and one E2M1 code keeps only two
+// significant bits.  So every activation row v is written as
+//
+//     v * 2^p = sum_{t<4} s_t[b] * q_t[i],   i in block b of 16 elements,
+//
+// with 2^p a per-row power of two, s_t[b] UE4M3 and q_t[i] E2M1: term 0 codes
+// v, term t codes what terms 0..t-1 left over.  Each scale is the smallest
+// UE4M3 value >= max|residual| / 6, so |q| <= 6 never saturates, and the
+// largest residual of a block shrinks by about 6x per term: after four terms
+// it is below 2^-9.5 of the block maximum (finer than the bf16 input itself),
+// and the layer output stays within ~1e-4 of the exact result.  Each term is
+// one "token row" of the MMA's B operand, so a token costs 4 rows of N; the
+// four partial products are summed in the epilogue.  The residual update
+// r -= s*q is exact in fp32 (s*q has at most 6 significant bits).
+#pragma once
+
+#include "common.cuh"
+
+namespace moe {
+
+constexpr int kTerms = 4;
+
+// Power-of-two factor that maps max|v| into [2^10, 2^11): the first term's
+// scales stay below 2^11/6 < 448 (the UE4M3 maximum) and the fourth term's
+// above the UE4M3 subnormal range for every block within 2^-8 of the row max.
+__device__ __forceinline__ float pow2_scale_terms(float amax) {
+  if (!(amax > 0.f) || !isfinite(amax)) return 1.f;
+  int e;
+  frexpf(amax, &e);  // amax = m * 2^e, 0.5 <= m < 1
+  return ldexpf(1.f, min(11 - e, 126));
+}
+
+// Smallest UE4M3 value >= v (v >= 0), as its code byte; *val gets the value.
+__device__ __forceinline__ uint32_t ue4m3_ceil(float v, float* val) {
+  uint16_t two;  // both bytes hold e4m3(v), whichever source lands in which byte
+  asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %1;" : "=h"(two) : "f"(v));
+  uint32_t code = two & 0xffu;
+  float f = __half2float(__ushort_as_half((uint16_t)(e4m3x2_to_f16x2(code) & 0xffffu)));
+  if (f < v && code < 0x7eu) {
+    ++code;  // the next larger magnitude
+    f = __half2float(__ushort_as_half((uint16_t)(e4m3x2_to_f16x2(code) & 0xffffu)));
+  }
+  *val = f;
+  return code;
+}
+
+// Eight floats to eight E2M1 codes, round to nearest even, saturating at 6;
+// element 2i in the low nibble of byte i (the weights' packing).
+__device__ __forceinline__ uint32_t e2m1x8_from_f32(const float* q) {
+  uint32_t w;
+  asm("{\n .reg .b8 b0, b1, b2, b3;\n"
+      " cvt.rn.satfinite.e2m1x2.f32 b0, %2, %1;\n"
+      " cvt.rn.satfinite.e2m1x2.f32 b1, %4, %3;\n"
+      " cvt.rn.satfinite.e2m1x2.f32 b2, %6, %5;\n"
+      " cvt.rn.satfinite.e2m1x2.f32 b3, %8, %7;\n"
+      " mov.b32 %0, {b0, b1, b2, b3};\n}\n"
+      : "=r"(w)
+      : "f"(q[0]), "f"(q[1]), "f"(q[2]), "f"(q[3]), "f"(q[4]), "f"(q[5]), "f"(q[6]), "f"(q[7]));
+  return w;
+}
+
+// Encode one 16-element block r (already scaled by the row's power of two)
+// into kTerms terms: codes[t] (16 E2M1 codes, 8 bytes) and sf[t] (UE4M3).
+// r is consumed (it ends as the final residual).
+__device__ __forceinline__ void encode_terms16(float (&r)[16], uint2 (&codes)[kTerms],
+                                               uint32_t (&sf)[kTerms]) {
+#pragma unroll
+  for (int t = 0; t < kTerms; ++t) {
+    float m = 0.f;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) m = fmaxf(m, fabsf(r[i]));
+    float s = 0.f;
+    const uint32_t c = ue4m3_ceil(m * (1.f / 6.f), &s);
+    sf[t] = (m > 0.f) ? c : 0u;
+    if (!(m > 0.f)) {
+      codes[t] = make_uint2(0u, 0u);
+      continue;
+    }
+    const float inv = 1.f / s;
+    float q[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) q[i] = r[i] * inv;
+    const uint32_t w0 = e2m1x8_from_f32(q), w1 = e2m1x8_from_f32(q + 8);
+    codes[t] = make_uint2(w0, w1);
+    // subtract the coded values (exact)
+    uint32_t d0[4], d1[4];
+    e2m1x8_to_f16x8(w0, d0);
+    e2m1x8_to_f16x8(w1, d1);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const uint32_t di = (i < 4) ? d0[i] : d1[i - 4];
+      const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&di));
+      r[2 * i] = fmaf(-f.x, s, r[2 * i]);
+      r[2 * i + 1] = fmaf(-f.y, s, r[2 * i + 1]);
+    }
+  }
+}
+
+// Write block b of a row's terms: row r of the term arrays is token/assignment
+// `row4 / kTerms`, term `row4 % kTerms`; q rows are K/2 bytes, sf rows K/16.
+__device__ __forceinline__ void store_terms16(const uint2 (&codes)[kTerms],
+                                              const uint32_t (&sf)[kTerms], uint8_t* q,
+                                              uint8_t* sfp, size_t row4, int K, int b) {
+#pragma unroll
+  for (int t = 0; t < kTerms; ++t) {
+    *reinterpret_cast<uint2*>(q + (row4 + t) * (size_t)(K / 2) + 8 * b) = codes[t];
+    sfp[(row4 + t) * (size_t)(K / 16) + b] = (uint8_t)sf[t];
+  }
+}
+
+// Sixteen consecutive bf16 values (32 bytes, 16-byte aligned) times `sc`.
+__device__ __forceinline__ void load_bf16x16_scaled(const __nv_bfloat16* src, float sc,
+                                                    float (&r)[16]) {
+  const uint4 a = *reinterpret_cast<const uint4*>(src);
+  const uint4 b = *reinterpret_cast<const uint4*>(src + 8);
+  const uint32_t w[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[i]));
+    r[2 * i] = f.x * sc;
+    r[2 * i + 1] = f.y * sc;
+  }
+}
+
+}  // namespace moe

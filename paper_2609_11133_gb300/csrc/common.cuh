@@ -55,13 +55,25 @@ struct WsLayout {
   size_t hinv;     // f32 [T*k]
   size_t h16;      // f16 [T*k, I]
   size_t oacc;     // f32 [T, H] combine accumulator
+  // NVFP4 activation terms of the block-scaled engine (zero-sized otherwise)
+  size_t xq;       // u8 [T*4, H/2]   E2M1 codes of x
+  size_t xsf;      // u8 [T*4, H/16]  UE4M3 scales of x
+  size_t hq;       // u8 [T*k*4, I/2] E2M1 codes of h
+  size_t hsf;      // u8 [T*k*4, I/16]
   size_t total;
   int nChunks;
 };
 
 inline size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
-inline WsLayout ws_layout(int T, int k, int E, int H, int I) {
+// Rows of the h-terms array: four per assignment, and at least one full
+// down-step B box (4 x 16 rows) so that a box never extends past the array.
+inline size_t hq_rows(int T, int k) {
+  const size_t r = 4 * (size_t)T * k;
+  return r < 64 ? 64 : r;
+}
+
+inline WsLayout ws_layout(int T, int k, int E, int H, int I, bool terms = false) {
   WsLayout L{};
   size_t o = 0;
   auto take = [&](size_t bytes) {
@@ -89,6 +101,11 @@ inline WsLayout ws_layout(int T, int k, int E, int H, int I) {
   L.hinv = take(4 * TK);
   L.h16 = take(2 * TK * (size_t)I);
   L.oacc = take(4 * (size_t)T * H);
+  const size_t nt = terms ? 1 : 0;
+  L.xq = take(nt * 4 * (size_t)T * H / 2);
+  L.xsf = take(nt * 4 * (size_t)T * H / 16);
+  L.hq = take(nt * hq_rows(T, k) * (size_t)I / 2);
+  L.hsf = take(nt * 4 * TK * (size_t)I / 16);
   L.total = o;
   return L;
 }

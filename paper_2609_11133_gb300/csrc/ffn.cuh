@@ -16,7 +16,8 @@
 // * Pipeline.  One producer thread issues 2-D TMA tensor copies of each
 //   stage (two 128-row x 128-byte weight boxes with 128B swizzle, the NVFP4
 //   scale boxes, and the stage's token rows) into a ring of shared-memory
-//   stages guarded by mbarriers; eight consumer warps decode and multiply.
+//   stages guarded by mbarriers; consumer warps (eight per 128-row box, or
+//   sixteen with each stage's K split in two) decode and multiply.
 // * Decode.  E4M3 and E2M1*E4M3 values are exact in f16, so weights are
 //   converted exactly in registers (cvt e4m3x2/e2m1x2 -> f16x2; the NVFP4
 //   per-16 scale multiplied in f16, still exact).  Activations are stored
@@ -109,12 +110,17 @@ struct FfnParams {
   // activations / accumulators
   const float* xinv;   // phase 1: [T]; phase 2: hinv [T*k]
   float* gu;           // phase 1 out / phase 2 (unused)
-  __half* h16;         // phase 1 ticket output
-  float* hinv;         // phase 1 ticket output
+  __half* h16;         // SwiGLU output (warp-MMA engine)
+  float* hinv;         // SwiGLU output row scales
   float* oacc;         // phase 2 fused accumulator [T, H]
   float* y_perm;       // phase 2 unfused output [T*k, H]
   __nv_bfloat16* out;  // phase 2 fused output
   const __nv_bfloat16* residual;
+  // block-scaled engine (ffn_bs.cuh): scales of the activation terms of this
+  // phase's B operand, and the SwiGLU output as terms
+  const uint8_t* bsf;  // [rows * 4, K/16] UE4M3
+  uint8_t* hq;         // [T*k*4, I/2] E2M1 codes
+  uint8_t* hsf;        // [T*k*4, I/16] UE4M3
   uint32_t* status;
   uint64_t wait_ns;
   int test_stall;      // test hook: producer withholds its first stage
@@ -403,9 +409,7 @@ __global__ void __launch_bounds__(ffn_threads<KS>(), 1)
       }
   };
 
-  // Adds the item's partial sums to the global accumulators, then takes the
-  // item's ticket; the CTA completing an expert (phase 1) or a row tile
-  // (phase 2) finishes it.
+  // Adds the item's partial sums to the global accumulators.
   // `dead`: this warp stopped at an expired wait; it adds nothing.
   auto flush = [&](bool dead) {
     float ts0 = 1.f, ts1 = 1.f;

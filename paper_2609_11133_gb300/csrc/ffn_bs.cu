@@ -1,0 +1,39 @@
+// The block-scaled tcgen05 engine for NVFP4 weights (ffn_bs.cuh) and the
+// SwiGLU step that feeds its down projection.
+#include "ffn_bs.cuh"
+#include "ffn_launch.cuh"
+
+namespace moe {
+
+template <int NT>
+static cudaError_t launch_ffn_bs_nt(int grid, const FfnMaps& m, const FfnParams& p,
+                                    cudaStream_t st) {
+  auto kern = ffn_bs_kernel<NT>;
+  const int smem = BsGeom<NT>::SMEM;
+  static std::atomic<unsigned long long> done{0};
+  cudaError_t err = set_smem_once(kern, smem, done);
+  if (err != cudaSuccess) return err;
+  return launch_pdl(kern, dim3(grid), dim3(kBsThreads), smem, st, m.a0, m.a1, m.s0, m.s1, m.b,
+                    p);
+}
+
+cudaError_t launch_ffn_bs(int nt, int grid, const FfnMaps& m, const FfnParams& p,
+                          cudaStream_t st) {
+  switch (nt) {
+    case 8:
+      return launch_ffn_bs_nt<8>(grid, m, p, st);
+    case 16:
+      return launch_ffn_bs_nt<16>(grid, m, p, st);
+    default:
+      return cudaErrorInvalidValue;
+  }
+}
+
+cudaError_t launch_swiglu_terms(int rows, int sms, const FfnParams& p, cudaStream_t st) {
+  int blocks = rows;
+  if (blocks > 8 * sms) blocks = 8 * sms;
+  if (blocks < 1) blocks = 1;
+  return launch_pdl(swiglu_terms_kernel, dim3(blocks), dim3(128), 0, st, p, rows);
+}
+
+}  // namespace moe

@@ -3,7 +3,6 @@
 
 namespace moe {
 MOE_DEFINE_FFN_LAUNCH(1)
-MOE_DEFINE_FFN_TC_LAUNCH(1)
 MOE_DEFINE_SWIGLU_LAUNCH(1)
 cudaError_t launch_finalize(int sms, const FfnParams& p, cudaStream_t st) {
   size_t blocks = ((size_t)p.T * p.H / 4 + 255) / 256;

@@ -3,7 +3,6 @@
 #pragma once
 
 #include "ffn.cuh"
-#include "ffn_tc.cuh"
 
 namespace moe {
 
@@ -43,10 +42,11 @@ template <int FMT>
 cudaError_t launch_swiglu(int rows, int sms, const FfnParams& p, bool perm, cudaStream_t st);
 cudaError_t launch_finalize(int sms, const FfnParams& p, cudaStream_t st);
 
-// The tcgen05 engine (ffn_tc.cuh); nt in {16, 32}.
-template <int FMT>
-cudaError_t launch_ffn_tc(int nt, int grid, const FfnMaps& maps, const FfnParams& p,
+// The block-scaled tcgen05 engine for NVFP4 (ffn_bs.cuh, instantiated in
+// ffn_bs.cu); nt in {8, 16}.  SwiGLU into NVFP4 terms for its down step.
+cudaError_t launch_ffn_bs(int nt, int grid, const FfnMaps& maps, const FfnParams& p,
                           cudaStream_t st);
+cudaError_t launch_swiglu_terms(int rows, int sms, const FfnParams& p, cudaStream_t st);
 
 
 #define MOE_DEFINE_FFN_LAUNCH(FMTV)                                                            \
@@ -100,31 +100,6 @@ cudaError_t launch_ffn_tc(int nt, int grid, const FfnMaps& maps, const FfnParams
     if (blocks < 1) blocks = 1;                                                                 \
     return launch_pdl(swiglu_kernel<FMTV>, dim3(blocks), dim3(256), 0, st, p, rows,            \
                       perm ? 1 : 0);                                                            \
-  }
-
-#define MOE_DEFINE_FFN_TC_LAUNCH(FMTV)                                                         \
-  template <int NT>                                                                             \
-  static cudaError_t launch_ffn_tc_nt_##FMTV(int grid, const FfnMaps& m, const FfnParams& p,   \
-                                             cudaStream_t st) {                                 \
-    auto kern = ffn_tc_kernel<FMTV, NT>;                                                        \
-    const int smem = TcGeom<FMTV, NT>::SMEM;                                                    \
-    static std::atomic<unsigned long long> done{0};                                             \
-    cudaError_t err = set_smem_once(kern, smem, done);                                          \
-    if (err != cudaSuccess) return err;                                                         \
-    return launch_pdl(kern, dim3(grid), dim3(kTcThreads), smem, st, m.a0, m.a1, m.s0, m.s1,   \
-                      m.b, p);                                                                  \
-  }                                                                                             \
-  template <>                                                                                   \
-  cudaError_t launch_ffn_tc<FMTV>(int nt, int grid, const FfnMaps& m, const FfnParams& p,      \
-                                  cudaStream_t st) {                                            \
-    switch (nt) {                                                                               \
-      case 16:                                                                                  \
-        return launch_ffn_tc_nt_##FMTV<16>(grid, m, p, st);                                     \
-      case 32:                                                                                  \
-        return launch_ffn_tc_nt_##FMTV<32>(grid, m, p, st);                                     \
-      default:                                                                                  \
-        return cudaErrorInvalidValue;                                                           \
-    }                                                                                           \
   }
 
 }  // namespace moe

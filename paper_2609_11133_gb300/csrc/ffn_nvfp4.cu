@@ -4,6 +4,5 @@
 
 namespace moe {
 MOE_DEFINE_FFN_LAUNCH(2)
-MOE_DEFINE_FFN_TC_LAUNCH(2)
 MOE_DEFINE_SWIGLU_LAUNCH(2)
 }  // namespace moe

@@ -1,5 +1,6 @@
 // Router GEMV + top-k, permutation / work plan, and the small elementwise
 // kernels (activation conversion, combine) of the MoE decode layer.
+#include "act_terms.cuh"
 #include "ffn.cuh"
 #include "route.cuh"
 
@@ -42,8 +43,8 @@ __device__ void convert_row_x16(const __nv_bfloat16* row, int H, __half* dst, fl
   if (lane == 0) *inv = 1.f / sc;
 }
 
-// perm: store the 16-byte units in the order of the warp-MMA engine (ffn.cuh);
-// the tcgen05 engine reads rows in natural order.
+// perm: store the 16-byte units in the order of the warp-MMA NVFP4 engine
+// (ffn.cuh); FP8 reads rows in natural order.
 __device__ __forceinline__ void convert_row_dispatch(int fmt, const __nv_bfloat16* row, int H,
                                                      __half* dst, float* inv, int lane,
                                                      bool perm) {
@@ -51,6 +52,70 @@ __device__ __forceinline__ void convert_row_dispatch(int fmt, const __nv_bfloat1
     convert_row_x16<2>(row, H, dst, inv, lane, perm);
   else
     convert_row_x16<1>(row, H, dst, inv, lane, perm);
+}
+
+// The NVFP4 terms of a chunk of token rows staged in shared memory (xs, nt
+// rows of H bf16): every CTA of the chunk encodes an equal share of the
+// 16-element blocks (`part` of `nparts`); every CTA derives the rows' scale.
+__device__ void convert_chunk_terms(const __nv_bfloat16* xs, int nt, int H, int t0, int part,
+                                    int nparts, uint8_t* xq, uint8_t* xsf, float* xinv) {
+  __shared__ float s_sc[kRouteTok];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (warp < nt) {
+    float amax = 0.f;
+    for (int h = lane * 8; h < H; h += 256) {
+      const uint4 v = *reinterpret_cast<const uint4*>(xs + (size_t)warp * H + h);
+      const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const float2 f = __bfloat1622float2(b[i]);
+        amax = fmaxf(amax, fmaxf(fabsf(f.x), fabsf(f.y)));
+      }
+    }
+    amax = warp_max(amax);
+    const float sc = pow2_scale_terms(amax);
+    if (lane == 0) {
+      s_sc[warp] = sc;
+      if (part == 0) xinv[t0 + warp] = 1.f / sc;
+    }
+  }
+  __syncthreads();
+  const int nb = H / 16;
+  for (int idx = part * blockDim.x + threadIdx.x; idx < nt * nb; idx += nparts * blockDim.x) {
+    const int j = idx / nb, b = idx - j * nb;
+    float r[16];
+    load_bf16x16_scaled(xs + (size_t)j * H + 16 * b, s_sc[j], r);
+    uint2 codes[kTerms];
+    uint32_t sf[kTerms];
+    encode_terms16(r, codes, sf);
+    store_terms16(codes, sf, xq, xsf, (size_t)(t0 + j) * kTerms, H, b);
+  }
+}
+
+// The NVFP4 terms of one token row in global memory, by one warp.
+__device__ void convert_row_terms(const __nv_bfloat16* row, int H, int t, uint8_t* xq,
+                                  uint8_t* xsf, float* inv, int lane) {
+  float amax = 0.f;
+  for (int h = lane * 8; h < H; h += 256) {
+    const uint4 v = *reinterpret_cast<const uint4*>(row + h);
+    const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 f = __bfloat1622float2(b[i]);
+      amax = fmaxf(amax, fmaxf(fabsf(f.x), fabsf(f.y)));
+    }
+  }
+  amax = warp_max(amax);
+  const float sc = pow2_scale_terms(amax);
+  for (int b = lane; b < H / 16; b += 32) {
+    float r[16];
+    load_bf16x16_scaled(row + 16 * b, sc, r);
+    uint2 codes[kTerms];
+    uint32_t sf[kTerms];
+    encode_terms16(r, codes, sf);
+    store_terms16(codes, sf, xq, xsf, (size_t)t * kTerms, H, b);
+  }
+  if (lane == 0) *inv = 1.f / sc;
 }
 
 __device__ __forceinline__ unsigned lanemask_lt() {
@@ -220,10 +285,14 @@ __global__ void __launch_bounds__(256) route_kernel(const RouteParams p) {
     for (int h = lane; h < H; h += 32) row[h] = __float2bfloat16_rn(__bfloat162float(row[h]) * r);
   }
   __syncthreads();
-  if (p.fused && eb == 0 && warp < nt) {
-    const int t = t0 + warp;
-    convert_row_dispatch(p.fmt, xs + (size_t)warp * H, H, p.x16 + (size_t)t * H, p.xinv + t,
-                         lane, p.unit_perm != 0);
+  if (p.fused) {
+    if (p.act == kActTerms) {
+      convert_chunk_terms(xs, nt, H, t0, eb, gridDim.x, p.xq, p.xsf, p.xinv);
+    } else if (eb == 0 && warp < nt) {
+      const int t = t0 + warp;
+      convert_row_dispatch(p.fmt, xs + (size_t)warp * H, H, p.x16 + (size_t)t * H, p.xinv + t,
+                           lane, p.act == kActF16Perm);
+    }
   }
 
   // router GEMV: two warps per expert row (one half of H each), lanes -> 4
@@ -418,9 +487,13 @@ __global__ void __launch_bounds__(256) prep_kernel(const PrepParams p) {
     for (size_t i = tid; i < p.zero_b_n4; i += nthr) p.zero_b[i] = z;
   }
   const int t = blockIdx.x * 8 + warp;
-  if (t < p.T)
-    convert_row_dispatch(p.fmt, p.x + (size_t)t * p.H, p.H, p.x16 + (size_t)t * p.H, p.xinv + t,
-                         lane, p.unit_perm != 0);
+  if (t < p.T) {
+    if (p.act == kActTerms)
+      convert_row_terms(p.x + (size_t)t * p.H, p.H, t, p.xq, p.xsf, p.xinv + t, lane);
+    else
+      convert_row_dispatch(p.fmt, p.x + (size_t)t * p.H, p.H, p.x16 + (size_t)t * p.H,
+                           p.xinv + t, lane, p.act == kActF16Perm);
+  }
   if (blockIdx.x == 0) {
     for (int e = threadIdx.x; e < p.E; e += blockDim.x)
       p.counts[e] = __ldg(p.offsets + e + 1) - __ldg(p.offsets + e);

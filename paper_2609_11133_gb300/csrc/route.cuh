@@ -18,12 +18,17 @@ namespace moe {
 
 constexpr int kMaxK = 32;
 
+// Activation forms the expert engines read.
+constexpr int kActF16 = 0;      // f16 rows (power-of-two scaled), natural order
+constexpr int kActF16Perm = 1;  // f16 rows in the warp-MMA NVFP4 unit order
+constexpr int kActTerms = 2;    // four NVFP4 terms per row (block-scaled engine)
+
 struct RouteParams {
   const __nv_bfloat16* x;
   const float* wr;
   const float* bias;
   int T, H, E, k, renorm, prenorm, fmt, fused, nt;
-  int unit_perm;  // x16 rows in the warp-MMA engine's unit order
+  int act;  // activation form for the expert kernels (kAct*)
   float* logits;  // [T, E]
   int* ids;       // [T, k]
   float* gates;   // [T, k]
@@ -33,6 +38,8 @@ struct RouteParams {
   unsigned* done_cnt;
   // fused layer only
   __half* x16;
+  uint8_t* xq;   // NVFP4 terms of x (kActTerms)
+  uint8_t* xsf;
   float* xinv;
   float4* zero_a;
   size_t zero_a_n4;
@@ -50,8 +57,10 @@ struct RouteParams {
 struct PrepParams {
   const __nv_bfloat16* x;
   int T, H, E, k, fmt, nt;
-  int unit_perm;
+  int act;
   __half* x16;
+  uint8_t* xq;
+  uint8_t* xsf;
   float* xinv;
   const int* offsets;  // [E+1] from the permutation
   const int* active;   // [E+1]
