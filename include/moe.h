@@ -31,6 +31,15 @@
  *   range) are recorded in a status word inside the workspace and read
  *   with moe_read_status().  No exception or abort crosses the ABI.
  *
+ * Arithmetic of the GPU path: fp32 router and gates; expert products
+ * accumulate in fp32.  FP8 weights are decoded exactly to f16 and multiplied
+ * with the f16 activations (exact for bf16 inputs after a power-of-two row
+ * scale).  NVFP4 weights are fed to the tensor cores as stored (block-scaled
+ * MMA, E2M1 x UE4M3 per 16 K); the activations (x, and h between the gate/up
+ * and down steps) are encoded as sums of four NVFP4 terms per row, each term
+ * coding the previous terms' residual, which leaves less than 2^-9.5 of each
+ * 16-element block's maximum uncoded.
+ *
  * Expert weight formats (moe_expert_weights_t)
  *   gate and up are [E, I, H]-shaped (N = I rows, K = H contiguous),
  *   down is [E, H, I]-shaped (N = H rows, K = I contiguous).
@@ -180,7 +189,7 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
  *   Scratch: a 16 MiB device array inside libmoe.so; every GPU that loads the
  *     library holds it until the process exits.  Shapes whose
  *     moe_workspace_size() exceeds 16 MiB return MOE_ERR_WORKSPACE_TOO_SMALL
- *     (e.g. the 235B-shaped NVFP4 layer fits up to T = 113 tokens).
+ *     (e.g. the 235B-shaped NVFP4 layer fits up to T = 110 tokens).
  *   The first call on a device looks up the array's device address; make
  *     that first call before capturing the stream into a CUDA graph.
  *   Every call shares the one array and clears its control words itself;

@@ -310,7 +310,7 @@ int moe_workspace_size(const moe_expert_weights_t* w, int T, int k, size_t* byte
   if (rc) return rc;
   rc = check_tk(T, k, w->E);
   if (rc) return rc;
-  *bytes = ws_layout(T, k, w->E, w->H, w->I, w->fmt == MOE_FMT_NVFP4).total;
+  *bytes = ws_layout(T, k, w->E, w->H, w->I, engine_for(w->fmt) == kEngBs).total;
   return MOE_OK;
 }
 
@@ -410,7 +410,7 @@ int moe_expert_ffn(const void* x, const moe_expert_weights_t* w, const int32_t* 
   if (T == 0) return MOE_OK;
   if (!x || !offsets || !sorted_assign || !active || !y_perm || !ws) return MOE_ERR_INVALID_ARG;
   if (!aligned(x, 16) || !aligned(y_perm, 16) || !aligned(ws, 256)) return MOE_ERR_INVALID_ARG;
-  const WsLayout L = ws_layout(T, k, w->E, w->H, w->I, w->fmt == MOE_FMT_NVFP4);
+  const WsLayout L = ws_layout(T, k, w->E, w->H, w->I, engine_for(w->fmt) == kEngBs);
   if (ws_bytes < L.total) return MOE_ERR_WORKSPACE_TOO_SMALL;
   if (T == 0) return MOE_OK;
   int sms = 0;
@@ -489,7 +489,7 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
     return MOE_ERR_INVALID_ARG;
   if (out == x) return MOE_ERR_INVALID_ARG;
   const int E = w->E, H = w->H, I = w->I;
-  const WsLayout L = ws_layout(T, k, E, H, I, w->fmt == MOE_FMT_NVFP4);
+  const WsLayout L = ws_layout(T, k, E, H, I, engine_for(w->fmt) == kEngBs);
   if (ws_bytes < L.total) return MOE_ERR_WORKSPACE_TOO_SMALL;
   if (T == 0) return MOE_OK;
   int sms = 0;

@@ -55,7 +55,8 @@ struct WsLayout {
   size_t hinv;     // f32 [T*k]
   size_t h16;      // f16 [T*k, I]
   size_t oacc;     // f32 [T, H] combine accumulator
-  // NVFP4 activation terms of the block-scaled engine (zero-sized otherwise)
+  // NVFP4 activation terms of the block-scaled engine (zero-sized otherwise;
+  // x16 and h16 are zero-sized when these are used)
   size_t xq;       // u8 [T*4, H/2]   E2M1 codes of x
   size_t xsf;      // u8 [T*4, H/16]  UE4M3 scales of x
   size_t hq;       // u8 [T*k*4, I/2] E2M1 codes of h
@@ -96,16 +97,17 @@ inline WsLayout ws_layout(int T, int k, int E, int H, int I, bool terms = false)
   L.active = take(4 * (size_t)(E + 1));
   L.cprefix = take(4 * (size_t)(E + 1));
   L.xinv = take(4 * (size_t)T);
-  L.x16 = take(2 * (size_t)T * H);
+  const size_t nf = terms ? 0 : 1;  // f16 activations: warp-MMA engine only
+  L.x16 = take(nf * 2 * (size_t)T * H);
   L.gu = take(4 * TK * 2 * (size_t)I);
   L.hinv = take(4 * TK);
-  L.h16 = take(2 * TK * (size_t)I);
+  L.h16 = take(nf * 2 * TK * (size_t)I);
   L.oacc = take(4 * (size_t)T * H);
   const size_t nt = terms ? 1 : 0;
   L.xq = take(nt * 4 * (size_t)T * H / 2);
   L.xsf = take(nt * 4 * (size_t)T * H / 16);
   L.hq = take(nt * hq_rows(T, k) * (size_t)I / 2);
-  L.hsf = take(nt * 4 * TK * (size_t)I / 16);
+  L.hsf = take(nt * hq_rows(T, k) * (size_t)I / 16);
   L.total = o;
   return L;
 }

@@ -6,7 +6,7 @@
 // memory, and their E4M3 scales (128 rows x 16 bytes) next to them.  The
 // activations arrive as four NVFP4 terms per token (act_terms.cuh), i.e. four
 // rows of the B operand.  Nothing is decoded on the CUDA cores; the kernel is
-// a pure TMA -> tensor-core stream, so it can run at the HBM rate.
+// a TMA -> tensor-core stream.
 //
 // Work decomposition as in ffn.cuh: a persistent grid, stream-K over the
 // K-stages of all (active expert, <=NT-token chunk, row tile) items.  Per
