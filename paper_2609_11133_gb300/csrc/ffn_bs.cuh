@@ -13,14 +13,17 @@
 // stage and matrix (gate/up in phase 1, the two 128-row halves of down in
 // phase 2) four MMAs of M=128, N=4*NT, K=64 accumulate into tensor memory.
 //
-// Roles (320 threads):
+// Roles (352 threads):
 //   warps 0-3  scale writers: copy the stage's A scales from shared memory and
 //              the B scales from global memory into tensor memory, in the
 //              layout the MMA reads (below); warp w owns TMEM lanes 32w..32w+31
 //   warps 4-7  epilogue: read an item's accumulators (tcgen05.ld), add the
 //              four terms of each token, apply the tensor and activation
 //              scales and add the partial sums to global memory (red.add)
-//   warp 8     TMA producer (one thread)
+//   warps 8,10 TMA producers (one thread each): warp 8 arms each stage's
+//              barrier and copies box A0 and its scales, warp 10 box A1, its
+//              scales and the activation rows (two issuing warps keep more
+//              copies going than one)
 //   warp 9     MMA issuer (one thread); allocates and frees tensor memory
 //
 // Scale-factor layout in tensor memory (scale_vec::4X, M = 128): the four
@@ -38,8 +41,9 @@
 
 namespace moe {
 
-constexpr int kBsThreads = 10 * 32;
+constexpr int kBsThreads = 11 * 32;
 constexpr int kBsSfWarp0 = 0, kBsEpiWarp0 = 4, kBsProducerWarp = 8, kBsMmaWarp = 9;
+constexpr int kBsProducerWarp2 = 10;
 constexpr uint32_t kBsTmemCols = 512;
 constexpr int kBsSfCols = 48;  // per stage: A scales 2 x 16 columns, B scales 16
 
@@ -157,7 +161,8 @@ __global__ void __launch_bounds__(kBsThreads, 1)
   constexpr int kTeardown = 9 * 32;  // scale writers, epilogue and MMA warps
 
   // ================================================================ producer
-  if (warp == kBsProducerWarp) {
+  if (warp == kBsProducerWarp || warp == kBsProducerWarp2) {
+    const bool lead = (warp == kBsProducerWarp);
     if (lane == 0 && nst > 0) {
       tma_prefetch_desc(&tmA0);
       tma_prefetch_desc(&tmA1);
@@ -175,7 +180,7 @@ __global__ void __launch_bounds__(kBsThreads, 1)
         if (it != cur_item) {
           cur_item = it;
           inf = decode_item(it, rtiles, s_cpre, nA, p, NT);
-          if (p.phase == 1)
+          if (!lead && p.phase == 1)
             for (int j = 0; j < inf.nvalid; ++j) s_tok[j] = __ldg(p.sorted + inf.arow0 + j) / p.k;
         }
         const int slot = (int)(issued % S);
@@ -190,7 +195,10 @@ __global__ void __launch_bounds__(kBsThreads, 1)
         uint32_t bytes = 2u * kRowsHalf * kRowBytes + 2u * kRowsHalf * 16u;
         bytes += (p.phase == 1) ? (uint32_t)inf.nvalid * kTerms * kRowBytes
                                 : (uint32_t)BN * kRowBytes;
-        mbar_arrive_expect_tx(&full_bar[slot], bytes);
+        // the second producer's copies may land before this arms the barrier:
+        // the transaction count then dips below zero, and the phase still
+        // cannot complete before the arrival below
+        if (lead) mbar_arrive_expect_tx(&full_bar[slot], bytes);
         int rowA0, rowA1;
         if (p.phase == 1) {
           rowA0 = inf.e * N + inf.rt * kRowsHalf;
@@ -199,9 +207,12 @@ __global__ void __launch_bounds__(kBsThreads, 1)
           rowA0 = inf.e * N + inf.rt * 2 * kRowsHalf;
           rowA1 = rowA0 + kRowsHalf;
         }
-        tma_load_2d(st + G::A0, &tmA0, &full_bar[slot], kb * kRowBytes, rowA0, pol_w);
+        if (lead) {
+          tma_load_2d(st + G::A0, &tmA0, &full_bar[slot], kb * kRowBytes, rowA0, pol_w);
+          tma_load_2d(st + G::S0, &tmS0, &full_bar[slot], kb * 16, rowA0, pol_w);
+          continue;
+        }
         tma_load_2d(st + G::A1, &tmA1, &full_bar[slot], kb * kRowBytes, rowA1, pol_w);
-        tma_load_2d(st + G::S0, &tmS0, &full_bar[slot], kb * 16, rowA0, pol_w);
         tma_load_2d(st + G::S1, &tmS1, &full_bar[slot], kb * 16, rowA1, pol_w);
         // activation terms: token j's four rows land at B rows 4j..4j+3
         if (p.phase == 1) {
@@ -213,7 +224,9 @@ __global__ void __launch_bounds__(kBsThreads, 1)
                       pol_a);
         }
       }
-      // Let every copy this CTA issued land before the CTA exits.
+      // Let every copy this CTA issued land before the CTA exits (the
+      // barriers complete only when both producers' copies have landed).
+      if (!lead) return;
       const long long first = issued > S ? issued - S : 0;
       for (long long j = first; j < issued; ++j) {
         if (p.test_stall && j == 0) continue;
