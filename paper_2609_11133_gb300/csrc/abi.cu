@@ -136,6 +136,12 @@ int nt_for(int T, int eng) {
   return T <= 64 ? 8 : 32;
 }
 
+// Experts per router CTA: small batches spread the router rows over more
+// CTAs (one expert per CTA, its row split over 8 warps); larger ones keep
+// four experts per CTA so that the token rows staged in shared memory are
+// reused.
+int route_epb(int T) { return T <= 16 ? 1 : 4; }
+
 // ------------------------------------------------------------------ validation
 int check_weights(const moe_expert_weights_t* w) {
   if (!w) return MOE_ERR_INVALID_ARG;
@@ -169,8 +175,9 @@ struct ExpertRun {
   int T, k, nt, sms;
   void* ws;
   WsLayout L;
-  const int *offsets, *sorted, *active;  // plan inputs (ws or caller)
-  const int* counts;
+  const int* sorted;  // assignment lists (see FfnParams::list_T)
+  int list_T;
+  const int* counts;  // tokens per expert
   const float* gates;
   int fused;
   float* y_perm;
@@ -225,10 +232,8 @@ int run_experts(const ExpertRun& r, cudaStream_t st, cudaEvent_t ev_mid) {
   p.H = H;
   p.I = I;
   p.counts = r.counts;
-  p.offsets = r.offsets;
   p.sorted = r.sorted;
-  p.active = r.active;
-  p.cprefix = ws_ptr<int>(r.ws, r.L.cprefix);
+  p.list_T = r.list_T;
   p.gates = r.gates;
   p.status = ws_ptr<uint32_t>(r.ws, r.L.status);
   p.wait_ns = wait_limit_ns();
@@ -261,6 +266,7 @@ int run_experts(const ExpertRun& r, cudaStream_t st, cudaEvent_t ev_mid) {
   p2.out = r.out;
   p2.residual = r.residual;
   p2.bsf = ws_ptr<uint8_t>(r.ws, r.L.hsf);
+  p2.acnt_reset = r.list_T ? ws_ptr<uint32_t>(r.ws, r.L.acnt) : nullptr;
 
   auto launch = [&](const FfnMaps& m, const FfnParams& pp) {
     if (eng == kEngBs) return launch_ffn_bs(r.nt, r.sms, m, pp, st);
@@ -379,8 +385,7 @@ int moe_route_topk(const void* x, const float* router_w, const float* router_bia
   p.ids = topk_ids;
   p.gates = topk_w;
   p.chunk_cnt = ws_ptr<unsigned>(ws, L.route_chunk);
-  p.done_cnt = ws_ptr<unsigned>(ws, L.route_done);
-  p.status = ws_ptr<uint32_t>(ws, L.status);
+  p.epb = route_epb(T);
   return launch_route(p, (cudaStream_t)stream) == cudaSuccess ? MOE_OK : MOE_ERR_CUDA;
 }
 
@@ -426,16 +431,13 @@ int moe_expert_ffn(const void* x, const moe_expert_weights_t* w, const int32_t* 
   pp.E = w->E;
   pp.k = k;
   pp.fmt = w->fmt;
-  pp.nt = nt;
   pp.act = act_for(w->fmt, eng);
   pp.x16 = ws_ptr<__half>(ws, L.x16);
   pp.xq = ws_ptr<uint8_t>(ws, L.xq);
   pp.xsf = ws_ptr<uint8_t>(ws, L.xsf);
   pp.xinv = ws_ptr<float>(ws, L.xinv);
   pp.offsets = offsets;
-  pp.active = active;
   pp.counts = ws_ptr<int>(ws, L.counts);
-  pp.cprefix = ws_ptr<int>(ws, L.cprefix);
   pp.zero_a = reinterpret_cast<float4*>(y_perm);
   pp.zero_a_n4 = (size_t)T * k * w->H / 4;
   pp.zero_b = ws_ptr<float4>(ws, L.gu);
@@ -449,9 +451,8 @@ int moe_expert_ffn(const void* x, const moe_expert_weights_t* w, const int32_t* 
   r.sms = sms;
   r.ws = ws;
   r.L = L;
-  r.offsets = offsets;
   r.sorted = sorted_assign;
-  r.active = active;
+  r.list_T = 0;
   r.counts = ws_ptr<int>(ws, L.counts);
   r.fused = 0;
   r.y_perm = y_perm;
@@ -514,7 +515,7 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
   p.prenorm = (flags & MOE_FLAG_PRENORM_RMS) ? 1 : 0;
   p.fmt = w->fmt;
   p.fused = 1;
-  p.nt = nt;
+  p.epb = route_epb(T);
   p.act = act_for(w->fmt, eng);
   p.logits = logits_out ? logits_out : ws_ptr<float>(ws, L.logits);
   p.ids = ws_ptr<int>(ws, L.ids);
@@ -522,7 +523,6 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
   p.ids2 = topk_ids_out;
   p.gates2 = topk_w_out;
   p.chunk_cnt = ws_ptr<unsigned>(ws, L.route_chunk);
-  p.done_cnt = ws_ptr<unsigned>(ws, L.route_done);
   p.x16 = ws_ptr<__half>(ws, L.x16);
   p.xq = ws_ptr<uint8_t>(ws, L.xq);
   p.xsf = ws_ptr<uint8_t>(ws, L.xsf);
@@ -531,13 +531,8 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
   p.zero_a_n4 = (size_t)T * k * 2 * I / 4;
   p.zero_b = ws_ptr<float4>(ws, L.oacc);
   p.zero_b_n4 = (size_t)T * H / 4;
-  p.counts = ws_ptr<int>(ws, L.counts);
-  p.offsets = ws_ptr<int>(ws, L.offsets);
-  p.sorted = ws_ptr<int>(ws, L.sorted);
-  p.inv = ws_ptr<int>(ws, L.inv);
-  p.active = ws_ptr<int>(ws, L.active);
-  p.cprefix = ws_ptr<int>(ws, L.cprefix);
-  p.status = ws_ptr<uint32_t>(ws, L.status);
+  p.acnt = ws_ptr<unsigned>(ws, L.acnt);
+  p.alist = ws_ptr<int>(ws, L.alist);
   if (ev[0] && cudaEventRecord(ev[0], st) != cudaSuccess) return MOE_ERR_CUDA;
   if (launch_route(p, st) != cudaSuccess) return MOE_ERR_CUDA;
   if (ev[1] && cudaEventRecord(ev[1], st) != cudaSuccess) return MOE_ERR_CUDA;
@@ -550,10 +545,9 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
   r.sms = sms;
   r.ws = ws;
   r.L = L;
-  r.offsets = p.offsets;
-  r.sorted = p.sorted;
-  r.active = p.active;
-  r.counts = p.counts;
+  r.sorted = p.alist;
+  r.list_T = 1;
+  r.counts = reinterpret_cast<const int*>(p.acnt);
   r.gates = p.gates;
   r.fused = 1;
   r.out = static_cast<__nv_bfloat16*>(out);

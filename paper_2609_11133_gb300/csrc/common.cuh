@@ -20,7 +20,6 @@ constexpr int kMaxTK = 65536;       // T * k
 constexpr int kMaxHI = 32768;       // H and I
 constexpr int kRouteTok = 8;        // tokens per router CTA
 constexpr int kRouteWarps = 8;      // warps per router CTA
-constexpr int kRouteEPB = 4;        // expert rows per router CTA (two warps each)
 
 // Device status bits (the first error wins; see moe_read_status).
 constexpr uint32_t kStatusTimeoutGateUp = 1u;
@@ -36,18 +35,14 @@ constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s
 struct WsLayout {
   // control block (zeroed once; every counter is reset by its last user)
   size_t status;       // u32 device status word
+  size_t acnt;         // u32 [kMaxE] assignments per expert (fused layer)
   size_t route_chunk;  // u32 [nChunks] per-token-chunk arrival tickets
-  size_t route_done;   // u32 chunk-completion ticket
   // routing
   size_t logits;   // f32 [T, E]
   size_t ids;      // i32 [T, k]
   size_t gates;    // f32 [T, k]
-  size_t counts;   // i32 [E]
-  size_t offsets;  // i32 [E+1]
-  size_t sorted;   // i32 [T*k]
-  size_t inv;      // i32 [T*k]
-  size_t active;   // i32 [E+1]
-  size_t cprefix;  // i32 [E+1] token-chunk prefix over active experts
+  size_t counts;   // i32 [E] tokens per expert (moe_expert_ffn)
+  size_t alist;    // i32 [E, T] per-expert assignment lists (fused layer)
   // activations
   size_t xinv;     // f32 [T]   power-of-two inverse scale of x16 rows
   size_t x16;      // f16 [T, H]
@@ -85,17 +80,13 @@ inline WsLayout ws_layout(int T, int k, int E, int H, int I, bool terms = false)
   L.nChunks = (T + kRouteTok - 1) / kRouteTok;
   const size_t TK = (size_t)T * k;
   L.status = take(4);
+  L.acnt = take(4 * (size_t)kMaxE);  // fixed size: the same offset for every T and E
   L.route_chunk = take(4 * (size_t)(L.nChunks > 0 ? L.nChunks : 1));
-  L.route_done = take(4);
   L.logits = take(4 * (size_t)T * E);
   L.ids = take(4 * TK);
   L.gates = take(4 * TK);
   L.counts = take(4 * (size_t)E);
-  L.offsets = take(4 * (size_t)(E + 1));
-  L.sorted = take(4 * TK);
-  L.inv = take(4 * TK);
-  L.active = take(4 * (size_t)(E + 1));
-  L.cprefix = take(4 * (size_t)(E + 1));
+  L.alist = take(4 * (size_t)E * T);
   L.xinv = take(4 * (size_t)T);
   const size_t nf = terms ? 0 : 1;  // f16 activations: warp-MMA engine only
   L.x16 = take(nf * 2 * (size_t)T * H);

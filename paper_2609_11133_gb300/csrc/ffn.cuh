@@ -87,7 +87,7 @@ struct StageGeom {
   static constexpr int BROW = KEL * 2;                               // bytes per token row
   static constexpr int RAW = B + NT * BROW;
   static constexpr int BYTES = (RAW + 1023) / 1024 * 1024;
-  static constexpr int STAGES_RAW = (220 * 1024) / BYTES;
+  static constexpr int STAGES_RAW = (212 * 1024) / BYTES;  // + ~10 KB static
   static constexpr int STAGES = STAGES_RAW > 8 ? 8 : STAGES_RAW;
   static constexpr int SMEM = STAGES * BYTES + 1024;  // + alignment slack
 };
@@ -95,13 +95,14 @@ struct StageGeom {
 struct FfnParams {
   int T, k, E, H, I, phase;  // phase 1 = gate/up, 2 = down
   int fused;                 // phase 2: 1 = scatter into oacc + bf16 out, 0 = y_perm
-  // routing plan (device)
-  const int* counts;
-  const int* offsets;
+  // routing: tokens per expert, and each expert's assignments (t*k + j).
+  // list_T = 1: expert e's list starts at sorted[e*T] (the fused layer's
+  // per-expert lists); 0: at sorted[offsets[e]] (one array sorted by expert).
+  const int* counts;   // [E]
   const int* sorted;
-  const int* active;
-  const int* cprefix;
+  int list_T;
   const float* gates;  // [T*k] by assignment (fused only)
+  uint32_t* acnt_reset;  // finalize_kernel zeroes these E counters (fused only)
   // scales
   const float* s0;     // FP8 block scales of the matrix behind box A0/A1
   const float* s1;
@@ -126,27 +127,80 @@ struct FfnParams {
   int test_stall;      // test hook: producer withholds its first stage
 };
 
-// ------------------------------------------------------------------ item decode
-struct ItemInfo {
-  int slot, e, arow0, nvalid, rt;
+// ------------------------------------------------------------------ work plan
+// The expert kernels build their work plan from the per-expert token counts
+// in shared memory: the active experts in increasing id order, their first
+// row in the compact [T*k] row space (rows ordered by expert), and the prefix
+// of their NT-token chunks, which numbers the items.
+struct PlanSmem {
+  int act[kMaxE];       // active expert ids, increasing
+  int acnt[kMaxE];      // their token counts
+  int aoff[kMaxE];      // their first compact row
+  int cpre[kMaxE + 1];  // chunk prefix; cpre[nA] = total chunks
+  int nA;
 };
 
-__device__ __forceinline__ ItemInfo decode_item(long long it, int rtiles, const int* s_cpre,
-                                                int nA, const FfnParams& p, int NT) {
+// One warp: scan the counts in groups of 32 (inclusive warp scans carried
+// across groups).  The caller synchronises the block afterwards.
+__device__ __forceinline__ void build_plan(const int* counts, int E, int NT, PlanSmem& pl,
+                                           int lane) {
+  int run_off = 0, run_act = 0, run_ch = 0;
+  unsigned lt;
+  asm("mov.u32 %0, %%lanemask_lt;" : "=r"(lt));
+  for (int base = 0; base < E; base += 32) {
+    const int e = base + lane;
+    const int c = (e < E) ? __ldcg(counts + e) : 0;
+    const int ch = (c + NT - 1) / NT;
+    int oc = c, och = ch;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y0 = __shfl_up_sync(0xffffffffu, oc, o);
+      const int y1 = __shfl_up_sync(0xffffffffu, och, o);
+      if (lane >= o) {
+        oc += y0;
+        och += y1;
+      }
+    }
+    const unsigned am = __ballot_sync(0xffffffffu, c > 0);
+    if (c > 0) {
+      const int slot = run_act + __popc(am & lt);
+      pl.act[slot] = e;
+      pl.acnt[slot] = c;
+      pl.aoff[slot] = run_off + oc - c;
+      pl.cpre[slot] = run_ch + och - ch;
+    }
+    run_off += __shfl_sync(0xffffffffu, oc, 31);
+    run_ch += __shfl_sync(0xffffffffu, och, 31);
+    run_act += __popc(am);
+  }
+  if (lane == 0) {
+    pl.nA = run_act;
+    pl.cpre[run_act] = run_ch;
+  }
+}
+
+struct ItemInfo {
+  int slot, e, arow0, lrow0, nvalid, rt;
+};
+
+// Item `it` = (chunk of an active expert, row tile): arow0 is the chunk's
+// first compact row, lrow0 the index of its first assignment in p.sorted.
+__device__ __forceinline__ ItemInfo decode_item(long long it, int rtiles, const PlanSmem& pl,
+                                                const FfnParams& p, int NT) {
   ItemInfo r;
   const int chunk_g = (int)(it / rtiles);
   r.rt = (int)(it % rtiles);
-  int lo = 0, hi = nA - 1;  // last slot with cprefix[slot] <= chunk_g
+  int lo = 0, hi = pl.nA - 1;  // last slot with cpre[slot] <= chunk_g
   while (lo < hi) {
     const int mid = (lo + hi + 1) >> 1;
-    if (s_cpre[mid] <= chunk_g) lo = mid; else hi = mid - 1;
+    if (pl.cpre[mid] <= chunk_g) lo = mid; else hi = mid - 1;
   }
   r.slot = lo;
-  const int chunk = chunk_g - s_cpre[lo];
-  r.e = __ldg(p.active + 1 + lo);
-  const int n_e = __ldg(p.counts + r.e);
-  r.arow0 = __ldg(p.offsets + r.e) + chunk * NT;
-  const int rem = n_e - chunk * NT;
+  const int chunk = chunk_g - pl.cpre[lo];
+  r.e = pl.act[lo];
+  r.arow0 = pl.aoff[lo] + chunk * NT;
+  r.lrow0 = (p.list_T ? r.e * p.T : pl.aoff[lo]) + chunk * NT;
+  const int rem = pl.acnt[lo] - chunk * NT;
   r.nvalid = rem < NT ? rem : NT;
   return r;
 }
@@ -213,6 +267,9 @@ __global__ void __launch_bounds__(256) swiglu_kernel(const FfnParams p, int rows
 // out = bf16(oacc + residual), four columns per thread.
 static __global__ void __launch_bounds__(256) finalize_kernel(const FfnParams p) {
   pdl_wait();
+  // the per-expert assignment counters start the next layer call from zero
+  if (p.acnt_reset && blockIdx.x == 0)
+    for (int e = threadIdx.x; e < p.E; e += blockDim.x) p.acnt_reset[e] = 0u;
   const size_t n4 = (size_t)p.T * p.H / 4;
   for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4;
        i += (size_t)gridDim.x * blockDim.x) {
@@ -252,7 +309,7 @@ __global__ void __launch_bounds__(ffn_threads<KS>(), 1)
 
   __shared__ __align__(8) uint64_t full_bar[S];
   __shared__ __align__(8) uint64_t empty_bar[S];
-  __shared__ int s_cpre[kMaxE + 1];
+  __shared__ PlanSmem pl;
   __shared__ int s_tok[NT];
   __shared__ volatile int s_abort;
 
@@ -272,15 +329,14 @@ __global__ void __launch_bounds__(ffn_threads<KS>(), 1)
   // previous kernel; from here on its outputs are read.
   pdl_wait();
   pdl_launch_dependents();
-  const int nA = __ldg(p.active);
-  for (int i = threadIdx.x; i <= nA; i += blockDim.x) s_cpre[i] = __ldg(p.cprefix + i);
+  if (warp == 0) build_plan(p.counts, p.E, NT, pl, lane);
   __syncthreads();
 
   const int N = (p.phase == 1) ? p.I : p.H;       // rows of one expert matrix
   const int K = (p.phase == 1) ? p.H : p.I;       // contraction length
   const int rtiles = (p.phase == 1) ? p.I / kRowsHalf : p.H / (2 * kRowsHalf);
   const int KB = K / KEL;
-  const long long items = (long long)s_cpre[nA] * rtiles;
+  const long long items = (long long)pl.cpre[pl.nA] * rtiles;
   const long long total = items * KB;
   const long long s_begin = total * blockIdx.x / gridDim.x;
   const long long s_end = total * (blockIdx.x + 1) / gridDim.x;
@@ -305,9 +361,9 @@ __global__ void __launch_bounds__(ffn_threads<KS>(), 1)
         const int kb = (int)(s % KB);
         if (it != cur_item) {
           cur_item = it;
-          inf = decode_item(it, rtiles, s_cpre, nA, p, NT);
+          inf = decode_item(it, rtiles, pl, p, NT);
           if (p.phase == 1)
-            for (int j = 0; j < inf.nvalid; ++j) s_tok[j] = __ldg(p.sorted + inf.arow0 + j) / p.k;
+            for (int j = 0; j < inf.nvalid; ++j) s_tok[j] = __ldg(p.sorted + inf.lrow0 + j) / p.k;
         }
         const int slot = (int)(issued % S);
         const uint32_t round = (uint32_t)(issued / S);
@@ -391,7 +447,7 @@ __global__ void __launch_bounds__(ffn_threads<KS>(), 1)
         colgate[n][c] = 0.f;
         if (j < inf.nvalid) {
           const int arow = inf.arow0 + j;
-          const int a = __ldg(p.sorted + arow);
+          const int a = __ldg(p.sorted + inf.lrow0 + j);
           if (p.phase == 1) {
             colscale[n][c] = __ldg(p.xinv + a / p.k);
             colrow[n][c] = arow;
@@ -457,7 +513,7 @@ __global__ void __launch_bounds__(ffn_threads<KS>(), 1)
         zero_acc();
       }
       cur_item = it;
-      inf = decode_item(it, rtiles, s_cpre, nA, p, NT);
+      inf = decode_item(it, rtiles, pl, p, NT);
       load_item_cols();
     }
     if (dead) continue;

@@ -57,7 +57,7 @@ struct BsGeom {
   static constexpr int B = S0 + 2 * kRowsHalf * 16;            // 36 KB, 1024-aligned
   static constexpr int RAW = B + BN * kRowBytes;
   static constexpr int BYTES = (RAW + 1023) / 1024 * 1024;
-  static constexpr int STAGES_RAW = (220 * 1024) / BYTES;
+  static constexpr int STAGES_RAW = (212 * 1024) / BYTES;  // + ~10 KB static
   static constexpr int STAGES = STAGES_RAW > 8 ? 8 : STAGES_RAW;
   static constexpr int SMEM = STAGES * BYTES + 1024;
   // tensor memory: accumulators D[db][mat] (BN columns each), then per-stage scales
@@ -112,7 +112,7 @@ __global__ void __launch_bounds__(kBsThreads, 1)
   __shared__ __align__(8) uint64_t dfull_bar[2];
   __shared__ __align__(8) uint64_t dempty_bar[2];
   __shared__ __align__(8) uint64_t final_bar;
-  __shared__ int s_cpre[kMaxE + 1];
+  __shared__ PlanSmem pl;
   __shared__ int s_tok[NT];
   __shared__ uint32_t s_tmem;
   __shared__ volatile int s_abort;
@@ -141,8 +141,7 @@ __global__ void __launch_bounds__(kBsThreads, 1)
   // previous kernel; from here on its outputs are read.
   pdl_wait();
   pdl_launch_dependents();
-  const int nA = __ldg(p.active);
-  for (int i = threadIdx.x; i <= nA; i += blockDim.x) s_cpre[i] = __ldg(p.cprefix + i);
+  if (warp == 0) build_plan(p.counts, p.E, NT, pl, lane);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -152,7 +151,7 @@ __global__ void __launch_bounds__(kBsThreads, 1)
   const int K = (p.phase == 1) ? p.H : p.I;  // contraction length
   const int rtiles = (p.phase == 1) ? p.I / kRowsHalf : p.H / (2 * kRowsHalf);
   const int KB = K / KEL;
-  const long long items = (long long)s_cpre[nA] * rtiles;
+  const long long items = (long long)pl.cpre[pl.nA] * rtiles;
   const long long total = items * KB;
   const long long s_begin = total * blockIdx.x / gridDim.x;
   const long long s_end = total * (blockIdx.x + 1) / gridDim.x;
@@ -179,9 +178,9 @@ __global__ void __launch_bounds__(kBsThreads, 1)
         const int kb = (int)(s % KB);
         if (it != cur_item) {
           cur_item = it;
-          inf = decode_item(it, rtiles, s_cpre, nA, p, NT);
+          inf = decode_item(it, rtiles, pl, p, NT);
           if (!lead && p.phase == 1)
-            for (int j = 0; j < inf.nvalid; ++j) s_tok[j] = __ldg(p.sorted + inf.arow0 + j) / p.k;
+            for (int j = 0; j < inf.nvalid; ++j) s_tok[j] = __ldg(p.sorted + inf.lrow0 + j) / p.k;
         }
         const int slot = (int)(issued % S);
         const uint32_t round = (uint32_t)(issued / S);
@@ -304,14 +303,14 @@ __global__ void __launch_bounds__(kBsThreads, 1)
       const int kb = (int)(s % KB);
       if (it != cur_item) {
         cur_item = it;
-        inf = decode_item(it, rtiles, s_cpre, nA, p, NT);
+        inf = decode_item(it, rtiles, pl, p, NT);
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
           const int n = lane + 32 * h;
           const int j = n / kTerms;
           grow[h] = -1;
           if (n < BN && j < inf.nvalid) {
-            const int base = (p.phase == 1) ? __ldg(p.sorted + inf.arow0 + j) / p.k
+            const int base = (p.phase == 1) ? __ldg(p.sorted + inf.lrow0 + j) / p.k
                                             : inf.arow0 + j;
             grow[h] = base * kTerms + n % kTerms;
           }
@@ -388,7 +387,7 @@ __global__ void __launch_bounds__(kBsThreads, 1)
     if (nst > 0) {
       const long long it0 = s_begin / KB, it1 = (s_end - 1) / KB;
       for (long long it = it0; it <= it1 && !dead; ++it, ++nitem) {
-        const ItemInfo inf = decode_item(it, rtiles, s_cpre, nA, p, NT);
+        const ItemInfo inf = decode_item(it, rtiles, pl, p, NT);
         const int db = (int)(nitem & 1);
         if (!mbar_wait_bounded(&dfull_bar[db], (uint32_t)(nitem >> 1) & 1u, p.wait_ns,
                                &s_abort)) {
@@ -422,7 +421,7 @@ __global__ void __launch_bounds__(kBsThreads, 1)
         for (int j = 0; j < NT; ++j) {
           if (j >= inf.nvalid) continue;
           const int arow = inf.arow0 + j;
-          const int a = __ldg(p.sorted + arow);
+          const int a = __ldg(p.sorted + inf.lrow0 + j);
           if (p.phase == 1) {
             const float sc = __ldg(p.xinv + a / p.k);
             const int f = inf.rt * kRowsHalf + row;

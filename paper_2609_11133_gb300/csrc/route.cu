@@ -118,26 +118,29 @@ __device__ void convert_row_terms(const __nv_bfloat16* row, int H, int t, uint8_
   if (lane == 0) *inv = 1.f / sc;
 }
 
+// Order-preserving unsigned key of a finite float (larger value, larger key;
+// -0 maps like +0), and its inverse.  Keys of finite values are never 0.
+__device__ __forceinline__ unsigned logit_key(float v) {
+  const unsigned b = __float_as_uint(v == 0.f ? 0.f : v);
+  return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+__device__ __forceinline__ float key_logit(unsigned k) {
+  return __uint_as_float((k & 0x80000000u) ? (k & 0x7fffffffu) : ~k);
+}
+
 __device__ __forceinline__ unsigned lanemask_lt() {
   unsigned m;
   asm("mov.u32 %0, %%lanemask_lt;" : "=r"(m));
   return m;
 }
 
-// Token -> expert permutation and the expert kernels' work plan, by one CTA of
-// 256 threads.  Assignments are ranked within eight contiguous segments (one
-// warp each, match_any per 32), the per-segment counts are prefix-summed per
-// expert, and every assignment is placed at offsets[e] + its stable rank.
+// Token -> expert permutation (moe_permute), by one CTA of 256 threads.
+// Assignments are ranked within eight contiguous segments (one warp each,
+// match_any per 32), the per-segment counts are prefix-summed per expert, and
+// every assignment is placed at offsets[e] + its stable rank.
 // cw: shared scratch of 8*E + 2*(E+1) ints.
-template <bool IDS_SHARED>
-__device__ __forceinline__ int load_id(const int* ids, int a) {
-  return IDS_SHARED ? ids[a] : __ldcg(ids + a);
-}
-
-template <bool IDS_SHARED>
-__device__ void permute_plan(const int* ids, int T, int k, int E, int nt, int* counts,
-                             int* offsets, int* sorted, int* inv, int* active, int* cprefix,
-                             uint32_t* status, int* cw) {
+__device__ void permute_plan(const int* ids, int T, int k, int E, int* counts, int* offsets,
+                             int* sorted, int* inv, int* active, int* cw) {
   const int A = T * k;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int seg = (A + 7) / 8;
@@ -152,7 +155,7 @@ __device__ void permute_plan(const int* ids, int T, int k, int E, int nt, int* c
       const int a = base + lane;
       int e = -1;
       if (a < a_hi) {
-        e = load_id<IDS_SHARED>(ids, a);
+        e = __ldcg(ids + a);
         if (e < 0 || e >= E) {
           e = -1;
           *s_bad = 1;
@@ -183,55 +186,45 @@ __device__ void permute_plan(const int* ids, int T, int k, int E, int nt, int* c
   if (warp == 0) {
     const int per = (E + 31) / 32;
     const int e0 = lane * per, e1 = min(E, e0 + per);
-    int sc = 0, sa = 0, sch = 0;
+    int sc = 0, sa = 0;
     for (int e = e0; e < e1; ++e) {
       const int c = s_off[e];
       sc += c;
       sa += (c > 0);
-      sch += (c + nt - 1) / nt;
     }
-    int xc = sc, xa = sa, xch = sch;  // inclusive scans
+    int xc = sc, xa = sa;  // inclusive scans
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
       const int yc = __shfl_up_sync(0xffffffffu, xc, o);
       const int ya = __shfl_up_sync(0xffffffffu, xa, o);
-      const int ych = __shfl_up_sync(0xffffffffu, xch, o);
       if (lane >= o) {
         xc += yc;
         xa += ya;
-        xch += ych;
       }
     }
-    int rc = xc - sc, ra = xa - sa, rch = xch - sch;  // exclusive
+    int rc = xc - sc, ra = xa - sa;  // exclusive
     for (int e = e0; e < e1; ++e) {
       const int c = s_off[e];
       s_off[e] = rc;
       offsets[e] = rc;
-      if (c > 0) {
-        active[1 + ra] = e;
-        cprefix[ra] = rch;
-        ++ra;
-        rch += (c + nt - 1) / nt;
-      }
+      if (c > 0) active[1 + ra++] = e;
       rc += c;
     }
     if (lane == 31) {
       offsets[E] = xc;
       s_off[E] = xc;
       active[0] = *s_bad ? -1 : xa;
-      cprefix[xa] = xch;
     }
   }
   __syncthreads();
   for (int a = threadIdx.x; a < A; a += blockDim.x) {
-    const int e = load_id<IDS_SHARED>(ids, a);
+    const int e = __ldcg(ids + a);
     if (e < 0 || e >= E) continue;
     const int w = a / seg;
     const int pos = s_off[e] + cw[w * E + e] + inv[a];
     sorted[pos] = a;
     inv[a] = pos;
   }
-  if (threadIdx.x == 0 && *s_bad) set_status(status, kStatusBadExpertId);
 }
 
 // ------------------------------------------------------------------ route kernel
@@ -295,55 +288,82 @@ __global__ void __launch_bounds__(256) route_kernel(const RouteParams p) {
     }
   }
 
-  // router GEMV: two warps per expert row (one half of H each), lanes -> 4
-  // consecutive h per 128; the halves meet in shared memory
-  __shared__ float s_part[kRouteWarps][kRouteTok];
-  const int e = eb * kRouteEPB + (warp >> 1);
-  const int hhalf = H / 2;
-  const int hbeg = (warp & 1) * hhalf;
-  if (e < E) {
-    float acc[kRouteTok];
+  // router GEMV: warp w covers one eighth of H for all epb experts of this
+  // CTA (each staged x value is read once per warp), lanes -> 4 consecutive
+  // h per 128.  The 4 x 8 partial sums of a lane meet across the warp in a
+  // butterfly (lane l ends with sum l = expert slot l/8, token l%8), then
+  // across the warps in shared memory in warp order.
+  __shared__ float s_part[kRouteWarps][32];
+  {
+    constexpr int MAXEPB = 4;
+    const int nexp = min(p.epb, E - eb * p.epb);  // experts of this CTA
+    const int hpart = H / kRouteWarps;
+    const int hbeg = warp * hpart;
+    float acc[MAXEPB][kRouteTok];
 #pragma unroll
-    for (int t = 0; t < kRouteTok; ++t) acc[t] = 0.f;
-    const float* wrow = p.wr + (size_t)e * H;
-    // 16 router loads in flight per lane before any is used
-    constexpr int DEPTH = 16;
-    for (int h0 = hbeg + lane * 4; h0 < hbeg + hhalf; h0 += 128 * DEPTH) {
-      float4 w[DEPTH];
+    for (int x = 0; x < MAXEPB; ++x)
+#pragma unroll
+      for (int t = 0; t < kRouteTok; ++t) acc[x][t] = 0.f;
+    constexpr int DEPTH = 4;  // 128-element steps whose router loads are in flight together
+    for (int h0 = hbeg + lane * 4; h0 < hbeg + hpart; h0 += 128 * DEPTH) {
+      float4 w[DEPTH][MAXEPB];
 #pragma unroll
       for (int q = 0; q < DEPTH; ++q)
-        w[q] = (h0 + 128 * q < hbeg + hhalf)
-                   ? __ldg(reinterpret_cast<const float4*>(wrow + h0 + 128 * q))
-                   : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int x = 0; x < MAXEPB; ++x)
+          w[q][x] = (x < nexp && h0 + 128 * q < hbeg + hpart)
+                        ? __ldg(reinterpret_cast<const float4*>(
+                              p.wr + (size_t)(eb * p.epb + x) * H + h0 + 128 * q))
+                        : make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
       for (int q = 0; q < DEPTH; ++q) {
         const int h = h0 + 128 * q;
-        if (h >= hbeg + hhalf) break;
+        if (h >= hbeg + hpart) break;
 #pragma unroll
         for (int t = 0; t < kRouteTok; ++t) {
           if (t < nt) {
             const uint2 xv = *reinterpret_cast<const uint2*>(xs + (size_t)t * H + h);
             const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&xv.x));
             const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&xv.y));
-            float sacc = acc[t];
-            sacc = fmaf(a.x, w[q].x, sacc);
-            sacc = fmaf(a.y, w[q].y, sacc);
-            sacc = fmaf(b.x, w[q].z, sacc);
-            sacc = fmaf(b.y, w[q].w, sacc);
-            acc[t] = sacc;
+#pragma unroll
+            for (int x = 0; x < MAXEPB; ++x) {
+              float sacc = acc[x][t];
+              sacc = fmaf(a.x, w[q][x].x, sacc);
+              sacc = fmaf(a.y, w[q][x].y, sacc);
+              sacc = fmaf(b.x, w[q][x].z, sacc);
+              sacc = fmaf(b.y, w[q][x].w, sacc);
+              acc[x][t] = sacc;
+            }
           }
         }
       }
     }
+    float v[32];
 #pragma unroll
-    for (int t = 0; t < kRouteTok; ++t) acc[t] = warp_sum(acc[t]);
-    if (lane == 0)
-      for (int t = 0; t < kRouteTok; ++t) s_part[warp][t] = acc[t];
+    for (int i = 0; i < 32; ++i) v[i] = acc[i / kRouteTok][i % kRouteTok];
+#pragma unroll
+    for (int sft = 16; sft >= 1; sft >>= 1) {
+      const bool upper = (lane & sft) != 0;
+#pragma unroll
+      for (int i = 0; i < sft; ++i) {
+        const float send = upper ? v[i] : v[i + sft];
+        const float keep = upper ? v[i + sft] : v[i];
+        v[i] = keep + __shfl_xor_sync(0xffffffffu, send, sft);
+      }
+    }
+    s_part[warp][lane] = v[0];
   }
   __syncthreads();
-  if (e < E && (warp & 1) == 0 && lane < nt) {
-    const float b = p.bias ? __ldg(p.bias + e) : 0.f;
-    p.logits[(size_t)(t0 + lane) * E + e] = (s_part[warp][lane] + s_part[warp + 1][lane]) + b;
+  if (threadIdx.x < 32) {
+    const int x = threadIdx.x / kRouteTok, t = threadIdx.x % kRouteTok;
+    const int e = eb * p.epb + x;
+    if (x < p.epb && e < E && t < nt) {
+      float sum = s_part[0][threadIdx.x];
+#pragma unroll
+      for (int w = 1; w < kRouteWarps; ++w) sum += s_part[w][threadIdx.x];
+      const float b = p.bias ? __ldg(p.bias + e) : 0.f;
+      p.logits[(size_t)(t0 + t) * E + e] = sum + b;
+    }
   }
 
   // accumulators and counters of the later kernels start from zero
@@ -378,42 +398,38 @@ __global__ void __launch_bounds__(256) route_kernel(const RouteParams p) {
       v[i] = (i < per && ee < E) ? __ldcg(p.logits + (size_t)t * E + ee) : -INFINITY;
     }
     // Each lane keeps the best of its own untaken logits; a round takes the
-    // warp's best (value desc, index asc) and only the winning lane rescans.
+    // warp's best by two warp reductions - the largest order-preserving key,
+    // then the lowest expert index holding it (ties go to the lower index;
+    // -0 and +0 share a key) - and only the winning lane rescans.
+    unsigned key[PER];
+#pragma unroll
+    for (int i = 0; i < PER; ++i) key[i] = logit_key(v[i]);
     unsigned taken = 0u;
-    float lbv;
-    int lbi;
+    unsigned lbk;  // best untaken key of this lane (0: none left)
+    unsigned lbi;
     auto local_best = [&]() {
-      lbv = -INFINITY;
-      lbi = 0x7fffffff;
+      lbk = 0u;
+      lbi = 0xffffffffu;
 #pragma unroll
       for (int i = 0; i < PER; ++i) {
         const int ee = lane + 32 * i;
-        if (i < per && ee < E && !((taken >> i) & 1u) && (v[i] > lbv || (v[i] == lbv && ee < lbi))) {
-          lbv = v[i];
-          lbi = ee;
+        if (i < per && ee < E && !((taken >> i) & 1u) && key[i] > lbk) {
+          lbk = key[i];  // a later (higher) index never wins a tie within a lane
+          lbi = (unsigned)ee;
         }
       }
     };
     local_best();
     for (int j = 0; j < p.k; ++j) {
-      float bv = lbv;
-      int bi = lbi;
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
-        const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-        if (ov > bv || (ov == bv && oi < bi)) {
-          bv = ov;
-          bi = oi;
-        }
-      }
-      if ((bi & 31) == lane) {
+      const unsigned m = __reduce_max_sync(0xffffffffu, lbk);
+      const unsigned bi = __reduce_min_sync(0xffffffffu, lbk == m ? lbi : 0xffffffffu);
+      if ((int)(bi & 31u) == lane) {
         taken |= 1u << (bi >> 5);
         local_best();
       }
       if (lane == 0) {
-        s_sel[warp][j] = bi;
-        s_selv[warp][j] = bv;
+        s_sel[warp][j] = (int)bi;
+        s_selv[warp][j] = key_logit(m);
       }
     }
     __syncwarp();
@@ -435,47 +451,25 @@ __global__ void __launch_bounds__(256) route_kernel(const RouteParams p) {
       p.gates[(size_t)t * p.k + j] = gw;
       if (p.ids2) p.ids2[(size_t)t * p.k + j] = id;
       if (p.gates2) p.gates2[(size_t)t * p.k + j] = gw;
+      if (p.fused) {
+        // append to expert id's list (order within a list is arbitrary)
+        const unsigned pos = atomicAdd(p.acnt + id, 1u);
+        p.alist[(size_t)id * p.T + pos] = t * p.k + j;
+      }
     }
   }
-  if (!p.fused) return;
-  if (gridDim.y == 1) {
-    // a single token chunk: this CTA already holds every id (s_sel, warp t =
-    // token t) and builds the permutation without another ticket
-    __syncthreads();
-    int* s_ids = reinterpret_cast<int*>(route_smem);  // [T*k], ahead of the scratch
-    for (int a = threadIdx.x; a < p.T * p.k; a += blockDim.x) s_ids[a] = s_sel[a / p.k][a % p.k];
-    __syncthreads();
-    permute_plan<true>(s_ids, p.T, p.k, E, p.nt, p.counts, p.offsets, p.sorted, p.inv, p.active,
-                       p.cprefix, p.status, s_ids + kRouteTok * kMaxK);
-    return;
-  }
-
-  // chunk-completion ticket: the last chunk builds the permutation and plan
-  __threadfence();
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    const unsigned old = atomicAdd(p.done_cnt, 1u);
-    s_flag = (old == gridDim.y - 1);
-    if (s_flag) *p.done_cnt = 0u;
-  }
-  __syncthreads();
-  if (!s_flag) return;
-  __threadfence();
-  permute_plan<false>(p.ids, p.T, p.k, E, p.nt, p.counts, p.offsets, p.sorted, p.inv, p.active,
-                      p.cprefix, p.status, reinterpret_cast<int*>(route_smem));
 }
 
 __global__ void __launch_bounds__(256) permute_kernel(const int* ids, int T, int k, int E,
                                                       int* counts, int* offsets, int* sorted,
                                                       int* inv, int* active) {
   extern __shared__ __align__(16) unsigned char route_smem[];
-  int* cw = reinterpret_cast<int*>(route_smem);
-  int* cprefix_scratch = cw + 8 * E + 2 * (E + 1);  // the standalone call has no plan output
-  permute_plan<false>(ids, T, k, E, 32, counts, offsets, sorted, inv, active, cprefix_scratch,
-                      nullptr, cw);
+  permute_plan(ids, T, k, E, counts, offsets, sorted, inv, active,
+               reinterpret_cast<int*>(route_smem));
 }
 
-// Activation conversion, zeroing and work plan for the unfused expert FFN.
+// Activation conversion, zeroing and per-expert counts for the unfused
+// expert FFN (the expert kernels build their plan from the counts).
 __global__ void __launch_bounds__(256) prep_kernel(const PrepParams p) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   pdl_launch_dependents();
@@ -494,35 +488,9 @@ __global__ void __launch_bounds__(256) prep_kernel(const PrepParams p) {
       convert_row_dispatch(p.fmt, p.x + (size_t)t * p.H, p.H, p.x16 + (size_t)t * p.H,
                            p.xinv + t, lane, p.act == kActF16Perm);
   }
-  if (blockIdx.x == 0) {
+  if (blockIdx.x == 0)
     for (int e = threadIdx.x; e < p.E; e += blockDim.x)
       p.counts[e] = __ldg(p.offsets + e + 1) - __ldg(p.offsets + e);
-    if (warp == 0) {
-      const int nA = max(0, __ldg(p.active));
-      const int per = (nA + 31) / 32;
-      const int a0 = lane * per, a1 = min(nA, a0 + per);
-      int sch = 0;
-      for (int a = a0; a < a1; ++a) {
-        const int e = __ldg(p.active + 1 + a);
-        const int c = __ldg(p.offsets + e + 1) - __ldg(p.offsets + e);
-        sch += (c + p.nt - 1) / p.nt;
-      }
-      int x = sch;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const int y = __shfl_up_sync(0xffffffffu, x, o);
-        if (lane >= o) x += y;
-      }
-      int r = x - sch;
-      for (int a = a0; a < a1; ++a) {
-        const int e = __ldg(p.active + 1 + a);
-        const int c = __ldg(p.offsets + e + 1) - __ldg(p.offsets + e);
-        p.cprefix[a] = r;
-        r += (c + p.nt - 1) / p.nt;
-      }
-      if (lane == 31) p.cprefix[nA] = x;
-    }
-  }
 }
 
 __global__ void __launch_bounds__(256) combine_kernel(const CombineParams p) {
@@ -562,9 +530,8 @@ __global__ void __launch_bounds__(256) combine_kernel(const CombineParams p) {
 
 // ------------------------------------------------------------------ launchers
 size_t route_smem_bytes(int H, int E) {
-  const size_t xs = (size_t)kRouteTok * H * 2;
-  const size_t perm = sizeof(int) * (size_t)(kRouteTok * kMaxK + 8 * E + 2 * (E + 1));
-  return xs > perm ? xs : perm;
+  (void)E;
+  return (size_t)kRouteTok * H * 2;  // the chunk's token rows
 }
 
 cudaError_t launch_route(const RouteParams& p, cudaStream_t st) {
@@ -573,7 +540,7 @@ cudaError_t launch_route(const RouteParams& p, cudaStream_t st) {
   const size_t smem = route_smem_bytes(p.H, p.E);
   cudaError_t err = set_smem_once(route_kernel, (int)route_smem_bytes(8192, kMaxE), done);
   if (err != cudaSuccess) return err;
-  dim3 grid((p.E + kRouteEPB - 1) / kRouteEPB, (p.T + kRouteTok - 1) / kRouteTok);
+  dim3 grid((p.E + p.epb - 1) / p.epb, (p.T + kRouteTok - 1) / kRouteTok);
   route_kernel<<<grid, 256, smem, st>>>(p);
   return cudaGetLastError();
 }

@@ -1,15 +1,16 @@
 // Router, top-k, permutation and small elementwise kernels of the MoE decode
 // layer.
 //
-// route_kernel (grid = [ceil(E/4) expert blocks, ceil(T/8) token chunks]):
+// route_kernel (grid = [ceil(E/epb) expert blocks, ceil(T/8) token chunks]):
 //   every CTA stages 8 token rows of x in shared memory and computes the fp32
-//   logits of 4 experts (two warps per expert row of the router, one half of
-//   H each, float4 loads, shuffle reduction).  The CTA that arrives last at a chunk's ticket does
-//   the softmax/top-k of those 8 tokens (one warp per token, k rounds of a
-//   warp arg-max with ties to the lower index); in the fused layer the CTA
-//   that completes the last chunk builds the token->expert permutation and
-//   the work plan of the expert kernels.  Tickets are atomic counters reset
-//   by their last user; nothing waits on another CTA.
+//   logits of epb experts (each warp covers one eighth of H for all of them,
+//   float4 loads, shuffle reduction).  The CTA that arrives last at
+//   a chunk's ticket does the softmax/top-k of those 8 tokens (one warp per
+//   token, k rounds of a warp arg-max with ties to the lower index); in the
+//   fused layer it also appends each assignment to its expert's list (an
+//   atomic counter per expert), from which the expert kernels build their
+//   work plan.  Tickets and counters are reset by their last user; nothing
+//   waits on another CTA.
 #pragma once
 
 #include "common.cuh"
@@ -27,7 +28,8 @@ struct RouteParams {
   const __nv_bfloat16* x;
   const float* wr;
   const float* bias;
-  int T, H, E, k, renorm, prenorm, fmt, fused, nt;
+  int T, H, E, k, renorm, prenorm, fmt, fused;
+  int epb;  // experts per CTA (1 to 4)
   int act;  // activation form for the expert kernels (kAct*)
   float* logits;  // [T, E]
   int* ids;       // [T, k]
@@ -35,7 +37,6 @@ struct RouteParams {
   int* ids2;      // optional copies
   float* gates2;
   unsigned* chunk_cnt;
-  unsigned* done_cnt;
   // fused layer only
   __half* x16;
   uint8_t* xq;   // NVFP4 terms of x (kActTerms)
@@ -45,27 +46,20 @@ struct RouteParams {
   size_t zero_a_n4;
   float4* zero_b;
   size_t zero_b_n4;
-  int* counts;
-  int* offsets;
-  int* sorted;
-  int* inv;
-  int* active;
-  int* cprefix;
-  uint32_t* status;
+  unsigned* acnt;  // [E] assignments per expert, zero on entry
+  int* alist;      // [E, T] expert e's assignments t*k + j at alist[e*T + 0..]
 };
 
 struct PrepParams {
   const __nv_bfloat16* x;
-  int T, H, E, k, fmt, nt;
+  int T, H, E, k, fmt;
   int act;
   __half* x16;
   uint8_t* xq;
   uint8_t* xsf;
   float* xinv;
   const int* offsets;  // [E+1] from the permutation
-  const int* active;   // [E+1]
   int* counts;         // [E] (derived here)
-  int* cprefix;        // [E+1]
   float4* zero_a;
   size_t zero_a_n4;
   float4* zero_b;
