@@ -298,6 +298,18 @@ def zipf_stats(ids, E):
             "fitted_s": fit}
 
 
+def kernel_sources_sha256():
+    """sha256 over every CUDA source of the library (sorted by name)."""
+    import hashlib
+    d = os.path.join(ROOT, "paper_2609_11133_gb300", "csrc")
+    h = hashlib.sha256()
+    for f in sorted(os.listdir(d)):
+        if f.endswith((".cu", ".cuh")):
+            h.update(f.encode())
+            h.update(open(os.path.join(d, f), "rb").read())
+    return h.hexdigest()
+
+
 # ---------------------------------------------------------------- our arm
 def run_ours(args):
     import numpy as np
@@ -473,14 +485,9 @@ def run_ours(args):
     traffic = None
     tp = os.path.join(ROOT, "profiles", "traffic.json")
     if os.path.exists(tp):
-        import hashlib
         tj = json.load(open(tp)).get(f"{args.workload}_T{T}")
-        if tj:
-            hsh = hashlib.sha256()
-            for f in ("ffn.cuh", "common.cuh"):
-                hsh.update(open(os.path.join(ROOT, "paper_2609_11133_gb300", "csrc", f), "rb").read())
-            if hsh.hexdigest() == tj.get("kernel_sources_sha256"):
-                traffic = tj.get("gateup_dram_bytes")
+        if tj and kernel_sources_sha256() == tj.get("kernel_sources_sha256"):
+            traffic = tj.get("gateup_dram_bytes")
 
     cfg = {"workload": f"{args.workload}_T{T}", "H": H, "E": E, "k": k, "I": I,
            "tokens": T, "format": "nvfp4" if fmt == 2 else "fp8_block128",
@@ -527,8 +534,7 @@ def run_ours(args):
     if energy:
         res["j_per_token"] = energy["j_per_token"]
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        res["cpu_baseline"] = cpu_oracle_sample(wl, args.seed, w=w0 if L == 1 and not wl["zipf"]
-                                                else None)
+        res["cpu_baseline"] = cpu_oracle_sample(wl, args.seed, w=w0)  # layer 0's weights
     if rank == 0:
         print(json.dumps(res))
     if world > 1:

@@ -108,7 +108,9 @@ int moe_workspace_size(const moe_expert_weights_t* w, int T, int k, size_t* byte
 int moe_route_workspace_size(int T, int E, size_t* bytes);
 
 /* Zero a workspace (cudaMemsetAsync).  A workspace must be zeroed once
- * before its first use; the library keeps it consistent afterwards. */
+ * before its first use; the library keeps it consistent afterwards (its
+ * counters are reset by their last user).  After moe_read_status() reports
+ * an error, zero it again before the next call. */
 int moe_workspace_init(void* ws, size_t ws_bytes, void* stream);
 
 /* Copy the device status word of a workspace to *status (host pointer) and
