@@ -102,10 +102,10 @@ bool map_sf(CUtensorMap* m, const void* sf, int E, int N, int K) {
 
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
-// Expert engines: the block-scaled tcgen05 engine (ffn_bs.cuh) for NVFP4, the
-// warp-MMA engine (ffn.cuh) for FP8.  MOE_ENGINE=mma runs NVFP4 on the
-// warp-MMA engine too (for comparisons).
-enum Engine { kEngMma = 0, kEngBs = 1 };
+// Expert engines: the block-scaled tcgen05 engine (ffn_bs.cuh) for NVFP4 and
+// the FP8 tcgen05 engine (ffn_f8.cuh) for FP8.  MOE_ENGINE=mma runs both
+// formats on the warp-MMA engine (ffn.cuh) instead (for comparisons).
+enum Engine { kEngMma = 0, kEngBs = 1, kEngF8 = 2 };
 
 int engine_for(int fmt) {
   static int force_mma = -1;
@@ -113,26 +113,29 @@ int engine_for(int fmt) {
     const char* s = std::getenv("MOE_ENGINE");
     force_mma = (s && std::strcmp(s, "mma") == 0) ? 1 : 0;
   }
-  return (fmt == MOE_FMT_NVFP4 && !force_mma) ? kEngBs : kEngMma;
+  if (force_mma) return kEngMma;
+  return fmt == MOE_FMT_NVFP4 ? kEngBs : kEngF8;
 }
 
 int act_for(int fmt, int eng) {
   if (eng == kEngBs) return kActTerms;
+  if (eng == kEngF8) return kActE4M3;
   return fmt == MOE_FMT_NVFP4 ? kActF16Perm : kActF16;
 }
 
 // Token-chunk size of the expert kernels (the N side of the MMA; the
-// block-scaled engine uses 4 rows of N per token).  MOE_NT overrides the
-// choice (for measurements).
+// tensor-core engines use 4 (NVFP4) or 2 (FP8) rows of N per token).
+// MOE_NT overrides the choice (for measurements).
 int nt_for(int T, int eng) {
   if (const char* s = std::getenv("MOE_NT")) {
     const int v = std::atoi(s);
-    if (v == 8 || v == 16 || (v == 32 && eng == kEngMma)) return v;
+    if (v == 8 || v == 16 || (v == 32 && eng != kEngBs)) return v;
   }
-  // 8-token chunks: at T <= 64 few experts get more than 8 tokens (those are
-  // processed in several chunks); the warp-MMA consumers then hold a whole
-  // stage in registers and release it at once.
+  // 8-token chunks while few experts get more tokens than that (T <= 64 with
+  // top-8 of >= 128 experts); larger batches take wider chunks so that a hot
+  // expert's weights are streamed fewer times.
   if (eng == kEngBs) return T <= 64 ? 8 : 16;
+  if (eng == kEngF8) return T <= 64 ? 8 : (T <= 128 ? 16 : 32);
   return T <= 64 ? 8 : 32;
 }
 
@@ -214,8 +217,16 @@ int run_experts(const ExpertRun& r, cudaStream_t st, cudaEvent_t ev_mid) {
                       (uint64_t)H / 2, (uint64_t)r.T * kTerms, (uint64_t)H / 2, kRowBytes, kTerms,
                       CU_TENSOR_MAP_SWIZZLE_128B);
     ok = ok && map_2d(&m2.b, CU_TENSOR_MAP_DATA_TYPE_UINT8, ws_ptr<uint8_t>(r.ws, r.L.hq),
-                      (uint64_t)I / 2, (uint64_t)hq_rows(r.T, r.k), (uint64_t)I / 2, kRowBytes,
-                      (uint32_t)(kTerms * r.nt), CU_TENSOR_MAP_SWIZZLE_128B);
+                      (uint64_t)I / 2, (uint64_t)hq_rows(r.T, r.k, kTerms), (uint64_t)I / 2,
+                      kRowBytes, (uint32_t)(kTerms * r.nt), CU_TENSOR_MAP_SWIZZLE_128B);
+  } else if (eng == kEngF8) {
+    // E4M3 terms: x rows 2t, 2t+1 (one box per token), h rows of a chunk
+    ok = ok && map_2d(&m1.b, CU_TENSOR_MAP_DATA_TYPE_UINT8, ws_ptr<uint8_t>(r.ws, r.L.xq),
+                      (uint64_t)H, (uint64_t)r.T * kF8Terms, (uint64_t)H, kRowBytes, kF8Terms,
+                      CU_TENSOR_MAP_SWIZZLE_128B);
+    ok = ok && map_2d(&m2.b, CU_TENSOR_MAP_DATA_TYPE_UINT8, ws_ptr<uint8_t>(r.ws, r.L.hq),
+                      (uint64_t)I, (uint64_t)hq_rows(r.T, r.k, kF8Terms), (uint64_t)I, kRowBytes,
+                      (uint32_t)(kF8Terms * r.nt), CU_TENSOR_MAP_SWIZZLE_128B);
   } else {
     ok = ok && map_2d(&m1.b, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, x16, (uint64_t)H, (uint64_t)r.T,
                       (uint64_t)H * 2, (uint32_t)KEL, 1, CU_TENSOR_MAP_SWIZZLE_NONE);
@@ -270,6 +281,7 @@ int run_experts(const ExpertRun& r, cudaStream_t st, cudaEvent_t ev_mid) {
 
   auto launch = [&](const FfnMaps& m, const FfnParams& pp) {
     if (eng == kEngBs) return launch_ffn_bs(r.nt, r.sms, m, pp, st);
+    if (eng == kEngF8) return launch_ffn_f8(r.nt, r.sms, m, pp, st);
     return fp4 ? launch_ffn<2>(r.nt, r.sms, m, pp, st, true)
                : launch_ffn<1>(r.nt, r.sms, m, pp, st, true);
   };
@@ -278,6 +290,8 @@ int run_experts(const ExpertRun& r, cudaStream_t st, cudaEvent_t ev_mid) {
   if (ev_mid && cudaEventRecord(ev_mid, st) != cudaSuccess) return MOE_ERR_CUDA;
   if (eng == kEngBs)
     err = launch_swiglu_terms(r.T * r.k, r.sms, p1, st);
+  else if (eng == kEngF8)
+    err = launch_swiglu_e4m3(r.T * r.k, r.sms, p1, st);
   else if (fp4)
     err = launch_swiglu<2>(r.T * r.k, r.sms, p1, true, st);  // h16 in the unit order
   else
@@ -316,7 +330,7 @@ int moe_workspace_size(const moe_expert_weights_t* w, int T, int k, size_t* byte
   if (rc) return rc;
   rc = check_tk(T, k, w->E);
   if (rc) return rc;
-  *bytes = ws_layout(T, k, w->E, w->H, w->I, engine_for(w->fmt) == kEngBs).total;
+  *bytes = ws_layout(T, k, w->E, w->H, w->I, act_for(w->fmt, engine_for(w->fmt))).total;
   return MOE_OK;
 }
 
@@ -415,7 +429,7 @@ int moe_expert_ffn(const void* x, const moe_expert_weights_t* w, const int32_t* 
   if (T == 0) return MOE_OK;
   if (!x || !offsets || !sorted_assign || !active || !y_perm || !ws) return MOE_ERR_INVALID_ARG;
   if (!aligned(x, 16) || !aligned(y_perm, 16) || !aligned(ws, 256)) return MOE_ERR_INVALID_ARG;
-  const WsLayout L = ws_layout(T, k, w->E, w->H, w->I, engine_for(w->fmt) == kEngBs);
+  const WsLayout L = ws_layout(T, k, w->E, w->H, w->I, act_for(w->fmt, engine_for(w->fmt)));
   if (ws_bytes < L.total) return MOE_ERR_WORKSPACE_TOO_SMALL;
   if (T == 0) return MOE_OK;
   int sms = 0;
@@ -490,7 +504,7 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
     return MOE_ERR_INVALID_ARG;
   if (out == x) return MOE_ERR_INVALID_ARG;
   const int E = w->E, H = w->H, I = w->I;
-  const WsLayout L = ws_layout(T, k, E, H, I, engine_for(w->fmt) == kEngBs);
+  const WsLayout L = ws_layout(T, k, E, H, I, act_for(w->fmt, engine_for(w->fmt)));
   if (ws_bytes < L.total) return MOE_ERR_WORKSPACE_TOO_SMALL;
   if (T == 0) return MOE_OK;
   int sms = 0;

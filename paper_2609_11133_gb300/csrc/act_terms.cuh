@@ -127,4 +127,52 @@ __device__ __forceinline__ void load_bf16x16_scaled(const __nv_bfloat16* src, fl
   }
 }
 
+
+// ------------------------------------------------------------------ E4M3 terms
+// The FP8 tensor-core engine (ffn_f8.cuh) multiplies E4M3 weights with E4M3
+// activations (kind::f8f6f4, no block scale).  An activation row v is written
+// as v * 2^p = hi + lo with hi = e4m3(v * 2^p) and lo = e4m3(v * 2^p - hi):
+// hi keeps four significant bits, lo the next four, so a bf16 input (eight
+// bits) is kept whole unless it is more than ~2^14 below the row maximum.
+// Two B rows per token; the epilogue adds the two columns.
+constexpr int kF8Terms = 2;
+
+// Power-of-two factor that maps max|v| into [2^7, 2^8) (E4M3 max 448).
+__device__ __forceinline__ float pow2_scale_e4m3(float amax) {
+  if (!(amax > 0.f) || !isfinite(amax)) return 1.f;
+  int e;
+  frexpf(amax, &e);
+  return ldexpf(1.f, min(8 - e, 126));
+}
+
+// Two floats to two E4M3 codes (round to nearest even, saturating), the
+// first in the low byte.
+__device__ __forceinline__ uint32_t e4m3x2_from_f32(float v0, float v1) {
+  uint16_t two;
+  asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(two) : "f"(v1), "f"(v0));
+  return two;
+}
+
+// Eight values (already scaled) to their hi and lo E4M3 codes (8 bytes each).
+__device__ __forceinline__ void encode_e4m3x2_8(const float (&v)[8], uint2& hi, uint2& lo) {
+  uint32_t h[4], l[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    h[i] = e4m3x2_from_f32(v[2 * i], v[2 * i + 1]);
+    const uint32_t hd = e4m3x2_to_f16x2(h[i]);  // exact
+    const float2 d = __half22float2(*reinterpret_cast<const __half2*>(&hd));
+    l[i] = e4m3x2_from_f32(v[2 * i] - d.x, v[2 * i + 1] - d.y);
+  }
+  hi = make_uint2(h[0] | (h[1] << 16), h[2] | (h[3] << 16));
+  lo = make_uint2(l[0] | (l[1] << 16), l[2] | (l[3] << 16));
+}
+
+// Store the two terms of 8 values at column c8*8 of row `row2` (= 2 * row):
+// rows are K bytes.
+__device__ __forceinline__ void store_e4m3x2_8(const uint2& hi, const uint2& lo, uint8_t* q,
+                                               size_t row2, int K, int c8) {
+  *reinterpret_cast<uint2*>(q + row2 * (size_t)K + 8 * c8) = hi;
+  *reinterpret_cast<uint2*>(q + (row2 + 1) * (size_t)K + 8 * c8) = lo;
+}
+
 }  // namespace moe

@@ -32,6 +32,12 @@ constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s
 // ------------------------------------------------------------------ workspace
 // Byte offsets of everything the kernels keep between launches.  Built on the
 // host by ws_layout() and passed by value to the kernels.
+// Activation forms the expert engines read.
+constexpr int kActF16 = 0;      // f16 rows (power-of-two scaled), natural order
+constexpr int kActF16Perm = 1;  // f16 rows in the warp-MMA NVFP4 unit order
+constexpr int kActTerms = 2;    // four NVFP4 terms per row (block-scaled engine)
+constexpr int kActE4M3 = 3;     // two E4M3 terms per row (FP8 tensor-core engine)
+
 struct WsLayout {
   // control block (zeroed once; every counter is reset by its last user)
   size_t status;       // u32 device status word
@@ -50,26 +56,28 @@ struct WsLayout {
   size_t hinv;     // f32 [T*k]
   size_t h16;      // f16 [T*k, I]
   size_t oacc;     // f32 [T, H] combine accumulator
-  // NVFP4 activation terms of the block-scaled engine (zero-sized otherwise;
-  // x16 and h16 are zero-sized when these are used)
-  size_t xq;       // u8 [T*4, H/2]   E2M1 codes of x
-  size_t xsf;      // u8 [T*4, H/16]  UE4M3 scales of x
-  size_t hq;       // u8 [T*k*4, I/2] E2M1 codes of h
-  size_t hsf;      // u8 [T*k*4, I/16]
+  // activation terms of the tensor-core engines (zero-sized otherwise; x16
+  // and h16 are zero-sized when these are used).  NVFP4: x codes [4T, H/2],
+  // x scales [4T, H/16], h codes [4Tk, I/2], h scales [4Tk, I/16]; FP8:
+  // x [2T, H] and h [2Tk, I] E4M3 (hi and lo rows).
+  size_t xq;
+  size_t xsf;
+  size_t hq;
+  size_t hsf;
   size_t total;
   int nChunks;
 };
 
 inline size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
-// Rows of the h-terms array: four per assignment, and at least one full
-// down-step B box (4 x 16 rows) so that a box never extends past the array.
-inline size_t hq_rows(int T, int k) {
-  const size_t r = 4 * (size_t)T * k;
+// Rows of an h-terms array (`terms` rows per assignment), at least one full
+// down-step B box (64 rows) so that a box never extends past the array.
+inline size_t hq_rows(int T, int k, int terms) {
+  const size_t r = (size_t)terms * T * k;
   return r < 64 ? 64 : r;
 }
 
-inline WsLayout ws_layout(int T, int k, int E, int H, int I, bool terms = false) {
+inline WsLayout ws_layout(int T, int k, int E, int H, int I, int act = kActF16) {
   WsLayout L{};
   size_t o = 0;
   auto take = [&](size_t bytes) {
@@ -88,17 +96,17 @@ inline WsLayout ws_layout(int T, int k, int E, int H, int I, bool terms = false)
   L.counts = take(4 * (size_t)E);
   L.alist = take(4 * (size_t)E * T);
   L.xinv = take(4 * (size_t)T);
-  const size_t nf = terms ? 0 : 1;  // f16 activations: warp-MMA engine only
+  const size_t nf = (act == kActF16 || act == kActF16Perm) ? 1 : 0;  // warp-MMA engine only
   L.x16 = take(nf * 2 * (size_t)T * H);
   L.gu = take(4 * TK * 2 * (size_t)I);
   L.hinv = take(4 * TK);
   L.h16 = take(nf * 2 * TK * (size_t)I);
   L.oacc = take(4 * (size_t)T * H);
-  const size_t nt = terms ? 1 : 0;
-  L.xq = take(nt * 4 * (size_t)T * H / 2);
-  L.xsf = take(nt * 4 * (size_t)T * H / 16);
-  L.hq = take(nt * hq_rows(T, k) * (size_t)I / 2);
-  L.hsf = take(nt * hq_rows(T, k) * (size_t)I / 16);
+  const size_t n4 = (act == kActTerms) ? 1 : 0, n8 = (act == kActE4M3) ? 1 : 0;
+  L.xq = take((n4 + n8) * 2 * (size_t)T * H);  // 4T rows x H/2, or 2T rows x H
+  L.xsf = take(n4 * 4 * (size_t)T * H / 16);
+  L.hq = take(n4 * hq_rows(T, k, 4) * (size_t)I / 2 + n8 * hq_rows(T, k, 2) * (size_t)I);
+  L.hsf = take(n4 * hq_rows(T, k, 4) * (size_t)I / 16);
   L.total = o;
   return L;
 }

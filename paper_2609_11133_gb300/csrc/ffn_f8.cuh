@@ -1,0 +1,408 @@
+// FP8 expert FFN on the tensor cores: tcgen05.mma kind::f8f6f4, E4M3 weights
+// as stored times E4M3 activation terms, fp32 accumulation in tensor memory.
+//
+// Work decomposition as in ffn.cuh / ffn_bs.cuh: a persistent grid, stream-K
+// over the K-stages of all (active expert, <=NT-token chunk, row tile) items.
+// A stage is 128 K, which is exactly one column of the weights' 128x128 fp32
+// block scales.  The MMA has no block scaling for this format pair, so every
+// stage accumulates into its own slot of a ring of tensor-memory accumulators
+// and the epilogue warps multiply it by the stage's two block scales while
+// adding it into registers; an item's sums are flushed with red.add at its
+// last stage (in this CTA).  The activations arrive as two E4M3 terms per
+// token (act_terms.cuh): B rows 2j, 2j+1 of token j; the epilogue adds the
+// two columns.
+//
+// Roles (224 threads):
+//   warps 0-3  epilogue: warp w reads TMEM lanes 32w..32w+31 (rows of the tile)
+//   warps 4,6  TMA producers (one thread each): warp 4 arms each stage's
+//              barrier and copies box A0, warp 6 box A1 and the activation rows
+//   warp 5     MMA issuer (one thread); allocates and frees tensor memory
+// Every wait is bounded (p.wait_ns); an expired wait sets the status word and
+// the kernel winds down, freeing its tensor memory.
+#pragma once
+
+#include "act_terms.cuh"
+#include "ffn.cuh"
+
+namespace moe {
+
+constexpr int kF8Threads = 7 * 32;
+constexpr int kF8EpiWarp0 = 0, kF8ProducerWarp = 4, kF8MmaWarp = 5, kF8ProducerWarp2 = 6;
+constexpr uint32_t kF8TmemCols = 256;
+
+template <int NT>
+struct F8Geom {
+  static constexpr int BN = kF8Terms * NT;  // B rows = MMA N
+  static constexpr int A0 = 0;
+  static constexpr int A1 = kRowsHalf * kRowBytes;      // 16 KB
+  static constexpr int B = 2 * kRowsHalf * kRowBytes;   // 32 KB, 1024-aligned
+  static constexpr int RAW = B + BN * kRowBytes;
+  static constexpr int BYTES = (RAW + 1023) / 1024 * 1024;
+  static constexpr int STAGES_RAW = (212 * 1024) / BYTES;  // + ~9 KB static
+  static constexpr int STAGES = STAGES_RAW > 8 ? 8 : STAGES_RAW;
+  static constexpr int SMEM = STAGES * BYTES + 1024;
+  static constexpr int DR = (NT <= 16) ? 4 : 2;  // accumulator ring (stages)
+  static_assert(DR * 2 * BN <= (int)kF8TmemCols, "tensor memory budget");
+  static_assert(BN % 16 == 0 && BN <= 256, "MMA N");
+};
+
+// Instruction descriptor of kind::f8f6f4: f32 D, E4M3 A and B, K-major.
+__host__ __device__ constexpr uint32_t tc_idesc_e4m3(int M, int N) {
+  return (1u << 4) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+__device__ __forceinline__ void tc_mma_f8(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                          uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.u32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+template <int NT>
+__global__ void __launch_bounds__(kF8Threads, 1)
+    ffn_f8_kernel(const __grid_constant__ CUtensorMap tmA0,
+                  const __grid_constant__ CUtensorMap tmA1,
+                  const __grid_constant__ CUtensorMap tmB, const FfnParams p) {
+  using G = F8Geom<NT>;
+  constexpr int BN = G::BN;
+  constexpr int S = G::STAGES;
+  constexpr int DR = G::DR;
+  constexpr int KEL = 128;  // K per stage
+
+  extern __shared__ __align__(1024) unsigned char smem_raw[];
+  unsigned char* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+
+  __shared__ __align__(8) uint64_t full_bar[S];
+  __shared__ __align__(8) uint64_t empty_bar[S];
+  __shared__ __align__(8) uint64_t dfull_bar[DR];
+  __shared__ __align__(8) uint64_t dempty_bar[DR];
+  __shared__ __align__(8) uint64_t final_bar;
+  __shared__ PlanSmem pl;
+  __shared__ int s_tok[NT];
+  __shared__ uint32_t s_tmem;
+  __shared__ volatile int s_abort;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    s_abort = 0;
+    for (int i = 0; i < S; ++i) {
+      mbar_init(&full_bar[i], 1);
+      mbar_init(&empty_bar[i], 1);
+    }
+    for (int i = 0; i < DR; ++i) {
+      mbar_init(&dfull_bar[i], 1);
+      mbar_init(&dempty_bar[i], 4);
+    }
+    mbar_init(&final_bar, 1);
+    fence_mbar_init();
+  }
+  if (warp == kF8MmaWarp) {
+    tmem_alloc(&s_tmem, kF8TmemCols);
+    tmem_relinquish();
+  }
+  // Launched as a programmatic dependent: everything above overlapped the
+  // previous kernel; from here on its outputs are read.
+  pdl_wait();
+  pdl_launch_dependents();
+  if (warp == 0) build_plan(p.counts, p.E, NT, pl, lane);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = s_tmem;
+
+  const int N = (p.phase == 1) ? p.I : p.H;  // rows of one expert matrix
+  const int K = (p.phase == 1) ? p.H : p.I;  // contraction length
+  const int rtiles = (p.phase == 1) ? p.I / kRowsHalf : p.H / (2 * kRowsHalf);
+  const int KB = K / KEL;
+  const long long items = (long long)pl.cpre[pl.nA] * rtiles;
+  const long long total = items * KB;
+  const long long s_begin = total * blockIdx.x / gridDim.x;
+  const long long s_end = total * (blockIdx.x + 1) / gridDim.x;
+  const long long nst = s_end - s_begin;
+  const uint32_t timeout_bit = (p.phase == 1) ? kStatusTimeoutGateUp : kStatusTimeoutDown;
+  constexpr int kTeardown = 5 * 32;  // epilogue and MMA warps
+
+  // ================================================================ producers
+  if (warp == kF8ProducerWarp || warp == kF8ProducerWarp2) {
+    const bool lead = (warp == kF8ProducerWarp);
+    if (lane == 0 && nst > 0) {
+      tma_prefetch_desc(lead ? &tmA0 : &tmA1);
+      if (!lead) tma_prefetch_desc(&tmB);
+      const uint64_t pol_w = policy_evict_first();
+      const uint64_t pol_a = policy_evict_last();
+      long long cur_item = -1;
+      ItemInfo inf{};
+      long long issued = 0;
+      for (long long s = s_begin; s < s_end; ++s, ++issued) {
+        const long long it = s / KB;
+        const int kb = (int)(s % KB);
+        if (it != cur_item) {
+          cur_item = it;
+          inf = decode_item(it, rtiles, pl, p, NT);
+          if (!lead && p.phase == 1)
+            for (int j = 0; j < inf.nvalid; ++j) s_tok[j] = __ldg(p.sorted + inf.lrow0 + j) / p.k;
+        }
+        const int slot = (int)(issued % S);
+        const uint32_t round = (uint32_t)(issued / S);
+        if (!mbar_wait_bounded(&empty_bar[slot], (round & 1u) ^ 1u, p.wait_ns, &s_abort)) {
+          set_status(p.status, timeout_bit);
+          s_abort = 1;
+          break;
+        }
+        if (p.test_stall && issued == 0) continue;  // test hook: this stage never arrives
+        unsigned char* st = smem + (size_t)slot * G::BYTES;
+        int rowA0, rowA1;
+        if (p.phase == 1) {
+          rowA0 = inf.e * N + inf.rt * kRowsHalf;
+          rowA1 = rowA0;
+        } else {
+          rowA0 = inf.e * N + inf.rt * 2 * kRowsHalf;
+          rowA1 = rowA0 + kRowsHalf;
+        }
+        if (lead) {
+          // the second producer's copies may land before this arms the
+          // barrier: the transaction count then dips below zero, and the
+          // phase still cannot complete before this arrival
+          uint32_t bytes = 2u * kRowsHalf * kRowBytes;
+          bytes += (p.phase == 1) ? (uint32_t)inf.nvalid * kF8Terms * kRowBytes
+                                  : (uint32_t)BN * kRowBytes;
+          mbar_arrive_expect_tx(&full_bar[slot], bytes);
+          tma_load_2d(st + G::A0, &tmA0, &full_bar[slot], kb * kRowBytes, rowA0, pol_w);
+          continue;
+        }
+        tma_load_2d(st + G::A1, &tmA1, &full_bar[slot], kb * kRowBytes, rowA1, pol_w);
+        // activation terms: token j's two rows land at B rows 2j, 2j+1
+        if (p.phase == 1) {
+          for (int j = 0; j < inf.nvalid; ++j)
+            tma_load_2d(st + G::B + j * kF8Terms * kRowBytes, &tmB, &full_bar[slot],
+                        kb * kRowBytes, s_tok[j] * kF8Terms, pol_a);
+        } else {
+          tma_load_2d(st + G::B, &tmB, &full_bar[slot], kb * kRowBytes, inf.arow0 * kF8Terms,
+                      pol_a);
+        }
+      }
+      // Let every copy land before the CTA exits (the barriers complete only
+      // when both producers' copies have landed).
+      if (!lead) return;
+      const long long first = issued > S ? issued - S : 0;
+      for (long long j = first; j < issued; ++j) {
+        if (p.test_stall && j == 0) continue;
+        mbar_wait_bounded(&full_bar[j % S], (uint32_t)((j / S) & 1), p.wait_ns, nullptr);
+      }
+    }
+    return;
+  }
+
+  // ================================================================ MMA issuer
+  if (warp == kF8MmaWarp) {
+    if (lane == 0) {
+      constexpr uint32_t idesc = tc_idesc_e4m3(128, BN);
+      bool ok = true;
+      for (long long i = 0; i < nst && ok; ++i) {
+        const int slot = (int)(i % S);
+        const int db = (int)(i % DR);
+        ok = mbar_wait_bounded(&dempty_bar[db], ((uint32_t)(i / DR) & 1u) ^ 1u, p.wait_ns,
+                               &s_abort) &&
+             mbar_wait_bounded(&full_bar[slot], (uint32_t)(i / S) & 1u, p.wait_ns, &s_abort);
+        if (!ok) break;
+        tc_fence_after();
+        const uint32_t st = smem_u32(smem + (size_t)slot * G::BYTES);
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk) {  // K = 32 per MMA
+          const uint64_t bdesc = tc_desc_sw128(st + G::B + 32 * kk);
+          tc_mma_f8(tmem + (uint32_t)(2 * db) * BN, tc_desc_sw128(st + G::A0 + 32 * kk), bdesc,
+                    idesc, kk > 0 ? 1u : 0u);
+          tc_mma_f8(tmem + (uint32_t)(2 * db + 1) * BN, tc_desc_sw128(st + G::A1 + 32 * kk),
+                    bdesc, idesc, kk > 0 ? 1u : 0u);
+        }
+        tc_commit(&empty_bar[slot]);
+        tc_commit(&dfull_bar[db]);
+      }
+      if (!ok) {
+        set_status(p.status, timeout_bit);
+        s_abort = 1;
+      }
+      // every MMA this thread issued has completed before TMEM is released
+      tc_commit(&final_bar);
+      mbar_wait_bounded(&final_bar, 0, p.wait_ns, nullptr);
+    }
+    __syncwarp();
+    asm volatile("bar.sync 2, %0;" ::"n"(kTeardown) : "memory");
+    tc_fence_after();
+    tmem_dealloc(tmem, kF8TmemCols);
+    return;
+  }
+
+  // ================================================================ epilogue
+  // Warp q reads TMEM lanes 32q..32q+31: row 32q+lane of both boxes.
+  {
+    const int quad = warp - kF8EpiWarp0;
+    const int row = quad * 32 + lane;
+    const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
+    const int KB128 = K / 128;
+    float acc0[NT], acc1[NT];
+#pragma unroll
+    for (int j = 0; j < NT; ++j) acc0[j] = acc1[j] = 0.f;
+    bool dead = false;
+    long long cur_item = -1;
+    ItemInfo inf{};
+    // the block scales of a stage's two boxes
+    auto scales = [&](const ItemInfo& f, int kb, float& b0, float& b1) {
+      if (p.phase == 1) {
+        const size_t tile = ((size_t)f.e * (N / 128) + f.rt) * KB128 + kb;
+        b0 = __ldg(p.s0 + tile);
+        b1 = __ldg(p.s1 + tile);
+      } else {
+        const size_t tile = ((size_t)f.e * (N / 128) + 2 * f.rt) * KB128 + kb;
+        b0 = __ldg(p.s0 + tile);
+        b1 = __ldg(p.s0 + tile + KB128);
+      }
+    };
+    float bs0 = 0.f, bs1 = 0.f;
+    if (nst > 0) {
+      inf = decode_item(s_begin / KB, rtiles, pl, p, NT);
+      cur_item = s_begin / KB;
+      scales(inf, (int)(s_begin % KB), bs0, bs1);
+    }
+    for (long long i = 0; i < nst && !dead; ++i) {
+      const long long s = s_begin + i;
+      const long long it = s / KB;
+      // the next stage's scales, loaded while this stage's accumulator is awaited
+      float nb0 = 0.f, nb1 = 0.f;
+      ItemInfo ninf = inf;
+      if (i + 1 < nst) {
+        const long long it1 = (s + 1) / KB;
+        if (it1 != it) ninf = decode_item(it1, rtiles, pl, p, NT);
+        scales(ninf, (int)((s + 1) % KB), nb0, nb1);
+      }
+      const int db = (int)(i % DR);
+      if (!mbar_wait_bounded(&dfull_bar[db], (uint32_t)(i / DR) & 1u, p.wait_ns, &s_abort)) {
+        set_status(p.status, timeout_bit);
+        s_abort = 1;
+        dead = true;
+        break;
+      }
+      tc_fence_after();
+      // token j's two terms are accumulator columns 2j and 2j+1
+#pragma unroll
+      for (int mat = 0; mat < 2; ++mat) {
+        const uint32_t d_t = tmem + lane_addr + (uint32_t)(2 * db + mat) * BN;
+        const float bsc = mat == 0 ? bs0 : bs1;
+#pragma unroll
+        for (int c0 = 0; c0 < BN; c0 += 16) {
+          uint32_t v[16];
+          tmem_ld16(d_t + c0, v);
+          tmem_ld_wait();
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            const float t2 = __uint_as_float(v[2 * q]) + __uint_as_float(v[2 * q + 1]);
+            if (mat == 0)
+              acc0[c0 / 2 + q] = fmaf(bsc, t2, acc0[c0 / 2 + q]);
+            else
+              acc1[c0 / 2 + q] = fmaf(bsc, t2, acc1[c0 / 2 + q]);
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&dempty_bar[db]);
+      const bool closes = (i + 1 == nst) || ((s + 1) / KB != it);
+      if (closes) {
+#pragma unroll
+        for (int j = 0; j < NT; ++j) {
+          if (j < inf.nvalid) {
+            const int arow = inf.arow0 + j;
+            const int a = __ldg(p.sorted + inf.lrow0 + j);
+            if (p.phase == 1) {
+              const float sc = __ldg(p.xinv + a / p.k);
+              const int f = inf.rt * kRowsHalf + row;
+              float* gr = p.gu + (size_t)arow * 2 * p.I + f;
+              red_add_f32(gr, acc0[j] * sc);
+              red_add_f32(gr + p.I, acc1[j] * sc);
+            } else {
+              const float sc = __ldcg(p.xinv + arow);  // hinv, written by the previous kernel
+              const int hrow = inf.rt * 2 * kRowsHalf + row;
+              if (p.fused) {
+                const float gw = __ldg(p.gates + a) * sc;
+                float* orow = p.oacc + (size_t)(a / p.k) * p.H + hrow;
+                red_add_f32(orow, gw * acc0[j]);
+                red_add_f32(orow + kRowsHalf, gw * acc1[j]);
+              } else {
+                float* yrow = p.y_perm + (size_t)arow * p.H + hrow;
+                red_add_f32(yrow, acc0[j] * sc);
+                red_add_f32(yrow + kRowsHalf, acc1[j] * sc);
+              }
+            }
+          }
+          acc0[j] = acc1[j] = 0.f;
+        }
+      }
+      inf = ninf;
+      cur_item = (s + 1) / KB;
+      bs0 = nb0;
+      bs1 = nb1;
+    }
+    (void)cur_item;
+    tc_fence_before();
+    asm volatile("bar.sync 2, %0;" ::"n"(kTeardown) : "memory");
+  }
+}
+
+// SwiGLU of every assignment row into two E4M3 terms (the B operand of the
+// FP8 engine's down step): h = silu(g) * u from the fp32 gate|up
+// accumulators, a per-row power of two, then hi/lo per 8 columns.  One CTA
+// per row; each thread owns up to 8 groups of 8 columns (I <= 8192).
+__global__ void __launch_bounds__(128) swiglu_e4m3_kernel(const FfnParams p, int rows) {
+  constexpr int G = 8;
+  __shared__ float s_max[4];
+  pdl_wait();
+  pdl_launch_dependents();
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int n8 = p.I / 8;
+  for (int row = blockIdx.x; row < rows; row += gridDim.x) {
+    const float* g = p.gu + (size_t)row * 2 * p.I;
+    const float* u = g + p.I;
+    float h[G][8];
+    float amax = 0.f;
+#pragma unroll
+    for (int q = 0; q < G; ++q) {
+      const int c = threadIdx.x + 128 * q;
+      if (c < n8) {
+#pragma unroll
+        for (int i = 0; i < 8; i += 4) {
+          const float4 gv = __ldcg(reinterpret_cast<const float4*>(g + 8 * c + i));
+          const float4 uv = __ldcg(reinterpret_cast<const float4*>(u + 8 * c + i));
+          h[q][i + 0] = gv.x / (1.f + expf(-gv.x)) * uv.x;
+          h[q][i + 1] = gv.y / (1.f + expf(-gv.y)) * uv.y;
+          h[q][i + 2] = gv.z / (1.f + expf(-gv.z)) * uv.z;
+          h[q][i + 3] = gv.w / (1.f + expf(-gv.w)) * uv.w;
+        }
+#pragma unroll
+        for (int i = 0; i < 8; ++i) amax = fmaxf(amax, fabsf(h[q][i]));
+      }
+    }
+    amax = warp_max(amax);
+    if (lane == 0) s_max[warp] = amax;
+    __syncthreads();
+    amax = fmaxf(fmaxf(s_max[0], s_max[1]), fmaxf(s_max[2], s_max[3]));
+    const float sc = pow2_scale_e4m3(amax);
+#pragma unroll
+    for (int q = 0; q < G; ++q) {
+      const int c = threadIdx.x + 128 * q;
+      if (c < n8) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) h[q][i] *= sc;
+        uint2 hi, lo;
+        encode_e4m3x2_8(h[q], hi, lo);
+        store_e4m3x2_8(hi, lo, p.hq, (size_t)row * kF8Terms, p.I, c);
+      }
+    }
+    if (threadIdx.x == 0) p.hinv[row] = 1.f / sc;
+    __syncthreads();  // s_max is reused by the next row
+  }
+}
+
+}  // namespace moe

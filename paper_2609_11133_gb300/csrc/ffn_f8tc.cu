@@ -1,0 +1,40 @@
+// The FP8 tcgen05 engine (ffn_f8.cuh) and the SwiGLU step that feeds its down
+// projection.
+#include "ffn_f8.cuh"
+#include "ffn_launch.cuh"
+
+namespace moe {
+
+template <int NT>
+static cudaError_t launch_ffn_f8_nt(int grid, const FfnMaps& m, const FfnParams& p,
+                                    cudaStream_t st) {
+  auto kern = ffn_f8_kernel<NT>;
+  const int smem = F8Geom<NT>::SMEM;
+  static std::atomic<unsigned long long> done{0};
+  cudaError_t err = set_smem_once(kern, smem, done);
+  if (err != cudaSuccess) return err;
+  return launch_pdl(kern, dim3(grid), dim3(kF8Threads), smem, st, m.a0, m.a1, m.b, p);
+}
+
+cudaError_t launch_ffn_f8(int nt, int grid, const FfnMaps& m, const FfnParams& p,
+                          cudaStream_t st) {
+  switch (nt) {
+    case 8:
+      return launch_ffn_f8_nt<8>(grid, m, p, st);
+    case 16:
+      return launch_ffn_f8_nt<16>(grid, m, p, st);
+    case 32:
+      return launch_ffn_f8_nt<32>(grid, m, p, st);
+    default:
+      return cudaErrorInvalidValue;
+  }
+}
+
+cudaError_t launch_swiglu_e4m3(int rows, int sms, const FfnParams& p, cudaStream_t st) {
+  int blocks = rows;
+  if (blocks > 8 * sms) blocks = 8 * sms;
+  if (blocks < 1) blocks = 1;
+  return launch_pdl(swiglu_e4m3_kernel, dim3(blocks), dim3(128), 0, st, p, rows);
+}
+
+}  // namespace moe

@@ -48,6 +48,12 @@ cudaError_t launch_ffn_bs(int nt, int grid, const FfnMaps& maps, const FfnParams
                           cudaStream_t st);
 cudaError_t launch_swiglu_terms(int rows, int sms, const FfnParams& p, cudaStream_t st);
 
+// The FP8 tcgen05 engine (ffn_f8.cuh, instantiated in ffn_f8tc.cu); nt in
+// {8, 16, 32}.  SwiGLU into E4M3 terms for its down step.
+cudaError_t launch_ffn_f8(int nt, int grid, const FfnMaps& maps, const FfnParams& p,
+                          cudaStream_t st);
+cudaError_t launch_swiglu_e4m3(int rows, int sms, const FfnParams& p, cudaStream_t st);
+
 
 #define MOE_DEFINE_FFN_LAUNCH(FMTV)                                                            \
   template <int NT>                                                                             \

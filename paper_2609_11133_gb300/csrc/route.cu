@@ -92,6 +92,81 @@ __device__ void convert_chunk_terms(const __nv_bfloat16* xs, int nt, int H, int 
   }
 }
 
+// The two E4M3 terms of a chunk of token rows staged in shared memory, every
+// CTA of the chunk an equal share of the 8-element groups.
+__device__ void convert_chunk_e4m3(const __nv_bfloat16* xs, int nt, int H, int t0, int part,
+                                   int nparts, uint8_t* xq, float* xinv) {
+  __shared__ float s_sc[kRouteTok];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (warp < nt) {
+    float amax = 0.f;
+    for (int h = lane * 8; h < H; h += 256) {
+      const uint4 v = *reinterpret_cast<const uint4*>(xs + (size_t)warp * H + h);
+      const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const float2 f = __bfloat1622float2(b[i]);
+        amax = fmaxf(amax, fmaxf(fabsf(f.x), fabsf(f.y)));
+      }
+    }
+    amax = warp_max(amax);
+    const float sc = pow2_scale_e4m3(amax);
+    if (lane == 0) {
+      s_sc[warp] = sc;
+      if (part == 0) xinv[t0 + warp] = 1.f / sc;
+    }
+  }
+  __syncthreads();
+  const int n8 = H / 8;
+  for (int idx = part * blockDim.x + threadIdx.x; idx < nt * n8; idx += nparts * blockDim.x) {
+    const int j = idx / n8, c = idx - j * n8;
+    const uint4 v = *reinterpret_cast<const uint4*>(xs + (size_t)j * H + 8 * c);
+    const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&v);
+    float f[8];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 t = __bfloat1622float2(b[i]);
+      f[2 * i] = t.x * s_sc[j];
+      f[2 * i + 1] = t.y * s_sc[j];
+    }
+    uint2 hi, lo;
+    encode_e4m3x2_8(f, hi, lo);
+    store_e4m3x2_8(hi, lo, xq, (size_t)(t0 + j) * kF8Terms, H, c);
+  }
+}
+
+// The two E4M3 terms of one token row in global memory, by one warp.
+__device__ void convert_row_e4m3(const __nv_bfloat16* row, int H, int t, uint8_t* xq, float* inv,
+                                 int lane) {
+  float amax = 0.f;
+  for (int h = lane * 8; h < H; h += 256) {
+    const uint4 v = *reinterpret_cast<const uint4*>(row + h);
+    const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 f = __bfloat1622float2(b[i]);
+      amax = fmaxf(amax, fmaxf(fabsf(f.x), fabsf(f.y)));
+    }
+  }
+  amax = warp_max(amax);
+  const float sc = pow2_scale_e4m3(amax);
+  for (int c = lane; c < H / 8; c += 32) {
+    const uint4 v = *reinterpret_cast<const uint4*>(row + 8 * c);
+    const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&v);
+    float f[8];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 tt = __bfloat1622float2(b[i]);
+      f[2 * i] = tt.x * sc;
+      f[2 * i + 1] = tt.y * sc;
+    }
+    uint2 hi, lo;
+    encode_e4m3x2_8(f, hi, lo);
+    store_e4m3x2_8(hi, lo, xq, (size_t)t * kF8Terms, H, c);
+  }
+  if (lane == 0) *inv = 1.f / sc;
+}
+
 // The NVFP4 terms of one token row in global memory, by one warp.
 __device__ void convert_row_terms(const __nv_bfloat16* row, int H, int t, uint8_t* xq,
                                   uint8_t* xsf, float* inv, int lane) {
@@ -281,6 +356,8 @@ __global__ void __launch_bounds__(256) route_kernel(const RouteParams p) {
   if (p.fused) {
     if (p.act == kActTerms) {
       convert_chunk_terms(xs, nt, H, t0, eb, gridDim.x, p.xq, p.xsf, p.xinv);
+    } else if (p.act == kActE4M3) {
+      convert_chunk_e4m3(xs, nt, H, t0, eb, gridDim.x, p.xq, p.xinv);
     } else if (eb == 0 && warp < nt) {
       const int t = t0 + warp;
       convert_row_dispatch(p.fmt, xs + (size_t)warp * H, H, p.x16 + (size_t)t * H, p.xinv + t,
@@ -484,6 +561,8 @@ __global__ void __launch_bounds__(256) prep_kernel(const PrepParams p) {
   if (t < p.T) {
     if (p.act == kActTerms)
       convert_row_terms(p.x + (size_t)t * p.H, p.H, t, p.xq, p.xsf, p.xinv + t, lane);
+    else if (p.act == kActE4M3)
+      convert_row_e4m3(p.x + (size_t)t * p.H, p.H, t, p.xq, p.xinv + t, lane);
     else
       convert_row_dispatch(p.fmt, p.x + (size_t)t * p.H, p.H, p.x16 + (size_t)t * p.H,
                            p.xinv + t, lane, p.act == kActF16Perm);

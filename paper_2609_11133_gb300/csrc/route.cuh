@@ -19,10 +19,6 @@ namespace moe {
 
 constexpr int kMaxK = 32;
 
-// Activation forms the expert engines read.
-constexpr int kActF16 = 0;      // f16 rows (power-of-two scaled), natural order
-constexpr int kActF16Perm = 1;  // f16 rows in the warp-MMA NVFP4 unit order
-constexpr int kActTerms = 2;    // four NVFP4 terms per row (block-scaled engine)
 
 struct RouteParams {
   const __nv_bfloat16* x;
@@ -39,7 +35,7 @@ struct RouteParams {
   unsigned* chunk_cnt;
   // fused layer only
   __half* x16;
-  uint8_t* xq;   // NVFP4 terms of x (kActTerms)
+  uint8_t* xq;   // terms of x (kActTerms, kActE4M3)
   uint8_t* xsf;
   float* xinv;
   float4* zero_a;
