@@ -135,7 +135,7 @@ int nt_for(int T, int eng) {
   // top-8 of >= 128 experts); larger batches take wider chunks so that a hot
   // expert's weights are streamed fewer times.
   if (eng == kEngBs) return T <= 64 ? 8 : 16;
-  if (eng == kEngF8) return T <= 64 ? 8 : (T <= 128 ? 16 : 32);
+  if (eng == kEngF8) return T <= 64 ? 8 : 32;
   return T <= 64 ? 8 : 32;
 }
 
@@ -181,6 +181,7 @@ struct ExpertRun {
   const int* sorted;  // assignment lists (see FfnParams::list_T)
   int list_T;
   const int* counts;  // tokens per expert
+  int gathered;       // x terms already in compact-row order (xg, xgsf)
   const float* gates;
   int fused;
   float* y_perm;
@@ -211,19 +212,30 @@ int run_experts(const ExpertRun& r, cudaStream_t st, cudaEvent_t ev_mid) {
   __half* h16 = ws_ptr<__half>(r.ws, r.L.h16);
   const int eng = engine_for(w->fmt);
   if (eng == kEngBs) {
-    // activation terms: x rows 4t..4t+3 (one box per token), h rows of a
-    // chunk's assignments (one box of 4*nt rows)
-    ok = ok && map_2d(&m1.b, CU_TENSOR_MAP_DATA_TYPE_UINT8, ws_ptr<uint8_t>(r.ws, r.L.xq),
-                      (uint64_t)H / 2, (uint64_t)r.T * kTerms, (uint64_t)H / 2, kRowBytes, kTerms,
-                      CU_TENSOR_MAP_SWIZZLE_128B);
+    // activation terms: x rows 4t..4t+3 (one box per token) or, gathered,
+    // the chunk's rows (one box of 4*nt rows); h rows of a chunk likewise
+    if (r.gathered)
+      ok = ok && map_2d(&m1.b, CU_TENSOR_MAP_DATA_TYPE_UINT8, ws_ptr<uint8_t>(r.ws, r.L.xg),
+                        (uint64_t)H / 2, (uint64_t)hq_rows(r.T, r.k, kTerms), (uint64_t)H / 2,
+                        kRowBytes, (uint32_t)(kTerms * r.nt), CU_TENSOR_MAP_SWIZZLE_128B);
+    else
+      ok = ok && map_2d(&m1.b, CU_TENSOR_MAP_DATA_TYPE_UINT8, ws_ptr<uint8_t>(r.ws, r.L.xq),
+                        (uint64_t)H / 2, (uint64_t)r.T * kTerms, (uint64_t)H / 2, kRowBytes,
+                        kTerms, CU_TENSOR_MAP_SWIZZLE_128B);
     ok = ok && map_2d(&m2.b, CU_TENSOR_MAP_DATA_TYPE_UINT8, ws_ptr<uint8_t>(r.ws, r.L.hq),
                       (uint64_t)I / 2, (uint64_t)hq_rows(r.T, r.k, kTerms), (uint64_t)I / 2,
                       kRowBytes, (uint32_t)(kTerms * r.nt), CU_TENSOR_MAP_SWIZZLE_128B);
   } else if (eng == kEngF8) {
-    // E4M3 terms: x rows 2t, 2t+1 (one box per token), h rows of a chunk
-    ok = ok && map_2d(&m1.b, CU_TENSOR_MAP_DATA_TYPE_UINT8, ws_ptr<uint8_t>(r.ws, r.L.xq),
-                      (uint64_t)H, (uint64_t)r.T * kF8Terms, (uint64_t)H, kRowBytes, kF8Terms,
-                      CU_TENSOR_MAP_SWIZZLE_128B);
+    // E4M3 terms: x rows 2t, 2t+1 (one box per token) or gathered (one box
+    // of 2*nt rows), h rows of a chunk
+    if (r.gathered)
+      ok = ok && map_2d(&m1.b, CU_TENSOR_MAP_DATA_TYPE_UINT8, ws_ptr<uint8_t>(r.ws, r.L.xg),
+                        (uint64_t)H, (uint64_t)hq_rows(r.T, r.k, kF8Terms), (uint64_t)H,
+                        kRowBytes, (uint32_t)(kF8Terms * r.nt), CU_TENSOR_MAP_SWIZZLE_128B);
+    else
+      ok = ok && map_2d(&m1.b, CU_TENSOR_MAP_DATA_TYPE_UINT8, ws_ptr<uint8_t>(r.ws, r.L.xq),
+                        (uint64_t)H, (uint64_t)r.T * kF8Terms, (uint64_t)H, kRowBytes, kF8Terms,
+                        CU_TENSOR_MAP_SWIZZLE_128B);
     ok = ok && map_2d(&m2.b, CU_TENSOR_MAP_DATA_TYPE_UINT8, ws_ptr<uint8_t>(r.ws, r.L.hq),
                       (uint64_t)I, (uint64_t)hq_rows(r.T, r.k, kF8Terms), (uint64_t)I, kRowBytes,
                       (uint32_t)(kF8Terms * r.nt), CU_TENSOR_MAP_SWIZZLE_128B);
@@ -259,7 +271,8 @@ int run_experts(const ExpertRun& r, cudaStream_t st, cudaEvent_t ev_mid) {
   p1.gu = ws_ptr<float>(r.ws, r.L.gu);
   p1.h16 = h16;
   p1.hinv = ws_ptr<float>(r.ws, r.L.hinv);
-  p1.bsf = ws_ptr<uint8_t>(r.ws, r.L.xsf);
+  p1.bsf = ws_ptr<uint8_t>(r.ws, r.gathered ? r.L.xgsf : r.L.xsf);
+  p1.b_compact = r.gathered;
   p1.hq = ws_ptr<uint8_t>(r.ws, r.L.hq);
   p1.hsf = ws_ptr<uint8_t>(r.ws, r.L.hsf);
   p1.test_stall = r.test_stall;
@@ -549,6 +562,24 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
   p.alist = ws_ptr<int>(ws, L.alist);
   if (ev[0] && cudaEventRecord(ev[0], st) != cudaSuccess) return MOE_ERR_CUDA;
   if (launch_route(p, st) != cudaSuccess) return MOE_ERR_CUDA;
+  const bool gathered = gather_terms(T, p.act);
+  if (gathered) {
+    const bool fp4 = (p.act == kActTerms);
+    GatherParams g{};
+    g.q = p.xq;
+    g.sf = fp4 ? p.xsf : nullptr;
+    g.gq = ws_ptr<uint8_t>(ws, L.xg);
+    g.gsf = ws_ptr<uint8_t>(ws, L.xgsf);
+    g.acnt = p.acnt;
+    g.alist = p.alist;
+    g.T = T;
+    g.k = k;
+    g.E = E;
+    g.terms = fp4 ? kTerms : kF8Terms;
+    g.qrow = fp4 ? H / 2 : H;
+    g.sfrow = H / 16;
+    if (launch_gather(g, st) != cudaSuccess) return MOE_ERR_CUDA;
+  }
   if (ev[1] && cudaEventRecord(ev[1], st) != cudaSuccess) return MOE_ERR_CUDA;
 
   ExpertRun r{};
@@ -561,6 +592,7 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
   r.L = L;
   r.sorted = p.alist;
   r.list_T = 1;
+  r.gathered = gathered ? 1 : 0;
   r.counts = reinterpret_cast<const int*>(p.acnt);
   r.gates = p.gates;
   r.fused = 1;

@@ -64,6 +64,10 @@ struct WsLayout {
   size_t xsf;
   size_t hq;
   size_t hsf;
+  // T > 64, tensor-core engines: x terms gathered into compact-row order
+  // (rows as h: terms per assignment), and their NVFP4 scales
+  size_t xg;
+  size_t xgsf;
   size_t total;
   int nChunks;
 };
@@ -75,6 +79,13 @@ inline size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 inline size_t hq_rows(int T, int k, int terms) {
   const size_t r = (size_t)terms * T * k;
   return r < 64 ? 64 : r;
+}
+
+// The fused layer gathers the activation terms into compact-row order when
+// chunks are wide (more than 64 tokens): one B box per chunk instead of one
+// per token.
+inline bool gather_terms(int T, int act) {
+  return T > 64 && (act == kActTerms || act == kActE4M3);
 }
 
 inline WsLayout ws_layout(int T, int k, int E, int H, int I, int act = kActF16) {
@@ -107,6 +118,9 @@ inline WsLayout ws_layout(int T, int k, int E, int H, int I, int act = kActF16) 
   L.xsf = take(n4 * 4 * (size_t)T * H / 16);
   L.hq = take(n4 * hq_rows(T, k, 4) * (size_t)I / 2 + n8 * hq_rows(T, k, 2) * (size_t)I);
   L.hsf = take(n4 * hq_rows(T, k, 4) * (size_t)I / 16);
+  const size_t ng = gather_terms(T, act) ? 1 : 0;
+  L.xg = take(ng * (n4 * hq_rows(T, k, 4) * (size_t)H / 2 + n8 * hq_rows(T, k, 2) * (size_t)H));
+  L.xgsf = take(ng * n4 * hq_rows(T, k, 4) * (size_t)H / 16);
   L.total = o;
   return L;
 }

@@ -101,6 +101,9 @@ struct FfnParams {
   const int* counts;   // [E]
   const int* sorted;
   int list_T;
+  // phase 1 of the tensor-core engines: 1 = the activation terms were
+  // gathered into compact-row order (one B box per chunk), 0 = per token
+  int b_compact;
   const float* gates;  // [T*k] by assignment (fused only)
   uint32_t* acnt_reset;  // finalize_kernel zeroes these E counters (fused only)
   // scales
@@ -183,20 +186,24 @@ struct ItemInfo {
   int slot, e, arow0, lrow0, nvalid, rt;
 };
 
-// Item `it` = (chunk of an active expert, row tile): arow0 is the chunk's
-// first compact row, lrow0 the index of its first assignment in p.sorted.
+// Item `it` = (active expert, row tile, chunk), chunk fastest: the items of
+// one expert's row tile are adjacent, so a hot expert's weight tile is read
+// from HBM once and its further token chunks find it in L2.  arow0 is the
+// chunk's first compact row, lrow0 the index of its first assignment in
+// p.sorted.
 __device__ __forceinline__ ItemInfo decode_item(long long it, int rtiles, const PlanSmem& pl,
                                                 const FfnParams& p, int NT) {
   ItemInfo r;
-  const int chunk_g = (int)(it / rtiles);
-  r.rt = (int)(it % rtiles);
-  int lo = 0, hi = pl.nA - 1;  // last slot with cpre[slot] <= chunk_g
+  int lo = 0, hi = pl.nA - 1;  // last slot with cpre[slot] * rtiles <= it
   while (lo < hi) {
     const int mid = (lo + hi + 1) >> 1;
-    if (pl.cpre[mid] <= chunk_g) lo = mid; else hi = mid - 1;
+    if ((long long)pl.cpre[mid] * rtiles <= it) lo = mid; else hi = mid - 1;
   }
   r.slot = lo;
-  const int chunk = chunk_g - pl.cpre[lo];
+  const int nch = pl.cpre[lo + 1] - pl.cpre[lo];  // chunks of this expert
+  const int local = (int)(it - (long long)pl.cpre[lo] * rtiles);
+  r.rt = local / nch;
+  const int chunk = local - r.rt * nch;
   r.e = pl.act[lo];
   r.arow0 = pl.aoff[lo] + chunk * NT;
   r.lrow0 = (p.list_T ? r.e * p.T : pl.aoff[lo]) + chunk * NT;

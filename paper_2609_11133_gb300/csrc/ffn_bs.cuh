@@ -157,6 +157,8 @@ __global__ void __launch_bounds__(kBsThreads, 1)
   const long long s_end = total * (blockIdx.x + 1) / gridDim.x;
   const long long nst = s_end - s_begin;
   const uint32_t timeout_bit = (p.phase == 1) ? kStatusTimeoutGateUp : kStatusTimeoutDown;
+  // B rows: per token (phase 1, tokens scattered) or one box per chunk
+  const bool btok = (p.phase == 1) && !p.b_compact;
   constexpr int kTeardown = 9 * 32;  // scale writers, epilogue and MMA warps
 
   // ================================================================ producer
@@ -179,7 +181,7 @@ __global__ void __launch_bounds__(kBsThreads, 1)
         if (it != cur_item) {
           cur_item = it;
           inf = decode_item(it, rtiles, pl, p, NT);
-          if (!lead && p.phase == 1)
+          if (!lead && btok)
             for (int j = 0; j < inf.nvalid; ++j) s_tok[j] = __ldg(p.sorted + inf.lrow0 + j) / p.k;
         }
         const int slot = (int)(issued % S);
@@ -192,7 +194,7 @@ __global__ void __launch_bounds__(kBsThreads, 1)
         if (p.test_stall && issued == 0) continue;  // test hook: this stage never arrives
         unsigned char* st = smem + (size_t)slot * G::BYTES;
         uint32_t bytes = 2u * kRowsHalf * kRowBytes + 2u * kRowsHalf * 16u;
-        bytes += (p.phase == 1) ? (uint32_t)inf.nvalid * kTerms * kRowBytes
+        bytes += btok ? (uint32_t)inf.nvalid * kTerms * kRowBytes
                                 : (uint32_t)BN * kRowBytes;
         // the second producer's copies may land before this arms the barrier:
         // the transaction count then dips below zero, and the phase still
@@ -214,7 +216,7 @@ __global__ void __launch_bounds__(kBsThreads, 1)
         tma_load_2d(st + G::A1, &tmA1, &full_bar[slot], kb * kRowBytes, rowA1, pol_w);
         tma_load_2d(st + G::S1, &tmS1, &full_bar[slot], kb * 16, rowA1, pol_w);
         // activation terms: token j's four rows land at B rows 4j..4j+3
-        if (p.phase == 1) {
+        if (btok) {
           for (int j = 0; j < inf.nvalid; ++j)
             tma_load_2d(st + G::B + j * kTerms * kRowBytes, &tmB, &full_bar[slot],
                         kb * kRowBytes, s_tok[j] * kTerms, pol_a);
@@ -310,8 +312,7 @@ __global__ void __launch_bounds__(kBsThreads, 1)
           const int j = n / kTerms;
           grow[h] = -1;
           if (n < BN && j < inf.nvalid) {
-            const int base = (p.phase == 1) ? __ldg(p.sorted + inf.lrow0 + j) / p.k
-                                            : inf.arow0 + j;
+            const int base = btok ? __ldg(p.sorted + inf.lrow0 + j) / p.k : inf.arow0 + j;
             grow[h] = base * kTerms + n % kTerms;
           }
         }

@@ -28,7 +28,6 @@ namespace moe {
 
 constexpr int kF8Threads = 7 * 32;
 constexpr int kF8EpiWarp0 = 0, kF8ProducerWarp = 4, kF8MmaWarp = 5, kF8ProducerWarp2 = 6;
-constexpr uint32_t kF8TmemCols = 256;
 
 template <int NT>
 struct F8Geom {
@@ -41,8 +40,9 @@ struct F8Geom {
   static constexpr int STAGES_RAW = (212 * 1024) / BYTES;  // + ~9 KB static
   static constexpr int STAGES = STAGES_RAW > 8 ? 8 : STAGES_RAW;
   static constexpr int SMEM = STAGES * BYTES + 1024;
-  static constexpr int DR = (NT <= 16) ? 4 : 2;  // accumulator ring (stages)
-  static_assert(DR * 2 * BN <= (int)kF8TmemCols, "tensor memory budget");
+  static constexpr int DR = 4;  // accumulator ring (stages)
+  static constexpr uint32_t TMEM_COLS = (DR * 2 * BN <= 256) ? 256u : 512u;
+  static_assert(DR * 2 * BN <= (int)TMEM_COLS, "tensor memory budget");
   static_assert(BN % 16 == 0 && BN <= 256, "MMA N");
 };
 
@@ -100,7 +100,7 @@ __global__ void __launch_bounds__(kF8Threads, 1)
     fence_mbar_init();
   }
   if (warp == kF8MmaWarp) {
-    tmem_alloc(&s_tmem, kF8TmemCols);
+    tmem_alloc(&s_tmem, G::TMEM_COLS);
     tmem_relinquish();
   }
   // Launched as a programmatic dependent: everything above overlapped the
@@ -123,6 +123,8 @@ __global__ void __launch_bounds__(kF8Threads, 1)
   const long long s_end = total * (blockIdx.x + 1) / gridDim.x;
   const long long nst = s_end - s_begin;
   const uint32_t timeout_bit = (p.phase == 1) ? kStatusTimeoutGateUp : kStatusTimeoutDown;
+  // B rows: per token (phase 1, tokens scattered) or one box per chunk
+  const bool btok = (p.phase == 1) && !p.b_compact;
   constexpr int kTeardown = 5 * 32;  // epilogue and MMA warps
 
   // ================================================================ producers
@@ -142,7 +144,7 @@ __global__ void __launch_bounds__(kF8Threads, 1)
         if (it != cur_item) {
           cur_item = it;
           inf = decode_item(it, rtiles, pl, p, NT);
-          if (!lead && p.phase == 1)
+          if (!lead && btok)
             for (int j = 0; j < inf.nvalid; ++j) s_tok[j] = __ldg(p.sorted + inf.lrow0 + j) / p.k;
         }
         const int slot = (int)(issued % S);
@@ -167,7 +169,7 @@ __global__ void __launch_bounds__(kF8Threads, 1)
           // barrier: the transaction count then dips below zero, and the
           // phase still cannot complete before this arrival
           uint32_t bytes = 2u * kRowsHalf * kRowBytes;
-          bytes += (p.phase == 1) ? (uint32_t)inf.nvalid * kF8Terms * kRowBytes
+          bytes += btok ? (uint32_t)inf.nvalid * kF8Terms * kRowBytes
                                   : (uint32_t)BN * kRowBytes;
           mbar_arrive_expect_tx(&full_bar[slot], bytes);
           tma_load_2d(st + G::A0, &tmA0, &full_bar[slot], kb * kRowBytes, rowA0, pol_w);
@@ -175,7 +177,7 @@ __global__ void __launch_bounds__(kF8Threads, 1)
         }
         tma_load_2d(st + G::A1, &tmA1, &full_bar[slot], kb * kRowBytes, rowA1, pol_w);
         // activation terms: token j's two rows land at B rows 2j, 2j+1
-        if (p.phase == 1) {
+        if (btok) {
           for (int j = 0; j < inf.nvalid; ++j)
             tma_load_2d(st + G::B + j * kF8Terms * kRowBytes, &tmB, &full_bar[slot],
                         kb * kRowBytes, s_tok[j] * kF8Terms, pol_a);
@@ -232,7 +234,7 @@ __global__ void __launch_bounds__(kF8Threads, 1)
     __syncwarp();
     asm volatile("bar.sync 2, %0;" ::"n"(kTeardown) : "memory");
     tc_fence_after();
-    tmem_dealloc(tmem, kF8TmemCols);
+    tmem_dealloc(tmem, G::TMEM_COLS);
     return;
   }
 
@@ -286,24 +288,23 @@ __global__ void __launch_bounds__(kF8Threads, 1)
         break;
       }
       tc_fence_after();
-      // token j's two terms are accumulator columns 2j and 2j+1
+      // token j's two terms are accumulator columns 2j and 2j+1; each box's
+      // columns are read with all loads in flight before one wait
 #pragma unroll
       for (int mat = 0; mat < 2; ++mat) {
         const uint32_t d_t = tmem + lane_addr + (uint32_t)(2 * db + mat) * BN;
         const float bsc = mat == 0 ? bs0 : bs1;
+        uint32_t v[BN];
 #pragma unroll
-        for (int c0 = 0; c0 < BN; c0 += 16) {
-          uint32_t v[16];
-          tmem_ld16(d_t + c0, v);
-          tmem_ld_wait();
+        for (int c0 = 0; c0 < BN; c0 += 16) tmem_ld16(d_t + c0, *reinterpret_cast<uint32_t(*)[16]>(v + c0));
+        tmem_ld_wait();
 #pragma unroll
-          for (int q = 0; q < 8; ++q) {
-            const float t2 = __uint_as_float(v[2 * q]) + __uint_as_float(v[2 * q + 1]);
-            if (mat == 0)
-              acc0[c0 / 2 + q] = fmaf(bsc, t2, acc0[c0 / 2 + q]);
-            else
-              acc1[c0 / 2 + q] = fmaf(bsc, t2, acc1[c0 / 2 + q]);
-          }
+        for (int j = 0; j < NT; ++j) {
+          const float t2 = __uint_as_float(v[2 * j]) + __uint_as_float(v[2 * j + 1]);
+          if (mat == 0)
+            acc0[j] = fmaf(bsc, t2, acc0[j]);
+          else
+            acc1[j] = fmaf(bsc, t2, acc1[j]);
         }
       }
       tc_fence_before();

@@ -572,6 +572,43 @@ __global__ void __launch_bounds__(256) prep_kernel(const PrepParams p) {
       p.counts[e] = __ldg(p.offsets + e + 1) - __ldg(p.offsets + e);
 }
 
+// grid (E, ceil(T/8)): CTA (e, g) copies list positions 8g..8g+7 of expert e.
+__global__ void __launch_bounds__(256) gather_kernel(const GatherParams p) {
+  __shared__ int s_off;
+  __shared__ int s_tok[8];
+  pdl_wait();  // the routing that wrote the lists is complete
+  pdl_launch_dependents();
+  const int e = blockIdx.x, g0 = blockIdx.y * 8;
+  const int n_e = (int)__ldcg(p.acnt + e);
+  if (g0 >= n_e) return;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (warp == 0) {  // first compact row of expert e: the counts of the experts before it
+    int sum = 0;
+    for (int i = lane; i < e; i += 32) sum += (int)__ldcg(p.acnt + i);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+    if (lane == 0) s_off = sum;
+  }
+  const int nj = min(8, n_e - g0);
+  if (threadIdx.x < nj) s_tok[threadIdx.x] = __ldcg(p.alist + (size_t)e * p.T + g0 + threadIdx.x) / p.k;
+  __syncthreads();
+  const int q16 = p.terms * p.qrow / 16;  // 16-byte units of one token's term rows
+  for (int i = threadIdx.x; i < nj * q16; i += blockDim.x) {
+    const int j = i / q16, u = i - j * q16;
+    const uint4 v = __ldcg(reinterpret_cast<const uint4*>(p.q + (size_t)s_tok[j] * p.terms * p.qrow) + u);
+    reinterpret_cast<uint4*>(p.gq + (size_t)(s_off + g0 + j) * p.terms * p.qrow)[u] = v;
+  }
+  if (p.sf) {
+    const int s16 = p.terms * p.sfrow / 16;
+    for (int i = threadIdx.x; i < nj * s16; i += blockDim.x) {
+      const int j = i / s16, u = i - j * s16;
+      const uint4 v =
+          __ldcg(reinterpret_cast<const uint4*>(p.sf + (size_t)s_tok[j] * p.terms * p.sfrow) + u);
+      reinterpret_cast<uint4*>(p.gsf + (size_t)(s_off + g0 + j) * p.terms * p.sfrow)[u] = v;
+    }
+  }
+}
+
 __global__ void __launch_bounds__(256) combine_kernel(const CombineParams p) {
   const size_t n4 = (size_t)p.T * p.H / 4;
   for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4;
@@ -622,6 +659,19 @@ cudaError_t launch_route(const RouteParams& p, cudaStream_t st) {
   dim3 grid((p.E + p.epb - 1) / p.epb, (p.T + kRouteTok - 1) / kRouteTok);
   route_kernel<<<grid, 256, smem, st>>>(p);
   return cudaGetLastError();
+}
+
+cudaError_t launch_gather(const GatherParams& p, cudaStream_t st) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)p.E, (unsigned)((p.T + 7) / 8));
+  cfg.blockDim = dim3(256);
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, gather_kernel, p);
 }
 
 cudaError_t launch_permute_standalone(const int* ids, int T, int k, int E, int* counts,

@@ -62,6 +62,19 @@ struct PrepParams {
   size_t zero_b_n4;
 };
 
+// Copy each assignment's activation-term rows (and NVFP4 scale rows) from
+// token order into compact-row order (expert by expert, list order inside an
+// expert), so that the gate/up kernel reads a chunk's B tile with one box.
+struct GatherParams {
+  const uint8_t* q;   // [T*terms, qrow] terms of x
+  const uint8_t* sf;  // [T*terms, sfrow] their UE4M3 scales, or null
+  uint8_t* gq;        // [T*k*terms, qrow]
+  uint8_t* gsf;       // [T*k*terms, sfrow] (when sf)
+  const unsigned* acnt;
+  const int* alist;   // [E, T]
+  int T, k, E, terms, qrow, sfrow;
+};
+
 struct CombineParams {
   const float* y_perm;
   const float* topk_w;
@@ -77,6 +90,7 @@ cudaError_t launch_permute_standalone(const int* ids, int T, int k, int E, int* 
                                       cudaStream_t st);
 cudaError_t launch_prep(const PrepParams& p, cudaStream_t st);
 cudaError_t launch_combine(const CombineParams& p, cudaStream_t st);
+cudaError_t launch_gather(const GatherParams& p, cudaStream_t st);
 size_t route_smem_bytes(int H, int E);
 
 }  // namespace moe
