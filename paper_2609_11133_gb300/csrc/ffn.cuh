@@ -150,9 +150,19 @@ __device__ __forceinline__ void build_plan(const int* counts, int E, int NT, Pla
   int run_off = 0, run_act = 0, run_ch = 0;
   unsigned lt;
   asm("mov.u32 %0, %%lanemask_lt;" : "=r"(lt));
-  for (int base = 0; base < E; base += 32) {
+  constexpr int G = kMaxE / 32;
+  int cnt[G];  // every count load in flight before the first is used
+#pragma unroll
+  for (int g = 0; g < G; ++g) {
+    const int e = 32 * g + lane;
+    cnt[g] = (e < E) ? __ldcg(counts + e) : 0;
+  }
+#pragma unroll
+  for (int g = 0; g < G; ++g) {
+    const int base = 32 * g;
+    if (base >= E) break;
     const int e = base + lane;
-    const int c = (e < E) ? __ldcg(counts + e) : 0;
+    const int c = cnt[g];
     const int ch = (c + NT - 1) / NT;
     int oc = c, och = ch;
 #pragma unroll

@@ -138,8 +138,13 @@ __global__ void __launch_bounds__(kBsThreads, 1)
     tmem_relinquish();
   }
   // Launched as a programmatic dependent: everything above overlapped the
-  // previous kernel; from here on its outputs are read.
-  pdl_wait();
+  // previous kernel.  The gate/up step waits for it here.  The down step's
+  // plan and weights do not depend on it (the counts were written by a kernel
+  // that completed before the gate/up step started), so its first weight
+  // copies start at once and only the roles that read the SwiGLU output wait
+  // (griddepcontrol.wait) before their first read of it.
+  const bool early = (p.phase == 2);
+  if (!early) pdl_wait();
   pdl_launch_dependents();
   if (warp == 0) build_plan(p.counts, p.E, NT, pl, lane);
   tc_fence_before();
@@ -164,6 +169,7 @@ __global__ void __launch_bounds__(kBsThreads, 1)
   // ================================================================ producer
   if (warp == kBsProducerWarp || warp == kBsProducerWarp2) {
     const bool lead = (warp == kBsProducerWarp);
+    if (!lead && early) pdl_wait();  // the activation rows are the SwiGLU output
     if (lane == 0 && nst > 0) {
       tma_prefetch_desc(&tmA0);
       tma_prefetch_desc(&tmA1);
@@ -208,13 +214,19 @@ __global__ void __launch_bounds__(kBsThreads, 1)
           rowA0 = inf.e * N + inf.rt * 2 * kRowsHalf;
           rowA1 = rowA0 + kRowsHalf;
         }
-        if (lead) {
+        if (lead) {  // gate/up: box A0; down: all weights (they may be copied early)
           tma_load_2d(st + G::A0, &tmA0, &full_bar[slot], kb * kRowBytes, rowA0, pol_w);
           tma_load_2d(st + G::S0, &tmS0, &full_bar[slot], kb * 16, rowA0, pol_w);
+          if (early) {
+            tma_load_2d(st + G::A1, &tmA1, &full_bar[slot], kb * kRowBytes, rowA1, pol_w);
+            tma_load_2d(st + G::S1, &tmS1, &full_bar[slot], kb * 16, rowA1, pol_w);
+          }
           continue;
         }
-        tma_load_2d(st + G::A1, &tmA1, &full_bar[slot], kb * kRowBytes, rowA1, pol_w);
-        tma_load_2d(st + G::S1, &tmS1, &full_bar[slot], kb * 16, rowA1, pol_w);
+        if (!early) {
+          tma_load_2d(st + G::A1, &tmA1, &full_bar[slot], kb * kRowBytes, rowA1, pol_w);
+          tma_load_2d(st + G::S1, &tmS1, &full_bar[slot], kb * 16, rowA1, pol_w);
+        }
         // activation terms: token j's four rows land at B rows 4j..4j+3
         if (btok) {
           for (int j = 0; j < inf.nvalid; ++j)
@@ -293,6 +305,7 @@ __global__ void __launch_bounds__(kBsThreads, 1)
 
   // ================================================================ scale writers
   if (warp < kBsEpiWarp0) {
+    if (early) pdl_wait();  // the B scales are the SwiGLU output
     const int quad = warp - kBsSfWarp0;
     const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
     const int bstride = K / 16;  // bytes per B-scale row
@@ -380,6 +393,7 @@ __global__ void __launch_bounds__(kBsThreads, 1)
   // ================================================================ epilogue
   // Warp 4+q reads TMEM lanes 32q..32q+31: row 32q+lane of both matrices.
   {
+    if (early) pdl_wait();  // the row scales are the SwiGLU output
     const int quad = warp - kBsEpiWarp0;
     const int row = quad * 32 + lane;
     const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;

@@ -104,8 +104,13 @@ __global__ void __launch_bounds__(kF8Threads, 1)
     tmem_relinquish();
   }
   // Launched as a programmatic dependent: everything above overlapped the
-  // previous kernel; from here on its outputs are read.
-  pdl_wait();
+  // previous kernel.  The gate/up step waits for it here.  The down step's
+  // plan and weights do not depend on it (the counts were written by a kernel
+  // that completed before the gate/up step started), so its first weight
+  // copies start at once and only the roles that read the SwiGLU output wait
+  // (griddepcontrol.wait) before their first read of it.
+  const bool early = (p.phase == 2);
+  if (!early) pdl_wait();
   pdl_launch_dependents();
   if (warp == 0) build_plan(p.counts, p.E, NT, pl, lane);
   tc_fence_before();
@@ -130,8 +135,10 @@ __global__ void __launch_bounds__(kF8Threads, 1)
   // ================================================================ producers
   if (warp == kF8ProducerWarp || warp == kF8ProducerWarp2) {
     const bool lead = (warp == kF8ProducerWarp);
+    if (!lead && early) pdl_wait();  // the activation rows are the SwiGLU output
     if (lane == 0 && nst > 0) {
-      tma_prefetch_desc(lead ? &tmA0 : &tmA1);
+      tma_prefetch_desc(&tmA0);
+      tma_prefetch_desc(&tmA1);
       if (!lead) tma_prefetch_desc(&tmB);
       const uint64_t pol_w = policy_evict_first();
       const uint64_t pol_a = policy_evict_last();
@@ -172,10 +179,12 @@ __global__ void __launch_bounds__(kF8Threads, 1)
           bytes += btok ? (uint32_t)inf.nvalid * kF8Terms * kRowBytes
                                   : (uint32_t)BN * kRowBytes;
           mbar_arrive_expect_tx(&full_bar[slot], bytes);
+          // gate/up: box A0; down: both weight boxes (they may be copied early)
           tma_load_2d(st + G::A0, &tmA0, &full_bar[slot], kb * kRowBytes, rowA0, pol_w);
+          if (early) tma_load_2d(st + G::A1, &tmA1, &full_bar[slot], kb * kRowBytes, rowA1, pol_w);
           continue;
         }
-        tma_load_2d(st + G::A1, &tmA1, &full_bar[slot], kb * kRowBytes, rowA1, pol_w);
+        if (!early) tma_load_2d(st + G::A1, &tmA1, &full_bar[slot], kb * kRowBytes, rowA1, pol_w);
         // activation terms: token j's two rows land at B rows 2j, 2j+1
         if (btok) {
           for (int j = 0; j < inf.nvalid; ++j)
@@ -241,6 +250,7 @@ __global__ void __launch_bounds__(kF8Threads, 1)
   // ================================================================ epilogue
   // Warp q reads TMEM lanes 32q..32q+31: row 32q+lane of both boxes.
   {
+    if (early) pdl_wait();  // the row scales are the SwiGLU output
     const int quad = warp - kF8EpiWarp0;
     const int row = quad * 32 + lane;
     const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
