@@ -511,8 +511,9 @@ def run_ours(args):
         "higher_is_better": True,
         "scaling": "weak",
         "vs_baseline": None,
-        "dtype": "nvfp4 weights, f16 MMA with fp32 accumulate" if fmt == 2 else
-                 "fp8 weights, f16 MMA with fp32 accumulate",
+        "dtype": "nvfp4 (e2m1 x e2m1 block-scaled MMA, activations as 4 nvfp4 terms, fp32 accumulate)"
+                 if fmt == 2 else
+                 "fp8 e4m3 (e4m3 x e4m3 MMA, activations as 2 e4m3 terms, fp32 accumulate)",
         "data": "synthetic (seeded N(0,1) activations, N(0,0.02) weights quantised)",
         "config": cfg,
         "hbm_gbs": layer_gbs,
