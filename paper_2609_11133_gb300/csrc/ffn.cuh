@@ -192,6 +192,27 @@ __device__ __forceinline__ void build_plan(const int* counts, int E, int NT, Pla
   }
 }
 
+// Position of a CTA's current stage without divisions: item `it`, K-block
+// `kb` inside it, ring slot and that slot's phase parity ((i / S) & 1).
+template <int S>
+struct StageCursor {
+  int it, kb, KB, slot;
+  uint32_t par;
+  __device__ __forceinline__ StageCursor(int s_begin, int kb_per_item)
+      : it(s_begin / kb_per_item), kb(s_begin - (s_begin / kb_per_item) * kb_per_item),
+        KB(kb_per_item), slot(0), par(0u) {}
+  __device__ __forceinline__ void next() {
+    if (++kb == KB) {
+      kb = 0;
+      ++it;
+    }
+    if (++slot == S) {
+      slot = 0;
+      par ^= 1u;
+    }
+  }
+};
+
 struct ItemInfo {
   int slot, e, arow0, lrow0, nvalid, rt;
 };

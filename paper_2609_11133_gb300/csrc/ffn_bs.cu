@@ -5,16 +5,23 @@
 
 namespace moe {
 
-template <int NT>
-static cudaError_t launch_ffn_bs_nt(int grid, const FfnMaps& m, const FfnParams& p,
+template <int NT, int PHASE>
+static cudaError_t launch_ffn_bs_ph(int grid, const FfnMaps& m, const FfnParams& p,
                                     cudaStream_t st) {
-  auto kern = ffn_bs_kernel<NT>;
+  auto kern = ffn_bs_kernel<NT, PHASE>;
   const int smem = BsGeom<NT>::SMEM;
   static std::atomic<unsigned long long> done{0};
   cudaError_t err = set_smem_once(kern, smem, done);
   if (err != cudaSuccess) return err;
   return launch_pdl(kern, dim3(grid), dim3(kBsThreads), smem, st, m.a0, m.a1, m.s0, m.s1, m.b,
                     p);
+}
+
+template <int NT>
+static cudaError_t launch_ffn_bs_nt(int grid, const FfnMaps& m, const FfnParams& p,
+                                    cudaStream_t st) {
+  return p.phase == 1 ? launch_ffn_bs_ph<NT, 1>(grid, m, p, st)
+                      : launch_ffn_bs_ph<NT, 2>(grid, m, p, st);
 }
 
 cudaError_t launch_ffn_bs(int nt, int grid, const FfnMaps& m, const FfnParams& p,

@@ -91,7 +91,7 @@ __device__ __forceinline__ uint4 ldg_nc_v4(const void* p) {
   return v;
 }
 
-template <int NT>
+template <int NT, int PHASE>
 __global__ void __launch_bounds__(kBsThreads, 1)
     ffn_bs_kernel(const __grid_constant__ CUtensorMap tmA0,
                   const __grid_constant__ CUtensorMap tmA1,
@@ -143,7 +143,7 @@ __global__ void __launch_bounds__(kBsThreads, 1)
   // that completed before the gate/up step started), so its first weight
   // copies start at once and only the roles that read the SwiGLU output wait
   // (griddepcontrol.wait) before their first read of it.
-  const bool early = (p.phase == 2);
+  constexpr bool early = (PHASE == 2);
   if (!early) pdl_wait();
   pdl_launch_dependents();
   if (warp == 0) build_plan(p.counts, p.E, NT, pl, lane);
@@ -152,18 +152,18 @@ __global__ void __launch_bounds__(kBsThreads, 1)
   tc_fence_after();
   const uint32_t tmem = s_tmem;
 
-  const int N = (p.phase == 1) ? p.I : p.H;  // rows of one expert matrix
-  const int K = (p.phase == 1) ? p.H : p.I;  // contraction length
-  const int rtiles = (p.phase == 1) ? p.I / kRowsHalf : p.H / (2 * kRowsHalf);
+  const int N = (PHASE == 1) ? p.I : p.H;  // rows of one expert matrix
+  const int K = (PHASE == 1) ? p.H : p.I;  // contraction length
+  const int rtiles = (PHASE == 1) ? p.I / kRowsHalf : p.H / (2 * kRowsHalf);
   const int KB = K / KEL;
-  const long long items = (long long)pl.cpre[pl.nA] * rtiles;
-  const long long total = items * KB;
-  const long long s_begin = total * blockIdx.x / gridDim.x;
-  const long long s_end = total * (blockIdx.x + 1) / gridDim.x;
-  const long long nst = s_end - s_begin;
-  const uint32_t timeout_bit = (p.phase == 1) ? kStatusTimeoutGateUp : kStatusTimeoutDown;
+  // stages of all items (< 2^31 for every supported shape), this CTA's share
+  const long long total = (long long)pl.cpre[pl.nA] * rtiles * KB;
+  const int s_begin = (int)(total * blockIdx.x / gridDim.x);
+  const int s_end = (int)(total * (blockIdx.x + 1) / gridDim.x);
+  const int nst = s_end - s_begin;
+  const uint32_t timeout_bit = (PHASE == 1) ? kStatusTimeoutGateUp : kStatusTimeoutDown;
   // B rows: per token (phase 1, tokens scattered) or one box per chunk
-  const bool btok = (p.phase == 1) && !p.b_compact;
+  const bool btok = (PHASE == 1) && !p.b_compact;
   constexpr int kTeardown = 9 * 32;  // scale writers, epilogue and MMA warps
 
   // ================================================================ producer
@@ -178,21 +178,20 @@ __global__ void __launch_bounds__(kBsThreads, 1)
       tma_prefetch_desc(&tmB);
       const uint64_t pol_w = policy_evict_first();
       const uint64_t pol_a = policy_evict_last();
-      long long cur_item = -1;
+      int cur_item = -1;
       ItemInfo inf{};
-      long long issued = 0;
-      for (long long s = s_begin; s < s_end; ++s, ++issued) {
-        const long long it = s / KB;
-        const int kb = (int)(s % KB);
+      int issued = 0;
+      for (StageCursor<S> c(s_begin, KB); issued < nst; ++issued, c.next()) {
+        const int it = c.it;
+        const int kb = c.kb;
         if (it != cur_item) {
           cur_item = it;
           inf = decode_item(it, rtiles, pl, p, NT);
           if (!lead && btok)
             for (int j = 0; j < inf.nvalid; ++j) s_tok[j] = __ldg(p.sorted + inf.lrow0 + j) / p.k;
         }
-        const int slot = (int)(issued % S);
-        const uint32_t round = (uint32_t)(issued / S);
-        if (!mbar_wait_bounded(&empty_bar[slot], (round & 1u) ^ 1u, p.wait_ns, &s_abort)) {
+        const int slot = c.slot;
+        if (!mbar_wait_bounded(&empty_bar[slot], c.par ^ 1u, p.wait_ns, &s_abort)) {
           set_status(p.status, timeout_bit);
           s_abort = 1;
           break;
@@ -207,7 +206,7 @@ __global__ void __launch_bounds__(kBsThreads, 1)
         // cannot complete before the arrival below
         if (lead) mbar_arrive_expect_tx(&full_bar[slot], bytes);
         int rowA0, rowA1;
-        if (p.phase == 1) {
+        if (PHASE == 1) {
           rowA0 = inf.e * N + inf.rt * kRowsHalf;
           rowA1 = rowA0;
         } else {
@@ -240,8 +239,8 @@ __global__ void __launch_bounds__(kBsThreads, 1)
       // Let every copy this CTA issued land before the CTA exits (the
       // barriers complete only when both producers' copies have landed).
       if (!lead) return;
-      const long long first = issued > S ? issued - S : 0;
-      for (long long j = first; j < issued; ++j) {
+      const int first = issued > S ? issued - S : 0;
+      for (int j = first; j < issued; ++j) {
         if (p.test_stall && j == 0) continue;
         mbar_wait_bounded(&full_bar[j % S], (uint32_t)((j / S) & 1), p.wait_ns, nullptr);
       }
@@ -253,21 +252,20 @@ __global__ void __launch_bounds__(kBsThreads, 1)
   if (warp == kBsMmaWarp) {
     if (lane == 0) {
       constexpr uint32_t idesc = tc_idesc_mxf4nvf4(128, BN);
-      long long nitem = 0;
+      int nitem = 0;
       bool ok = true;
-      for (long long i = 0; i < nst && ok; ++i) {
-        const long long s = s_begin + i;
-        const int kb = (int)(s % KB);
+      StageCursor<S> c(s_begin, KB);
+      for (int i = 0; i < nst && ok; ++i, c.next()) {
+        const int kb = c.kb;
         const bool first = (i == 0) || (kb == 0);
         const bool last = (i + 1 == nst) || (kb + 1 == KB);
-        const int slot = (int)(i % S);
-        const uint32_t round = (uint32_t)(i / S);
-        const int db = (int)(nitem & 1);
+        const int slot = c.slot;
+        const int db = nitem & 1;
         if (first)
           ok = mbar_wait_bounded(&dempty_bar[db], ((uint32_t)(nitem >> 1) & 1u) ^ 1u, p.wait_ns,
                                  &s_abort);
-        ok = ok && mbar_wait_bounded(&full_bar[slot], round & 1u, p.wait_ns, &s_abort) &&
-             mbar_wait_bounded(&sf_bar[slot], round & 1u, p.wait_ns, &s_abort);
+        ok = ok && mbar_wait_bounded(&full_bar[slot], c.par, p.wait_ns, &s_abort) &&
+             mbar_wait_bounded(&sf_bar[slot], c.par, p.wait_ns, &s_abort);
         if (!ok) break;
         tc_fence_after();
         const uint32_t st = smem_u32(smem + (size_t)slot * G::BYTES);
@@ -309,13 +307,13 @@ __global__ void __launch_bounds__(kBsThreads, 1)
     const int quad = warp - kBsSfWarp0;
     const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
     const int bstride = K / 16;  // bytes per B-scale row
-    long long cur_item = -1;
+    int cur_item = -1;
     ItemInfo inf{};
     int grow[2] = {-1, -1};  // global B-scale rows of B rows lane and lane + 32
-    for (long long i = 0; i < nst; ++i) {
-      const long long s = s_begin + i;
-      const long long it = s / KB;
-      const int kb = (int)(s % KB);
+    StageCursor<S> c(s_begin, KB);
+    for (int i = 0; i < nst; ++i, c.next()) {
+      const int it = c.it;
+      const int kb = c.kb;
       if (it != cur_item) {
         cur_item = it;
         inf = decode_item(it, rtiles, pl, p, NT);
@@ -337,12 +335,11 @@ __global__ void __launch_bounds__(kBsThreads, 1)
         bsf[h] = (grow[h] >= 0)
                      ? ldg_nc_v4(p.bsf + (size_t)grow[h] * bstride + 16 * kb)
                      : make_uint4(0u, 0u, 0u, 0u);
-      const int slot = (int)(i % S);
-      const uint32_t round = (uint32_t)(i / S);
+      const int slot = c.slot;
       // the MMAs that read this slot's scales last round are done, and this
       // round's A scales have landed
-      if (!mbar_wait_bounded(&empty_bar[slot], (round & 1u) ^ 1u, p.wait_ns, &s_abort) ||
-          !mbar_wait_bounded(&full_bar[slot], round & 1u, p.wait_ns, &s_abort)) {
+      if (!mbar_wait_bounded(&empty_bar[slot], c.par ^ 1u, p.wait_ns, &s_abort) ||
+          !mbar_wait_bounded(&full_bar[slot], c.par, p.wait_ns, &s_abort)) {
         set_status(p.status, timeout_bit);
         s_abort = 1;
         break;
@@ -398,10 +395,10 @@ __global__ void __launch_bounds__(kBsThreads, 1)
     const int row = quad * 32 + lane;
     const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
     bool dead = false;
-    long long nitem = 0;
+    int nitem = 0;
     if (nst > 0) {
-      const long long it0 = s_begin / KB, it1 = (s_end - 1) / KB;
-      for (long long it = it0; it <= it1 && !dead; ++it, ++nitem) {
+      const int it0 = s_begin / KB, it1 = (s_end - 1) / KB;
+      for (int it = it0; it <= it1 && !dead; ++it, ++nitem) {
         const ItemInfo inf = decode_item(it, rtiles, pl, p, NT);
         const int db = (int)(nitem & 1);
         if (!mbar_wait_bounded(&dfull_bar[db], (uint32_t)(nitem >> 1) & 1u, p.wait_ns,
@@ -437,7 +434,7 @@ __global__ void __launch_bounds__(kBsThreads, 1)
           if (j >= inf.nvalid) continue;
           const int arow = inf.arow0 + j;
           const int a = __ldg(p.sorted + inf.lrow0 + j);
-          if (p.phase == 1) {
+          if (PHASE == 1) {
             const float sc = __ldg(p.xinv + a / p.k);
             const int f = inf.rt * kRowsHalf + row;
             float* gr = p.gu + (size_t)arow * 2 * p.I + f;

@@ -60,7 +60,7 @@ __device__ __forceinline__ void tc_mma_f8(uint32_t d_tmem, uint64_t a_desc, uint
       : "memory");
 }
 
-template <int NT>
+template <int NT, int PHASE>
 __global__ void __launch_bounds__(kF8Threads, 1)
     ffn_f8_kernel(const __grid_constant__ CUtensorMap tmA0,
                   const __grid_constant__ CUtensorMap tmA1,
@@ -109,7 +109,7 @@ __global__ void __launch_bounds__(kF8Threads, 1)
   // that completed before the gate/up step started), so its first weight
   // copies start at once and only the roles that read the SwiGLU output wait
   // (griddepcontrol.wait) before their first read of it.
-  const bool early = (p.phase == 2);
+  constexpr bool early = (PHASE == 2);
   if (!early) pdl_wait();
   pdl_launch_dependents();
   if (warp == 0) build_plan(p.counts, p.E, NT, pl, lane);
@@ -118,18 +118,18 @@ __global__ void __launch_bounds__(kF8Threads, 1)
   tc_fence_after();
   const uint32_t tmem = s_tmem;
 
-  const int N = (p.phase == 1) ? p.I : p.H;  // rows of one expert matrix
-  const int K = (p.phase == 1) ? p.H : p.I;  // contraction length
-  const int rtiles = (p.phase == 1) ? p.I / kRowsHalf : p.H / (2 * kRowsHalf);
+  const int N = (PHASE == 1) ? p.I : p.H;  // rows of one expert matrix
+  const int K = (PHASE == 1) ? p.H : p.I;  // contraction length
+  const int rtiles = (PHASE == 1) ? p.I / kRowsHalf : p.H / (2 * kRowsHalf);
   const int KB = K / KEL;
-  const long long items = (long long)pl.cpre[pl.nA] * rtiles;
-  const long long total = items * KB;
-  const long long s_begin = total * blockIdx.x / gridDim.x;
-  const long long s_end = total * (blockIdx.x + 1) / gridDim.x;
-  const long long nst = s_end - s_begin;
-  const uint32_t timeout_bit = (p.phase == 1) ? kStatusTimeoutGateUp : kStatusTimeoutDown;
+  // stages of all items (< 2^31 for every supported shape), this CTA's share
+  const long long total = (long long)pl.cpre[pl.nA] * rtiles * KB;
+  const int s_begin = (int)(total * blockIdx.x / gridDim.x);
+  const int s_end = (int)(total * (blockIdx.x + 1) / gridDim.x);
+  const int nst = s_end - s_begin;
+  const uint32_t timeout_bit = (PHASE == 1) ? kStatusTimeoutGateUp : kStatusTimeoutDown;
   // B rows: per token (phase 1, tokens scattered) or one box per chunk
-  const bool btok = (p.phase == 1) && !p.b_compact;
+  const bool btok = (PHASE == 1) && !p.b_compact;
   constexpr int kTeardown = 5 * 32;  // epilogue and MMA warps
 
   // ================================================================ producers
@@ -142,21 +142,20 @@ __global__ void __launch_bounds__(kF8Threads, 1)
       if (!lead) tma_prefetch_desc(&tmB);
       const uint64_t pol_w = policy_evict_first();
       const uint64_t pol_a = policy_evict_last();
-      long long cur_item = -1;
+      int cur_item = -1;
       ItemInfo inf{};
-      long long issued = 0;
-      for (long long s = s_begin; s < s_end; ++s, ++issued) {
-        const long long it = s / KB;
-        const int kb = (int)(s % KB);
+      int issued = 0;
+      for (StageCursor<S> c(s_begin, KB); issued < nst; ++issued, c.next()) {
+        const int it = c.it;
+        const int kb = c.kb;
         if (it != cur_item) {
           cur_item = it;
           inf = decode_item(it, rtiles, pl, p, NT);
           if (!lead && btok)
             for (int j = 0; j < inf.nvalid; ++j) s_tok[j] = __ldg(p.sorted + inf.lrow0 + j) / p.k;
         }
-        const int slot = (int)(issued % S);
-        const uint32_t round = (uint32_t)(issued / S);
-        if (!mbar_wait_bounded(&empty_bar[slot], (round & 1u) ^ 1u, p.wait_ns, &s_abort)) {
+        const int slot = c.slot;
+        if (!mbar_wait_bounded(&empty_bar[slot], c.par ^ 1u, p.wait_ns, &s_abort)) {
           set_status(p.status, timeout_bit);
           s_abort = 1;
           break;
@@ -164,7 +163,7 @@ __global__ void __launch_bounds__(kF8Threads, 1)
         if (p.test_stall && issued == 0) continue;  // test hook: this stage never arrives
         unsigned char* st = smem + (size_t)slot * G::BYTES;
         int rowA0, rowA1;
-        if (p.phase == 1) {
+        if (PHASE == 1) {
           rowA0 = inf.e * N + inf.rt * kRowsHalf;
           rowA1 = rowA0;
         } else {
@@ -198,8 +197,8 @@ __global__ void __launch_bounds__(kF8Threads, 1)
       // Let every copy land before the CTA exits (the barriers complete only
       // when both producers' copies have landed).
       if (!lead) return;
-      const long long first = issued > S ? issued - S : 0;
-      for (long long j = first; j < issued; ++j) {
+      const int first = issued > S ? issued - S : 0;
+      for (int j = first; j < issued; ++j) {
         if (p.test_stall && j == 0) continue;
         mbar_wait_bounded(&full_bar[j % S], (uint32_t)((j / S) & 1), p.wait_ns, nullptr);
       }
@@ -212,12 +211,13 @@ __global__ void __launch_bounds__(kF8Threads, 1)
     if (lane == 0) {
       constexpr uint32_t idesc = tc_idesc_e4m3(128, BN);
       bool ok = true;
-      for (long long i = 0; i < nst && ok; ++i) {
-        const int slot = (int)(i % S);
-        const int db = (int)(i % DR);
-        ok = mbar_wait_bounded(&dempty_bar[db], ((uint32_t)(i / DR) & 1u) ^ 1u, p.wait_ns,
-                               &s_abort) &&
-             mbar_wait_bounded(&full_bar[slot], (uint32_t)(i / S) & 1u, p.wait_ns, &s_abort);
+      StageCursor<S> c(s_begin, KB);
+      StageCursor<DR> d(0, 1);  // accumulator ring position
+      for (int i = 0; i < nst && ok; ++i, c.next(), d.next()) {
+        const int slot = c.slot;
+        const int db = d.slot;
+        ok = mbar_wait_bounded(&dempty_bar[db], d.par ^ 1u, p.wait_ns, &s_abort) &&
+             mbar_wait_bounded(&full_bar[slot], c.par, p.wait_ns, &s_abort);
         if (!ok) break;
         tc_fence_after();
         const uint32_t st = smem_u32(smem + (size_t)slot * G::BYTES);
@@ -259,11 +259,10 @@ __global__ void __launch_bounds__(kF8Threads, 1)
 #pragma unroll
     for (int j = 0; j < NT; ++j) acc0[j] = acc1[j] = 0.f;
     bool dead = false;
-    long long cur_item = -1;
     ItemInfo inf{};
     // the block scales of a stage's two boxes
     auto scales = [&](const ItemInfo& f, int kb, float& b0, float& b1) {
-      if (p.phase == 1) {
+      if (PHASE == 1) {
         const size_t tile = ((size_t)f.e * (N / 128) + f.rt) * KB128 + kb;
         b0 = __ldg(p.s0 + tile);
         b1 = __ldg(p.s1 + tile);
@@ -274,24 +273,22 @@ __global__ void __launch_bounds__(kF8Threads, 1)
       }
     };
     float bs0 = 0.f, bs1 = 0.f;
+    StageCursor<DR> c(s_begin, KB);  // it, kb of this stage; slot = accumulator ring slot
     if (nst > 0) {
-      inf = decode_item(s_begin / KB, rtiles, pl, p, NT);
-      cur_item = s_begin / KB;
-      scales(inf, (int)(s_begin % KB), bs0, bs1);
+      inf = decode_item(c.it, rtiles, pl, p, NT);
+      scales(inf, c.kb, bs0, bs1);
     }
-    for (long long i = 0; i < nst && !dead; ++i) {
-      const long long s = s_begin + i;
-      const long long it = s / KB;
+    for (int i = 0; i < nst && !dead; ++i) {
       // the next stage's scales, loaded while this stage's accumulator is awaited
       float nb0 = 0.f, nb1 = 0.f;
       ItemInfo ninf = inf;
+      const bool closes = (i + 1 == nst) || (c.kb + 1 == KB);
       if (i + 1 < nst) {
-        const long long it1 = (s + 1) / KB;
-        if (it1 != it) ninf = decode_item(it1, rtiles, pl, p, NT);
-        scales(ninf, (int)((s + 1) % KB), nb0, nb1);
+        if (c.kb + 1 == KB) ninf = decode_item(c.it + 1, rtiles, pl, p, NT);
+        scales(ninf, c.kb + 1 == KB ? 0 : c.kb + 1, nb0, nb1);
       }
-      const int db = (int)(i % DR);
-      if (!mbar_wait_bounded(&dfull_bar[db], (uint32_t)(i / DR) & 1u, p.wait_ns, &s_abort)) {
+      const int db = c.slot;
+      if (!mbar_wait_bounded(&dfull_bar[db], c.par, p.wait_ns, &s_abort)) {
         set_status(p.status, timeout_bit);
         s_abort = 1;
         dead = true;
@@ -320,14 +317,13 @@ __global__ void __launch_bounds__(kF8Threads, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&dempty_bar[db]);
-      const bool closes = (i + 1 == nst) || ((s + 1) / KB != it);
       if (closes) {
 #pragma unroll
         for (int j = 0; j < NT; ++j) {
           if (j < inf.nvalid) {
             const int arow = inf.arow0 + j;
             const int a = __ldg(p.sorted + inf.lrow0 + j);
-            if (p.phase == 1) {
+            if (PHASE == 1) {
               const float sc = __ldg(p.xinv + a / p.k);
               const int f = inf.rt * kRowsHalf + row;
               float* gr = p.gu + (size_t)arow * 2 * p.I + f;
@@ -352,11 +348,10 @@ __global__ void __launch_bounds__(kF8Threads, 1)
         }
       }
       inf = ninf;
-      cur_item = (s + 1) / KB;
       bs0 = nb0;
       bs1 = nb1;
+      c.next();
     }
-    (void)cur_item;
     tc_fence_before();
     asm volatile("bar.sync 2, %0;" ::"n"(kTeardown) : "memory");
   }

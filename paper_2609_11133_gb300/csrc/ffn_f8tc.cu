@@ -5,15 +5,22 @@
 
 namespace moe {
 
-template <int NT>
-static cudaError_t launch_ffn_f8_nt(int grid, const FfnMaps& m, const FfnParams& p,
+template <int NT, int PHASE>
+static cudaError_t launch_ffn_f8_ph(int grid, const FfnMaps& m, const FfnParams& p,
                                     cudaStream_t st) {
-  auto kern = ffn_f8_kernel<NT>;
+  auto kern = ffn_f8_kernel<NT, PHASE>;
   const int smem = F8Geom<NT>::SMEM;
   static std::atomic<unsigned long long> done{0};
   cudaError_t err = set_smem_once(kern, smem, done);
   if (err != cudaSuccess) return err;
   return launch_pdl(kern, dim3(grid), dim3(kF8Threads), smem, st, m.a0, m.a1, m.b, p);
+}
+
+template <int NT>
+static cudaError_t launch_ffn_f8_nt(int grid, const FfnMaps& m, const FfnParams& p,
+                                    cudaStream_t st) {
+  return p.phase == 1 ? launch_ffn_f8_ph<NT, 1>(grid, m, p, st)
+                      : launch_ffn_f8_ph<NT, 2>(grid, m, p, st);
 }
 
 cudaError_t launch_ffn_f8(int nt, int grid, const FfnMaps& m, const FfnParams& p,
