@@ -60,8 +60,10 @@ struct BsGeom {
   static constexpr int STAGES_RAW = (212 * 1024) / BYTES;  // + ~10 KB static
   static constexpr int STAGES = STAGES_RAW > 8 ? 8 : STAGES_RAW;
   static constexpr int SMEM = STAGES * BYTES + 1024;
-  // tensor memory: accumulators D[db][mat] (BN columns each), then per-stage scales
-  static constexpr uint32_t D_COLS = 4 * BN;
+  // tensor memory: accumulators D[db][mat] (BN columns each; ND items in
+  // flight between the MMA and the epilogue), then per-stage scales
+  static constexpr int ND = (NT == 8) ? 3 : 2;
+  static constexpr uint32_t D_COLS = 2 * ND * BN;
   static_assert(D_COLS + STAGES * kBsSfCols <= kBsTmemCols, "tensor memory budget");
   static_assert(B % 1024 == 0, "B tile must start a swizzle atom");
 };
@@ -109,8 +111,8 @@ __global__ void __launch_bounds__(kBsThreads, 1)
   __shared__ __align__(8) uint64_t full_bar[S];
   __shared__ __align__(8) uint64_t empty_bar[S];
   __shared__ __align__(8) uint64_t sf_bar[S];
-  __shared__ __align__(8) uint64_t dfull_bar[2];
-  __shared__ __align__(8) uint64_t dempty_bar[2];
+  __shared__ __align__(8) uint64_t dfull_bar[G::ND];
+  __shared__ __align__(8) uint64_t dempty_bar[G::ND];
   __shared__ __align__(8) uint64_t final_bar;
   __shared__ PlanSmem pl;
   __shared__ int s_tok[NT];
@@ -126,7 +128,7 @@ __global__ void __launch_bounds__(kBsThreads, 1)
       mbar_init(&empty_bar[i], 1);
       mbar_init(&sf_bar[i], 4);
     }
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < G::ND; ++i) {
       mbar_init(&dfull_bar[i], 1);
       mbar_init(&dempty_bar[i], 4);
     }
@@ -213,16 +215,20 @@ __global__ void __launch_bounds__(kBsThreads, 1)
           rowA0 = inf.e * N + inf.rt * 2 * kRowsHalf;
           rowA1 = rowA0 + kRowsHalf;
         }
-        if (lead) {  // gate/up: box A0; down: all weights (they may be copied early)
+        // Box A0 (and its scales) always come from the lead producer, box A1
+        // from the second one - except for the down step's first ring of
+        // stages, whose weights the lead copies before the SwiGLU kernel ends.
+        const bool a1_lead = early && issued < S;
+        if (lead) {
           tma_load_2d(st + G::A0, &tmA0, &full_bar[slot], kb * kRowBytes, rowA0, pol_w);
           tma_load_2d(st + G::S0, &tmS0, &full_bar[slot], kb * 16, rowA0, pol_w);
-          if (early) {
+          if (a1_lead) {
             tma_load_2d(st + G::A1, &tmA1, &full_bar[slot], kb * kRowBytes, rowA1, pol_w);
             tma_load_2d(st + G::S1, &tmS1, &full_bar[slot], kb * 16, rowA1, pol_w);
           }
           continue;
         }
-        if (!early) {
+        if (!a1_lead) {
           tma_load_2d(st + G::A1, &tmA1, &full_bar[slot], kb * kRowBytes, rowA1, pol_w);
           tma_load_2d(st + G::S1, &tmS1, &full_bar[slot], kb * 16, rowA1, pol_w);
         }
@@ -260,10 +266,10 @@ __global__ void __launch_bounds__(kBsThreads, 1)
         const bool first = (i == 0) || (kb == 0);
         const bool last = (i + 1 == nst) || (kb + 1 == KB);
         const int slot = c.slot;
-        const int db = nitem & 1;
+        const int db = nitem % G::ND;
         if (first)
-          ok = mbar_wait_bounded(&dempty_bar[db], ((uint32_t)(nitem >> 1) & 1u) ^ 1u, p.wait_ns,
-                                 &s_abort);
+          ok = mbar_wait_bounded(&dempty_bar[db], ((uint32_t)(nitem / G::ND) & 1u) ^ 1u,
+                                 p.wait_ns, &s_abort);
         ok = ok && mbar_wait_bounded(&full_bar[slot], c.par, p.wait_ns, &s_abort) &&
              mbar_wait_bounded(&sf_bar[slot], c.par, p.wait_ns, &s_abort);
         if (!ok) break;
@@ -310,13 +316,13 @@ __global__ void __launch_bounds__(kBsThreads, 1)
     int cur_item = -1;
     ItemInfo inf{};
     int grow[2] = {-1, -1};  // global B-scale rows of B rows lane and lane + 32
-    StageCursor<S> c(s_begin, KB);
-    for (int i = 0; i < nst; ++i, c.next()) {
-      const int it = c.it;
-      const int kb = c.kb;
-      if (it != cur_item) {
-        cur_item = it;
-        inf = decode_item(it, rtiles, pl, p, NT);
+    // B scales (16 bytes per row: 4 MMAs x 4 blocks) are loaded one stage
+    // ahead, by a second cursor
+    StageCursor<S> cn(s_begin, KB);
+    auto load_bsf = [&](uint4 (&out)[2]) {
+      if (cn.it != cur_item) {
+        cur_item = cn.it;
+        inf = decode_item(cn.it, rtiles, pl, p, NT);
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
           const int n = lane + 32 * h;
@@ -328,13 +334,17 @@ __global__ void __launch_bounds__(kBsThreads, 1)
           }
         }
       }
-      // B scales of this stage (16 bytes per row: 4 MMAs x 4 blocks)
-      uint4 bsf[2];
 #pragma unroll
       for (int h = 0; h < 2; ++h)
-        bsf[h] = (grow[h] >= 0)
-                     ? ldg_nc_v4(p.bsf + (size_t)grow[h] * bstride + 16 * kb)
-                     : make_uint4(0u, 0u, 0u, 0u);
+        out[h] = (grow[h] >= 0) ? ldg_nc_v4(p.bsf + (size_t)grow[h] * bstride + 16 * cn.kb)
+                                : make_uint4(0u, 0u, 0u, 0u);
+      cn.next();
+    };
+    uint4 bsf[2], bnext[2];
+    if (nst > 0) load_bsf(bsf);
+    StageCursor<S> c(s_begin, KB);
+    for (int i = 0; i < nst; ++i, c.next()) {
+      if (i + 1 < nst) load_bsf(bnext);
       const int slot = c.slot;
       // the MMAs that read this slot's scales last round are done, and this
       // round's A scales have landed
@@ -381,6 +391,8 @@ __global__ void __launch_bounds__(kBsThreads, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&sf_bar[slot]);
+      bsf[0] = bnext[0];
+      bsf[1] = bnext[1];
     }
     tc_fence_before();
     asm volatile("bar.sync 2, %0;" ::"n"(kTeardown) : "memory");
@@ -400,8 +412,8 @@ __global__ void __launch_bounds__(kBsThreads, 1)
       const int it0 = s_begin / KB, it1 = (s_end - 1) / KB;
       for (int it = it0; it <= it1 && !dead; ++it, ++nitem) {
         const ItemInfo inf = decode_item(it, rtiles, pl, p, NT);
-        const int db = (int)(nitem & 1);
-        if (!mbar_wait_bounded(&dfull_bar[db], (uint32_t)(nitem >> 1) & 1u, p.wait_ns,
+        const int db = nitem % G::ND;
+        if (!mbar_wait_bounded(&dfull_bar[db], (uint32_t)(nitem / G::ND) & 1u, p.wait_ns,
                                &s_abort)) {
           set_status(p.status, timeout_bit);
           s_abort = 1;

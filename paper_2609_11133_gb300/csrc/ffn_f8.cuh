@@ -178,12 +178,15 @@ __global__ void __launch_bounds__(kF8Threads, 1)
           bytes += btok ? (uint32_t)inf.nvalid * kF8Terms * kRowBytes
                                   : (uint32_t)BN * kRowBytes;
           mbar_arrive_expect_tx(&full_bar[slot], bytes);
-          // gate/up: box A0; down: both weight boxes (they may be copied early)
+          // box A0 always; box A1 too for the down step's first ring of
+          // stages, copied before the SwiGLU kernel ends
           tma_load_2d(st + G::A0, &tmA0, &full_bar[slot], kb * kRowBytes, rowA0, pol_w);
-          if (early) tma_load_2d(st + G::A1, &tmA1, &full_bar[slot], kb * kRowBytes, rowA1, pol_w);
+          if (early && issued < S)
+            tma_load_2d(st + G::A1, &tmA1, &full_bar[slot], kb * kRowBytes, rowA1, pol_w);
           continue;
         }
-        if (!early) tma_load_2d(st + G::A1, &tmA1, &full_bar[slot], kb * kRowBytes, rowA1, pol_w);
+        if (!(early && issued < S))
+          tma_load_2d(st + G::A1, &tmA1, &full_bar[slot], kb * kRowBytes, rowA1, pol_w);
         // activation terms: token j's two rows land at B rows 2j, 2j+1
         if (btok) {
           for (int j = 0; j < inf.nvalid; ++j)
