@@ -63,7 +63,7 @@ def workload(args):
     return wl
 
 
-def parse():
+def parse(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=200)
@@ -74,7 +74,7 @@ def parse():
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-energy", action="store_true")
-    return ap.parse_args()
+    return ap.parse_args(argv)
 
 
 # ---------------------------------------------------------------- distributed
@@ -86,14 +86,23 @@ def dist_env():
 
 
 def barrier_max(value, world):
-    """Barrier, then the maximum of `value` over ranks."""
+    """Barrier, then the maximum of `value` over ranks (an all-reduce, so every
+    rank returns the slowest rank's figure).  The reduction buffer lives where
+    the process group's backend wants it: the GPU for nccl, the host for gloo."""
     if world == 1:
         return value
     import torch
     import torch.distributed as dist
-    t = torch.tensor([value], dtype=torch.float64, device="cuda")
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([value], dtype=torch.float64, device=dev)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def job_throughput(ms_step_max, tokens_per_rank, world):
+    """Whole-job tokens/s of `world` replicas, each decoding `tokens_per_rank`
+    tokens per step, paced by the slowest rank's step time."""
+    return world * tokens_per_rank / (ms_step_max * 1e-3)
 
 
 def barrier(world):
@@ -410,7 +419,7 @@ def run_ours(args):
     h_end = time.perf_counter()
     ms_total = t_beg.elapsed_time(t_end)
     ms_step = barrier_max(ms_total / args.steps, world)
-    tok_s = world * T / (ms_step * 1e-3)
+    tok_s = job_throughput(ms_step, T, world)
 
     # ---- energy per token (NVML counter over >= 2 s of back-to-back steps)
     energy = None
@@ -525,7 +534,7 @@ def run_ours(args):
         "roofline": {"bound": "hbm", "achieved": gu_gbs, "peak": hbm, "unit": "GB/s",
                      "frac": gu_gbs / hbm, "traffic": traffic, "kernel": "ffn gate/up",
                      "peak_source": peak_src},
-        "e2e": {"value": world * T / (ms_e2e * 1e-3), "unit": "tokens/s",
+        "e2e": {"value": job_throughput(ms_e2e, T, world), "unit": "tokens/s",
                 "h2d_bytes_per_step": T * H * 2, "d2h_bytes_per_step": T * H * 2},
         "gpu_launches": 5 * L * args.steps,
         "timing": "CUDA-graph replay of one step's layer calls per step",
