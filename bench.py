@@ -60,6 +60,10 @@ def workload(args):
     wl.update(WORKLOADS[args.workload])
     if args.tokens is not None:
         wl["T"] = args.tokens
+    if args.experts is not None:
+        wl["E"] = args.experts
+    wl["name"] = args.workload + (f"_E{wl['E']}" if args.experts is not None else "") \
+        + f"_T{wl['T']}"
     return wl
 
 
@@ -71,6 +75,9 @@ def parse(argv=None):
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="qwen3_235b_nvfp4", choices=sorted(WORKLOADS))
     ap.add_argument("--tokens", type=int, default=None, help="batch size (default per workload)")
+    ap.add_argument("--experts", type=int, default=None,
+                    help="expert count (default per workload); a smaller count keeps the "
+                         "layer's per-expert shapes with less memory, for profiler captures")
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-energy", action="store_true")
@@ -367,30 +374,60 @@ def run_ours(args):
                                             topk_ids_out=None if ids is None else ids[l])
         return io(L - 1, x_in)[2]
 
-    # routing of this batch -> unique experts per layer -> algorithmic bytes
-    ids = [torch.empty((T, k), dtype=torch.int32, device=dev) for _ in range(L)]
-    run_layers(x, ids=ids)
-    torch.cuda.synchronize()
-    assert binding.moe_read_status(ws) == 0
-    n_active = [int(torch.unique(i).numel()) for i in ids]
+    def touched(x_in):
+        """Unique experts per layer of one batch, and the step's algorithmic bytes."""
+        ids = [torch.empty((T, k), dtype=torch.int32, device=dev) for _ in range(L)]
+        run_layers(x_in, ids=ids)
+        torch.cuda.synchronize()
+        assert binding.moe_read_status(ws) == 0
+        n = [int(torch.unique(i).numel()) for i in ids]
+        return n, ids, sum(router_bytes + a * per_expert + act_bytes for a in n)
+
     w0 = layers[0][0]
     per_expert = w0.nbytes_expert()
     gu_bytes, dn_bytes = expert_bytes(w0)
     router_bytes = E * H * 4
     act_bytes = 2 * T * H * 2  # x in, out
-    B = sum(router_bytes + n * per_expert + act_bytes for n in n_active)
+    n_active, ids, B = touched(x)
+
+    # Steps rotate over distinct input batches, all resident before timing,
+    # when one step touches less than four times L2: consecutive steps then
+    # route to different experts and a step does not find the weights of the
+    # previous ones in L2.
+    l2 = torch.cuda.get_device_properties(0).L2_cache_size
+    n_rot = 1 if B >= 4 * l2 else min(16, math.ceil(4 * l2 / B))
+    xs = [x] + [synth.make_x(T, H, seed=args.seed + rank + 7919 * r, device=dev)
+                for r in range(1, n_rot)]
+    if n_rot > 1:
+        rot = [touched(xr) for xr in xs]
+        n_active = [statistics.mean(r[0][l] for r in rot) for l in range(L)]
+        B = statistics.mean(r[2] for r in rot)
+    # Steps per CUDA graph: one rotation cycle, at least eight layer calls.
+    # Within a graph the layer calls follow one another as in a decode loop;
+    # the host takes no decision between them.
+    G = n_rot * max(1, math.ceil(8 / (n_rot * L)))
+
+    def capture(nsteps, body):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            for s_ in range(nsteps):
+                body(s_ % n_rot)
+        return g
+
+    def timed(g_full, g_rem, steps):
+        """Replays that run exactly `steps` steps."""
+        for _ in range(steps // G):
+            g_full.replay()
+        if g_rem is not None:
+            g_rem.replay()
 
     for _ in range(max(3, args.warmup)):
         run_layers(x)
     torch.cuda.synchronize()
 
-    # The step's layer calls captured in one CUDA graph: the timed loop replays
-    # it, so the host's launch work is not part of the measurement (the layer
-    # takes no host-side decisions between its kernels).
-    g_step = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(g_step):
-        out = run_layers(x)
-    for _ in range(max(3, args.warmup)):
+    g_step = capture(G, lambda r: run_layers(xs[r]))
+    g_rem = capture(args.steps % G, lambda r: run_layers(xs[r])) if args.steps % G else None
+    for _ in range(max(3, math.ceil(args.warmup / G))):
         g_step.replay()
     torch.cuda.synchronize()
     barrier(world)
@@ -412,8 +449,7 @@ def run_ours(args):
     barrier(world)
     h_beg = time.perf_counter()
     t_beg.record(stream)
-    for _ in range(args.steps):
-        g_step.replay()
+    timed(g_step, g_rem, args.steps)
     t_end.record(stream)
     torch.cuda.synchronize()
     h_end = time.perf_counter()
@@ -426,7 +462,7 @@ def run_ours(args):
     if not args.no_energy:
         nv = Nvml(local)
         if nv.ok:
-            n_rep = max(1, int(2.0 / (ms_step * 1e-3)))
+            n_rep = max(1, int(2.0 / (ms_step * 1e-3 * G)))
             torch.cuda.synchronize()
             j0 = nv.energy_mj()
             t0 = time.perf_counter()
@@ -436,32 +472,37 @@ def run_ours(args):
             h_end = time.perf_counter()
             dt = h_end - t0
             j1 = nv.energy_mj()
-            energy = {"j_per_token": (j1 - j0) * 1e-3 / (n_rep * T), "avg_w": (j1 - j0) * 1e-3 / dt,
+            energy = {"j_per_token": (j1 - j0) * 1e-3 / (n_rep * G * T),
+                      "avg_w": (j1 - j0) * 1e-3 / dt,
                       "window_s": dt, "source": "nvmlDeviceGetTotalEnergyConsumption"}
     clk = clocks.stop(h_beg, h_end)
-    clk["window"] = "timed region" + (" + energy window (same step replayed)" if energy else "")
+    clk["window"] = "timed region" + (" + energy window (same steps replayed)" if energy else "")
 
     # per-kernel durations: eager calls with events between the kernels
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(L)]
     kern = [[], [], []]
-    for _ in range(max(1, min(args.steps, 20 if L == 1 else 2))):
-        run_layers(x, ev=ev)
+    for i_ in range(max(1, min(args.steps, 20 if L == 1 else 2))):
+        run_layers(xs[i_ % n_rot], ev=ev)
         torch.cuda.synchronize()
         for i in range(3):
             kern[i].append(sum(ev[l][i].elapsed_time(ev[l][i + 1]) for l in range(L)))
 
-    # ---- end to end through the public API with host buffers: the input is
-    # copied from pinned host memory, the step runs, the output is copied
-    # back, every step (captured together in one graph)
-    x_host = torch.empty((T, H), dtype=torch.bfloat16, pin_memory=True)
-    x_host.copy_(x.cpu())
+    # ---- end to end through the public API with host buffers: every step
+    # copies its input from pinned host memory, runs, and copies its output
+    # back (the same steps per graph and the same input rotation)
+    x_host = [torch.empty((T, H), dtype=torch.bfloat16, pin_memory=True) for _ in range(n_rot)]
+    for xh, xr in zip(x_host, xs):
+        xh.copy_(xr.cpu())
     out_host = torch.empty((T, H), dtype=torch.bfloat16, pin_memory=True)
     x_dev = torch.empty_like(x)
-    g_e2e = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(g_e2e):
-        x_dev.copy_(x_host, non_blocking=True)
-        out_e2e = run_layers(x_dev)
-        out_host.copy_(out_e2e, non_blocking=True)
+
+    def e2e_step(r):
+        x_dev.copy_(x_host[r], non_blocking=True)
+        o = run_layers(x_dev)
+        out_host.copy_(o, non_blocking=True)
+
+    g_e2e = capture(G, e2e_step)
+    g_e2e_rem = capture(args.steps % G, e2e_step) if args.steps % G else None
     for _ in range(3):
         g_e2e.replay()
     torch.cuda.synchronize()
@@ -469,8 +510,7 @@ def run_ours(args):
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record(stream)
-    for _ in range(args.steps):
-        g_e2e.replay()
+    timed(g_e2e, g_e2e_rem, args.steps)
     e1.record(stream)
     torch.cuda.synchronize()
     ms_e2e = barrier_max(e0.elapsed_time(e1) / args.steps, world)
@@ -494,14 +534,18 @@ def run_ours(args):
     traffic = None
     tp = os.path.join(ROOT, "profiles", "traffic.json")
     if os.path.exists(tp):
-        tj = json.load(open(tp)).get(f"{args.workload}_T{T}")
+        tj = json.load(open(tp)).get(wl["name"])
         if tj and kernel_sources_sha256() == tj.get("kernel_sources_sha256"):
             traffic = tj.get("gateup_dram_bytes")
 
-    cfg = {"workload": f"{args.workload}_T{T}", "H": H, "E": E, "k": k, "I": I,
+    cfg = {"workload": wl["name"], "H": H, "E": E, "k": k, "I": I,
            "tokens": T, "format": "nvfp4" if fmt == 2 else "fp8_block128",
            "active_experts": n_active[0] if L == 1 else statistics.mean(n_active),
-           "l2": f"inputs larger than L2: {B / 1e9:.2f} GB of weights touched per step",
+           "l2": (f"inputs larger than L2: {B / 1e9:.2f} GB of weights touched per step"
+                  if n_rot == 1 else
+                  f"{n_rot} resident input batches rotated step by step: {B / 1e9:.3f} GB "
+                  f"touched per step, {n_rot * B / 1e9:.2f} GB per rotation (L2 {l2 / 1e6:.0f} MB)"),
+           "steps_per_graph": G,
            "parallelism": f"replicas x{world}"}
     if L > 1:
         cfg.update(layers=L, prenorm="rms, eps 1e-6, unit weight", residual="threaded",
@@ -537,7 +581,7 @@ def run_ours(args):
         "e2e": {"value": job_throughput(ms_e2e, T, world), "unit": "tokens/s",
                 "h2d_bytes_per_step": T * H * 2, "d2h_bytes_per_step": T * H * 2},
         "gpu_launches": 5 * L * args.steps,
-        "timing": "CUDA-graph replay of one step's layer calls per step",
+        "timing": f"CUDA-graph replay, {G} steps (layer calls) per graph",
         "clocks": clk,
         "energy": energy,
     }
@@ -571,7 +615,7 @@ def run_reference(args):
            "steps": steps, "warmup": warm, "ms_per_step": dt * L * 1e3 * T / s.n,
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
            "data": "synthetic", "impl": "reference",
-           "config": {"workload": f"{args.workload}_T{T}", "H": wl["H"], "E": wl["E"],
+           "config": {"workload": wl["name"], "H": wl["H"], "E": wl["E"],
                       "k": wl["k"], "I": wl["I"], "tokens": T},
            "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": s.cores, "kind": "oracle",
                             "sample": f"first {s.n} of {T} tokens per step ({s.experts} experts)"

@@ -138,7 +138,7 @@ struct FfnParams {
 struct PlanSmem {
   int act[kMaxE];       // active expert ids, increasing
   int acnt[kMaxE];      // their token counts
-  int aoff[kMaxE];      // their first compact row
+  int aoff[kMaxE + 1];  // their first compact row; aoff[nA] = all assignments
   int cpre[kMaxE + 1];  // chunk prefix; cpre[nA] = total chunks
   int nA;
 };
@@ -189,7 +189,61 @@ __device__ __forceinline__ void build_plan(const int* counts, int E, int NT, Pla
   if (lane == 0) {
     pl.nA = run_act;
     pl.cpre[run_act] = run_ch;
+    pl.aoff[run_act] = run_off;
   }
+}
+
+// Relative cost of one stage of an item with n tokens: kStageCost + n *
+// kTokenCost.  The weight tile of a stage is the same for every item; each
+// token adds its own activation-row copy and scale loads (one TMA box and one
+// scale row per token when the rows are copied token by token) and its output
+// rows in the epilogue.  Measured on the 235B-shaped NVFP4 layer at 64 tokens:
+// a CTA's finishing time grows by ~1/25 of a one-token stage per extra token
+// when the rows come token by token.
+constexpr int kTokenCost = 1;
+__host__ __device__ constexpr int stage_cost_base(bool per_token_rows) {
+  return per_token_rows ? 24 : 64;
+}
+
+// First stage of CTA c of `grid` when the stages (item-major, decode_item's
+// order) are divided by cost instead of by count: the first stage that begins
+// at or after c / grid of the total cost.  The cost prefix over active experts
+// follows from the chunk and token prefixes: sum of (a * chunks + b * tokens)
+// per row tile and K-stage.  f(0) = 0, f(grid) = every stage, f increasing.
+__device__ __forceinline__ int cost_split_stage(const PlanSmem& pl, int rtiles, int KB, int NT,
+                                                int a, int b, int c, int grid) {
+  const long long per = (long long)rtiles * KB;
+  auto prefix = [&](int s) {
+    return per * ((long long)a * pl.cpre[s] + (long long)b * pl.aoff[s]);
+  };
+  const long long X = prefix(pl.nA) * c / grid;
+  int lo = 0, hi = pl.nA;  // last slot whose cost prefix is <= X
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (prefix(mid) <= X) lo = mid; else hi = mid - 1;
+  }
+  if (lo == pl.nA) return pl.cpre[pl.nA] * rtiles * KB;
+  const long long r = X - prefix(lo);
+  const int n = pl.acnt[lo];
+  const int ch = pl.cpre[lo + 1] - pl.cpre[lo];
+  const long long c_rt = (long long)KB * ((long long)a * ch + (long long)b * n);
+  const int rt = (int)(r / c_rt);
+  const long long r2 = r - rt * c_rt;
+  const int nfull = n / NT;  // chunks of NT tokens
+  const long long wf = a + (long long)b * NT;
+  int chunk;
+  long long r3, w;
+  if (r2 < nfull * KB * wf) {
+    chunk = (int)(r2 / (KB * wf));
+    r3 = r2 - chunk * KB * wf;
+    w = wf;
+  } else {  // the last, partial chunk
+    chunk = nfull;
+    r3 = r2 - nfull * KB * wf;
+    w = a + (long long)b * (n - nfull * NT);
+  }
+  const int kb = (int)((r3 + w - 1) / w);  // <= KB: a stage that starts at or after X
+  return ((pl.cpre[lo] * rtiles) + rt * ch + chunk) * KB + kb;
 }
 
 // Position of a CTA's current stage without divisions: item `it`, K-block

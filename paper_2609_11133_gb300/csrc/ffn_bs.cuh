@@ -159,9 +159,12 @@ __global__ void __launch_bounds__(kBsThreads, 1)
   const int rtiles = (PHASE == 1) ? p.I / kRowsHalf : p.H / (2 * kRowsHalf);
   const int KB = K / KEL;
   // stages of all items (< 2^31 for every supported shape), this CTA's share
-  const long long total = (long long)pl.cpre[pl.nA] * rtiles * KB;
-  const int s_begin = (int)(total * blockIdx.x / gridDim.x);
-  const int s_end = (int)(total * (blockIdx.x + 1) / gridDim.x);
+  // this CTA's share of the stages, divided by cost (items of many tokens
+  // cost more per stage when their rows come token by token)
+  const int cost_a = stage_cost_base((PHASE == 1) && !p.b_compact);
+  const int s_begin = cost_split_stage(pl, rtiles, KB, NT, cost_a, kTokenCost, blockIdx.x, gridDim.x);
+  const int s_end = cost_split_stage(pl, rtiles, KB, NT, cost_a, kTokenCost, blockIdx.x + 1,
+                                     gridDim.x);
   const int nst = s_end - s_begin;
   const uint32_t timeout_bit = (PHASE == 1) ? kStatusTimeoutGateUp : kStatusTimeoutDown;
   // B rows: per token (phase 1, tokens scattered) or one box per chunk

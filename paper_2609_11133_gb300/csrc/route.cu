@@ -302,6 +302,81 @@ __device__ void permute_plan(const int* ids, int T, int k, int E, int* counts, i
   }
 }
 
+// Top-k of token t's logits by one warp, lane l holding logits l, l+32, ...
+// (PER of them, E <= 32 * PER): the ids and gates, and - in the fused layer -
+// the token's entries in the per-expert assignment lists.
+template <int PER>
+__device__ __forceinline__ void chunk_topk(const RouteParams& p, int t, int warp, int lane,
+                                           int (*s_sel)[kMaxK], float (*s_selv)[kMaxK]) {
+  const int E = p.E;
+  float v[PER];
+#pragma unroll
+  for (int i = 0; i < PER; ++i) {
+    const int ee = lane + 32 * i;
+    v[i] = (ee < E) ? __ldcg(p.logits + (size_t)t * E + ee) : -INFINITY;
+  }
+  // Each lane keeps the best of its own untaken logits; a round takes the
+  // warp's best by two warp reductions - the largest order-preserving key,
+  // then the lowest expert index holding it (ties go to the lower index;
+  // -0 and +0 share a key) - and only the winning lane rescans.
+  unsigned key[PER];
+#pragma unroll
+  for (int i = 0; i < PER; ++i) key[i] = logit_key(v[i]);
+  unsigned taken = 0u;
+  unsigned lbk;  // best untaken key of this lane (0: none left)
+  unsigned lbi;
+  auto local_best = [&]() {
+    lbk = 0u;
+    lbi = 0xffffffffu;
+#pragma unroll
+    for (int i = 0; i < PER; ++i) {
+      const int ee = lane + 32 * i;
+      if (ee < E && !((taken >> i) & 1u) && key[i] > lbk) {
+        lbk = key[i];  // a later (higher) index never wins a tie within a lane
+        lbi = (unsigned)ee;
+      }
+    }
+  };
+  local_best();
+  for (int j = 0; j < p.k; ++j) {
+    const unsigned m = __reduce_max_sync(0xffffffffu, lbk);
+    const unsigned bi = __reduce_min_sync(0xffffffffu, lbk == m ? lbi : 0xffffffffu);
+    if ((int)(bi & 31u) == lane) {
+      taken |= 1u << (bi >> 5);
+      local_best();
+    }
+    if (lane == 0) {
+      s_sel[warp][j] = (int)bi;
+      s_selv[warp][j] = key_logit(m);
+    }
+  }
+  __syncwarp();
+  const float lmax = s_selv[warp][0];
+  float den = 0.f;
+  if (p.renorm) {
+    for (int j = 0; j < p.k; ++j) den += expf(s_selv[warp][j] - lmax);
+  } else {
+    float part = 0.f;
+#pragma unroll
+    for (int i = 0; i < PER; ++i)
+      if (lane + 32 * i < E) part += expf(v[i] - lmax);
+    den = warp_sum(part);
+  }
+  for (int j = lane; j < p.k; j += 32) {
+    const int id = s_sel[warp][j];
+    const float gw = expf(s_selv[warp][j] - lmax) / den;
+    p.ids[(size_t)t * p.k + j] = id;
+    p.gates[(size_t)t * p.k + j] = gw;
+    if (p.ids2) p.ids2[(size_t)t * p.k + j] = id;
+    if (p.gates2) p.gates2[(size_t)t * p.k + j] = gw;
+    if (p.fused) {
+      // append to expert id's list (order within a list is arbitrary)
+      const unsigned pos = atomicAdd(p.acnt + id, 1u);
+      p.alist[(size_t)id * p.T + pos] = t * p.k + j;
+    }
+  }
+}
+
 // ------------------------------------------------------------------ route kernel
 __global__ void __launch_bounds__(256) route_kernel(const RouteParams p) {
   extern __shared__ __align__(16) unsigned char route_smem[];
@@ -452,88 +527,31 @@ __global__ void __launch_bounds__(256) route_kernel(const RouteParams p) {
     for (size_t i = tid; i < p.zero_b_n4; i += nthr) p.zero_b[i] = z;
   }
 
-  // chunk ticket: the last of this chunk's expert blocks does the top-k
-  __threadfence();
+  // chunk ticket: the last of this chunk's expert blocks does the top-k.  The
+  // barrier orders every thread's writes before thread 0's fence and ticket
+  // (release); the winner's fence after the ticket and the second barrier
+  // order its reads of the other blocks' logits after it (acquire).
   __syncthreads();
   if (threadIdx.x == 0) {
+    __threadfence();
     const unsigned old = atomicAdd(p.chunk_cnt + chunk, 1u);
     s_flag = (old == gridDim.x - 1);
-    if (s_flag) p.chunk_cnt[chunk] = 0u;
+    if (s_flag) {
+      p.chunk_cnt[chunk] = 0u;
+      __threadfence();
+    }
   }
   __syncthreads();
   if (!s_flag) return;
-  __threadfence();
 
   if (warp < nt) {
-    const int t = t0 + warp;
-    constexpr int PER = kMaxE / 32;
     const int per = (E + 31) / 32;  // logits held by each lane
-    float v[PER];
-#pragma unroll
-    for (int i = 0; i < PER; ++i) {
-      const int ee = lane + 32 * i;
-      v[i] = (i < per && ee < E) ? __ldcg(p.logits + (size_t)t * E + ee) : -INFINITY;
-    }
-    // Each lane keeps the best of its own untaken logits; a round takes the
-    // warp's best by two warp reductions - the largest order-preserving key,
-    // then the lowest expert index holding it (ties go to the lower index;
-    // -0 and +0 share a key) - and only the winning lane rescans.
-    unsigned key[PER];
-#pragma unroll
-    for (int i = 0; i < PER; ++i) key[i] = logit_key(v[i]);
-    unsigned taken = 0u;
-    unsigned lbk;  // best untaken key of this lane (0: none left)
-    unsigned lbi;
-    auto local_best = [&]() {
-      lbk = 0u;
-      lbi = 0xffffffffu;
-#pragma unroll
-      for (int i = 0; i < PER; ++i) {
-        const int ee = lane + 32 * i;
-        if (i < per && ee < E && !((taken >> i) & 1u) && key[i] > lbk) {
-          lbk = key[i];  // a later (higher) index never wins a tie within a lane
-          lbi = (unsigned)ee;
-        }
-      }
-    };
-    local_best();
-    for (int j = 0; j < p.k; ++j) {
-      const unsigned m = __reduce_max_sync(0xffffffffu, lbk);
-      const unsigned bi = __reduce_min_sync(0xffffffffu, lbk == m ? lbi : 0xffffffffu);
-      if ((int)(bi & 31u) == lane) {
-        taken |= 1u << (bi >> 5);
-        local_best();
-      }
-      if (lane == 0) {
-        s_sel[warp][j] = (int)bi;
-        s_selv[warp][j] = key_logit(m);
-      }
-    }
-    __syncwarp();
-    const float lmax = s_selv[warp][0];
-    float den = 0.f;
-    if (p.renorm) {
-      for (int j = 0; j < p.k; ++j) den += expf(s_selv[warp][j] - lmax);
-    } else {
-      float part = 0.f;
-#pragma unroll
-      for (int i = 0; i < PER; ++i)
-        if (lane + 32 * i < E) part += expf(v[i] - lmax);
-      den = warp_sum(part);
-    }
-    for (int j = lane; j < p.k; j += 32) {
-      const int id = s_sel[warp][j];
-      const float gw = expf(s_selv[warp][j] - lmax) / den;
-      p.ids[(size_t)t * p.k + j] = id;
-      p.gates[(size_t)t * p.k + j] = gw;
-      if (p.ids2) p.ids2[(size_t)t * p.k + j] = id;
-      if (p.gates2) p.gates2[(size_t)t * p.k + j] = gw;
-      if (p.fused) {
-        // append to expert id's list (order within a list is arbitrary)
-        const unsigned pos = atomicAdd(p.acnt + id, 1u);
-        p.alist[(size_t)id * p.T + pos] = t * p.k + j;
-      }
-    }
+    if (per <= 4)
+      chunk_topk<4>(p, t0 + warp, warp, lane, s_sel, s_selv);
+    else if (per <= 8)
+      chunk_topk<8>(p, t0 + warp, warp, lane, s_sel, s_selv);
+    else
+      chunk_topk<kMaxE / 32>(p, t0 + warp, warp, lane, s_sel, s_selv);
   }
 }
 
