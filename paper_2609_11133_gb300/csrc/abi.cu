@@ -259,6 +259,7 @@ int run_experts(const ExpertRun& r, cudaStream_t st, cudaEvent_t ev_mid) {
   p.list_T = r.list_T;
   p.gates = r.gates;
   p.status = ws_ptr<uint32_t>(r.ws, r.L.status);
+  p.units = ws_ptr<uint32_t>(r.ws, r.L.units);
   p.wait_ns = wait_limit_ns();
 
   FfnParams p1 = p;

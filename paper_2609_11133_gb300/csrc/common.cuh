@@ -42,6 +42,7 @@ struct WsLayout {
   // control block (zeroed once; every counter is reset by its last user)
   size_t status;       // u32 device status word
   size_t acnt;         // u32 [kMaxE] assignments per expert (fused layer)
+  size_t units;        // u32 [4] shared-tail counters of the two expert phases
   size_t route_chunk;  // u32 [nChunks] per-token-chunk arrival tickets
   // routing
   size_t logits;   // f32 [T, E]
@@ -100,6 +101,7 @@ inline WsLayout ws_layout(int T, int k, int E, int H, int I, int act = kActF16) 
   const size_t TK = (size_t)T * k;
   L.status = take(4);
   L.acnt = take(4 * (size_t)kMaxE);  // fixed size: the same offset for every T and E
+  L.units = take(16);
   L.route_chunk = take(4 * (size_t)(L.nChunks > 0 ? L.nChunks : 1));
   L.logits = take(4 * (size_t)T * E);
   L.ids = take(4 * TK);

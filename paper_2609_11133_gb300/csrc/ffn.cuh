@@ -126,6 +126,9 @@ struct FfnParams {
   uint8_t* hq;         // [T*k*4, I/2] E2M1 codes
   uint8_t* hsf;        // [T*k*4, I/16] UE4M3
   uint32_t* status;
+  // tensor-core engines: {next unit, CTAs done} of this phase's shared tail;
+  // the last CTA to finish puts both back to zero
+  uint32_t* units;
   uint64_t wait_ns;
   int test_stall;      // test hook: producer withholds its first stage
 };
@@ -205,18 +208,18 @@ __host__ __device__ constexpr int stage_cost_base(bool per_token_rows) {
   return per_token_rows ? 24 : 64;
 }
 
-// First stage of CTA c of `grid` when the stages (item-major, decode_item's
-// order) are divided by cost instead of by count: the first stage that begins
-// at or after c / grid of the total cost.  The cost prefix over active experts
-// follows from the chunk and token prefixes: sum of (a * chunks + b * tokens)
-// per row tile and K-stage.  f(0) = 0, f(grid) = every stage, f increasing.
+// The first stage (item-major, decode_item's order) that begins at or after
+// the fraction num / den of the total cost.  The cost prefix over active
+// experts follows from the chunk and token prefixes: sum of (a * chunks + b *
+// tokens) per row tile and K-stage.  f(0) = 0, f(den) = every stage, f
+// increasing in num.
 __device__ __forceinline__ int cost_split_stage(const PlanSmem& pl, int rtiles, int KB, int NT,
-                                                int a, int b, int c, int grid) {
+                                                int a, int b, long long num, long long den) {
   const long long per = (long long)rtiles * KB;
   auto prefix = [&](int s) {
     return per * ((long long)a * pl.cpre[s] + (long long)b * pl.aoff[s]);
   };
-  const long long X = prefix(pl.nA) * c / grid;
+  const long long X = prefix(pl.nA) * num / den;
   int lo = 0, hi = pl.nA;  // last slot whose cost prefix is <= X
   while (lo < hi) {
     const int mid = (lo + hi + 1) >> 1;
@@ -265,7 +268,85 @@ struct StageCursor {
       par ^= 1u;
     }
   }
+  // jump to stage s of the sequence; the ring position runs on
+  __device__ __forceinline__ void seek(int s) {
+    it = s / KB;
+    kb = s - it * KB;
+  }
 };
+
+// ------------------------------------------------------------------ shared tail
+// A CTA of the FP8 tensor-core engine streams its own share of the stages first
+// (divided by cost, kStaticNum / kStaticDen of the total cost), then units of
+// kUnitStages stages of the rest, taken one at a time from a global counter
+// by the lead producer and handed to the CTA's other roles through a ring in
+// shared memory.  A CTA whose copies land faster takes more of the tail.
+constexpr int kUnitStages = 8;
+constexpr int kStaticNum = 4, kStaticDen = 5;
+constexpr int kTailMinStages = 200;  // per CTA
+constexpr int kUnitRing = 32;  // > the units one role can run ahead of another
+
+struct UnitRing {
+  int first[kUnitRing];  // first stage of the unit; -1: no more units
+  uint64_t full[kUnitRing];
+  uint64_t empty[kUnitRing];
+};
+
+// Lead producer: publish unit j (its first stage a, or -1) once every reader
+// of entry j - kUnitRing has taken it.
+__device__ __forceinline__ bool unit_push(UnitRing& r, int j, int a, uint64_t wait_ns,
+                                          volatile int* abort) {
+  const int q = j % kUnitRing;
+  if (!mbar_wait_bounded(&r.empty[q], ((uint32_t)(j / kUnitRing) & 1u) ^ 1u, wait_ns, abort))
+    return false;
+  *reinterpret_cast<volatile int*>(&r.first[q]) = a;
+  mbar_arrive(&r.full[q]);
+  return true;
+}
+
+// Reader: unit j as the stage range [a, b); false at the end of the tail or
+// when the wait expired (*ok = false).  A warp-wide reader calls this on all
+// lanes and lane 0 reports the entry read; a one-thread reader reports it
+// itself (warp_wide false).
+__device__ __forceinline__ bool unit_next(UnitRing& r, int& j, int total, int& a, int& b,
+                                          bool warp_wide, uint64_t wait_ns, volatile int* abort,
+                                          bool* ok) {
+  const int q = j % kUnitRing;
+  if (!mbar_wait_bounded(&r.full[q], (uint32_t)(j / kUnitRing) & 1u, wait_ns, abort)) {
+    *ok = false;
+    return false;
+  }
+  const int first = *reinterpret_cast<volatile int*>(&r.first[q]);
+  if (warp_wide) {
+    __syncwarp();
+    if ((threadIdx.x & 31) == 0) mbar_arrive(&r.empty[q]);
+  } else {
+    mbar_arrive(&r.empty[q]);
+  }
+  ++j;
+  if (first < 0) return false;
+  a = first;
+  b = min(first + kUnitStages, total);
+  return true;
+}
+
+// Lead producer, after its last unit: count this CTA done; the last CTA puts
+// the counters back to zero for the next launch (every CTA has taken its
+// last unit by then).
+__device__ __forceinline__ void unit_done(uint32_t* units) {
+  __threadfence();
+  if (atomicAdd(units + 1, 1u) == gridDim.x - 1) {
+    units[0] = 0u;
+    units[1] = 0u;
+    __threadfence();
+  }
+}
+
+// The unit that follows a CTA's last one: first stage, or -1 past the end.
+__device__ __forceinline__ int unit_take(uint32_t* units, int s_dyn, int total) {
+  const long long a = (long long)s_dyn + (long long)atomicAdd(units, 1u) * kUnitStages;
+  return a < total ? (int)a : -1;
+}
 
 struct ItemInfo {
   int slot, e, arow0, lrow0, nvalid, rt;

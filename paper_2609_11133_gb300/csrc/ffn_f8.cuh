@@ -83,6 +83,7 @@ __global__ void __launch_bounds__(kF8Threads, 1)
   __shared__ int s_tok[NT];
   __shared__ uint32_t s_tmem;
   __shared__ volatile int s_abort;
+  __shared__ __align__(8) UnitRing s_units;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
@@ -97,6 +98,11 @@ __global__ void __launch_bounds__(kF8Threads, 1)
       mbar_init(&dempty_bar[i], 4);
     }
     mbar_init(&final_bar, 1);
+    // readers of each unit: second producer, MMA issuer, 4 epilogue warps
+    for (int i = 0; i < kUnitRing; ++i) {
+      mbar_init(&s_units.full[i], 1);
+      mbar_init(&s_units.empty[i], 6);
+    }
     fence_mbar_init();
   }
   if (warp == kF8MmaWarp) {
@@ -122,14 +128,26 @@ __global__ void __launch_bounds__(kF8Threads, 1)
   const int K = (PHASE == 1) ? p.H : p.I;  // contraction length
   const int rtiles = (PHASE == 1) ? p.I / kRowsHalf : p.H / (2 * kRowsHalf);
   const int KB = K / KEL;
-  // stages of all items (< 2^31 for every supported shape), this CTA's share
-  // this CTA's share of the stages, divided by cost (items of many tokens
-  // cost more per stage when their rows come token by token)
+  // Stages of all items (< 2^31 for every supported shape), divided between
+  // the CTAs by cost (items of many tokens cost more per stage when their rows
+  // come token by token).  With 8-token chunks and enough stages per CTA for
+  // the units to be small, the CTAs divide only the first kStaticNum /
+  // kStaticDen of the cost and the stages from s_dyn on are the shared tail
+  // (measured: it evens out the CTAs' finishing times on the 480B-shaped layer
+  // at 64 tokens; with wider chunks or little work per CTA the static split
+  // alone is faster).
+  const int total = pl.cpre[pl.nA] * rtiles * KB;
+  const bool tail = (NT == 8) && total >= kTailMinStages * (int)gridDim.x;
+  const int snum = tail ? kStaticNum : 1, sden = tail ? kStaticDen : 1;
   const int cost_a = stage_cost_base((PHASE == 1) && !p.b_compact);
-  const int s_begin = cost_split_stage(pl, rtiles, KB, NT, cost_a, kTokenCost, blockIdx.x, gridDim.x);
-  const int s_end = cost_split_stage(pl, rtiles, KB, NT, cost_a, kTokenCost, blockIdx.x + 1,
-                                     gridDim.x);
-  const int nst = s_end - s_begin;
+  const long long den = (long long)gridDim.x * sden;
+  const int s_begin = cost_split_stage(pl, rtiles, KB, NT, cost_a, kTokenCost,
+                                       (long long)blockIdx.x * snum, den);
+  const int s_end = cost_split_stage(pl, rtiles, KB, NT, cost_a, kTokenCost,
+                                     (long long)(blockIdx.x + 1) * snum, den);
+  const int s_dyn = tail ? cost_split_stage(pl, rtiles, KB, NT, cost_a, kTokenCost, snum, sden)
+                         : total;
+  uint32_t* units = p.units + 2 * (PHASE - 1);
   const uint32_t timeout_bit = (PHASE == 1) ? kStatusTimeoutGateUp : kStatusTimeoutDown;
   // B rows: per token (phase 1, tokens scattered) or one box per chunk
   const bool btok = (PHASE == 1) && !p.b_compact;
@@ -139,7 +157,7 @@ __global__ void __launch_bounds__(kF8Threads, 1)
   if (warp == kF8ProducerWarp || warp == kF8ProducerWarp2) {
     const bool lead = (warp == kF8ProducerWarp);
     if (!lead && early) pdl_wait();  // the activation rows are the SwiGLU output
-    if (lane == 0 && nst > 0) {
+    if (lane == 0) {
       tma_prefetch_desc(&tmA0);
       tma_prefetch_desc(&tmA1);
       if (!lead) tma_prefetch_desc(&tmB);
@@ -147,66 +165,94 @@ __global__ void __launch_bounds__(kF8Threads, 1)
       const uint64_t pol_a = policy_evict_last();
       int cur_item = -1;
       ItemInfo inf{};
-      int issued = 0;
-      for (StageCursor<S> c(s_begin, KB); issued < nst; ++issued, c.next()) {
-        const int it = c.it;
-        const int kb = c.kb;
-        if (it != cur_item) {
-          cur_item = it;
-          inf = decode_item(it, rtiles, pl, p, NT);
-          if (!lead && btok)
-            for (int j = 0; j < inf.nvalid; ++j) s_tok[j] = __ldg(p.sorted + inf.lrow0 + j) / p.k;
+      int issued = 0, uj = 0;
+      bool ok = true;
+      StageCursor<S> c(s_begin, KB);
+      // segments: this CTA's own share, then units of the shared tail (the
+      // lead takes them and publishes them; the second producer reads them)
+      for (int a = s_begin, b = s_end; ok;) {
+        for (int s = a; s < b; ++s, ++issued, c.next()) {
+          const int it = c.it;
+          const int kb = c.kb;
+          if (it != cur_item) {
+            cur_item = it;
+            inf = decode_item(it, rtiles, pl, p, NT);
+            if (!lead && btok)
+              for (int j = 0; j < inf.nvalid; ++j) s_tok[j] = __ldg(p.sorted + inf.lrow0 + j) / p.k;
+          }
+          const int slot = c.slot;
+          if (!mbar_wait_bounded(&empty_bar[slot], c.par ^ 1u, p.wait_ns, &s_abort)) {
+            ok = false;
+            break;
+          }
+          if (p.test_stall && issued == 0) continue;  // test hook: this stage never arrives
+          unsigned char* st = smem + (size_t)slot * G::BYTES;
+          int rowA0, rowA1;
+          if (PHASE == 1) {
+            rowA0 = inf.e * N + inf.rt * kRowsHalf;
+            rowA1 = rowA0;
+          } else {
+            rowA0 = inf.e * N + inf.rt * 2 * kRowsHalf;
+            rowA1 = rowA0 + kRowsHalf;
+          }
+          if (lead) {
+            // the second producer's copies may land before this arms the
+            // barrier: the transaction count then dips below zero, and the
+            // phase still cannot complete before this arrival
+            uint32_t bytes = 2u * kRowsHalf * kRowBytes;
+            bytes += btok ? (uint32_t)inf.nvalid * kF8Terms * kRowBytes
+                                    : (uint32_t)BN * kRowBytes;
+            mbar_arrive_expect_tx(&full_bar[slot], bytes);
+            // box A0 always; box A1 too for the down step's first ring of
+            // stages, copied before the SwiGLU kernel ends
+            tma_load_2d(st + G::A0, &tmA0, &full_bar[slot], kb * kRowBytes, rowA0, pol_w);
+            if (early && issued < S)
+              tma_load_2d(st + G::A1, &tmA1, &full_bar[slot], kb * kRowBytes, rowA1, pol_w);
+            continue;
+          }
+          if (!(early && issued < S))
+            tma_load_2d(st + G::A1, &tmA1, &full_bar[slot], kb * kRowBytes, rowA1, pol_w);
+          // activation terms: token j's two rows land at B rows 2j, 2j+1
+          if (btok) {
+            for (int j = 0; j < inf.nvalid; ++j)
+              tma_load_2d(st + G::B + j * kF8Terms * kRowBytes, &tmB, &full_bar[slot],
+                          kb * kRowBytes, s_tok[j] * kF8Terms, pol_a);
+          } else {
+            tma_load_2d(st + G::B, &tmB, &full_bar[slot], kb * kRowBytes, inf.arow0 * kF8Terms,
+                        pol_a);
+          }
         }
-        const int slot = c.slot;
-        if (!mbar_wait_bounded(&empty_bar[slot], c.par ^ 1u, p.wait_ns, &s_abort)) {
-          set_status(p.status, timeout_bit);
-          s_abort = 1;
+        if (!ok || !tail) break;
+        if (lead) {
+          const int next = unit_take(units, s_dyn, total);
+          if (!unit_push(s_units, uj++, next, p.wait_ns, &s_abort)) {
+            ok = false;
+            break;
+          }
+          if (next < 0) break;
+          a = next;
+          b = min(next + kUnitStages, total);
+        } else if (!unit_next(s_units, uj, total, a, b, false, p.wait_ns, &s_abort, &ok)) {
           break;
         }
-        if (p.test_stall && issued == 0) continue;  // test hook: this stage never arrives
-        unsigned char* st = smem + (size_t)slot * G::BYTES;
-        int rowA0, rowA1;
-        if (PHASE == 1) {
-          rowA0 = inf.e * N + inf.rt * kRowsHalf;
-          rowA1 = rowA0;
-        } else {
-          rowA0 = inf.e * N + inf.rt * 2 * kRowsHalf;
-          rowA1 = rowA0 + kRowsHalf;
-        }
-        if (lead) {
-          // the second producer's copies may land before this arms the
-          // barrier: the transaction count then dips below zero, and the
-          // phase still cannot complete before this arrival
-          uint32_t bytes = 2u * kRowsHalf * kRowBytes;
-          bytes += btok ? (uint32_t)inf.nvalid * kF8Terms * kRowBytes
-                                  : (uint32_t)BN * kRowBytes;
-          mbar_arrive_expect_tx(&full_bar[slot], bytes);
-          // box A0 always; box A1 too for the down step's first ring of
-          // stages, copied before the SwiGLU kernel ends
-          tma_load_2d(st + G::A0, &tmA0, &full_bar[slot], kb * kRowBytes, rowA0, pol_w);
-          if (early && issued < S)
-            tma_load_2d(st + G::A1, &tmA1, &full_bar[slot], kb * kRowBytes, rowA1, pol_w);
-          continue;
-        }
-        if (!(early && issued < S))
-          tma_load_2d(st + G::A1, &tmA1, &full_bar[slot], kb * kRowBytes, rowA1, pol_w);
-        // activation terms: token j's two rows land at B rows 2j, 2j+1
-        if (btok) {
-          for (int j = 0; j < inf.nvalid; ++j)
-            tma_load_2d(st + G::B + j * kF8Terms * kRowBytes, &tmB, &full_bar[slot],
-                        kb * kRowBytes, s_tok[j] * kF8Terms, pol_a);
-        } else {
-          tma_load_2d(st + G::B, &tmB, &full_bar[slot], kb * kRowBytes, inf.arow0 * kF8Terms,
-                      pol_a);
-        }
+        c.seek(a);
       }
-      // Let every copy land before the CTA exits (the barriers complete only
-      // when both producers' copies have landed).
-      if (!lead) return;
-      const int first = issued > S ? issued - S : 0;
-      for (int j = first; j < issued; ++j) {
-        if (p.test_stall && j == 0) continue;
-        mbar_wait_bounded(&full_bar[j % S], (uint32_t)((j / S) & 1), p.wait_ns, nullptr);
+      if (!ok) {
+        set_status(p.status, timeout_bit);
+        s_abort = 1;
+      }
+      if (lead) {
+        if (tail) {
+          if (!ok) unit_push(s_units, uj, -1, p.wait_ns, &s_abort);  // best effort
+          unit_done(units);
+        }
+        // Let every copy land before the CTA exits (the barriers complete
+        // only when both producers' copies have landed).
+        const int first = issued > S ? issued - S : 0;
+        for (int j = first; j < issued; ++j) {
+          if (p.test_stall && j == 0) continue;
+          mbar_wait_bounded(&full_bar[j % S], (uint32_t)((j / S) & 1), p.wait_ns, nullptr);
+        }
       }
     }
     return;
@@ -217,26 +263,33 @@ __global__ void __launch_bounds__(kF8Threads, 1)
     if (lane == 0) {
       constexpr uint32_t idesc = tc_idesc_e4m3(128, BN);
       bool ok = true;
+      int uj = 0;
       StageCursor<S> c(s_begin, KB);
       StageCursor<DR> d(0, 1);  // accumulator ring position
-      for (int i = 0; i < nst && ok; ++i, c.next(), d.next()) {
-        const int slot = c.slot;
-        const int db = d.slot;
-        ok = mbar_wait_bounded(&dempty_bar[db], d.par ^ 1u, p.wait_ns, &s_abort) &&
-             mbar_wait_bounded(&full_bar[slot], c.par, p.wait_ns, &s_abort);
-        if (!ok) break;
-        tc_fence_after();
-        const uint32_t st = smem_u32(smem + (size_t)slot * G::BYTES);
+      // every stage has its own accumulator: only the number of stages of
+      // each segment matters here
+      for (int a = s_begin, b = s_end; ok;) {
+        for (int i = a; i < b && ok; ++i, c.next(), d.next()) {
+          const int slot = c.slot;
+          const int db = d.slot;
+          ok = mbar_wait_bounded(&dempty_bar[db], d.par ^ 1u, p.wait_ns, &s_abort) &&
+               mbar_wait_bounded(&full_bar[slot], c.par, p.wait_ns, &s_abort);
+          if (!ok) break;
+          tc_fence_after();
+          const uint32_t st = smem_u32(smem + (size_t)slot * G::BYTES);
 #pragma unroll
-        for (int kk = 0; kk < 4; ++kk) {  // K = 32 per MMA
-          const uint64_t bdesc = tc_desc_sw128(st + G::B + 32 * kk);
-          tc_mma_f8(tmem + (uint32_t)(2 * db) * BN, tc_desc_sw128(st + G::A0 + 32 * kk), bdesc,
-                    idesc, kk > 0 ? 1u : 0u);
-          tc_mma_f8(tmem + (uint32_t)(2 * db + 1) * BN, tc_desc_sw128(st + G::A1 + 32 * kk),
-                    bdesc, idesc, kk > 0 ? 1u : 0u);
+          for (int kk = 0; kk < 4; ++kk) {  // K = 32 per MMA
+            const uint64_t bdesc = tc_desc_sw128(st + G::B + 32 * kk);
+            tc_mma_f8(tmem + (uint32_t)(2 * db) * BN, tc_desc_sw128(st + G::A0 + 32 * kk), bdesc,
+                      idesc, kk > 0 ? 1u : 0u);
+            tc_mma_f8(tmem + (uint32_t)(2 * db + 1) * BN, tc_desc_sw128(st + G::A1 + 32 * kk),
+                      bdesc, idesc, kk > 0 ? 1u : 0u);
+          }
+          tc_commit(&empty_bar[slot]);
+          tc_commit(&dfull_bar[db]);
         }
-        tc_commit(&empty_bar[slot]);
-        tc_commit(&dfull_bar[db]);
+        if (!ok || !tail || !unit_next(s_units, uj, total, a, b, false, p.wait_ns, &s_abort, &ok))
+          break;
       }
       if (!ok) {
         set_status(p.status, timeout_bit);
@@ -279,19 +332,39 @@ __global__ void __launch_bounds__(kF8Threads, 1)
       }
     };
     float bs0 = 0.f, bs1 = 0.f;
-    StageCursor<DR> c(s_begin, KB);  // it, kb of this stage; slot = accumulator ring slot
-    if (nst > 0) {
+    // c: this stage (it, kb) and its accumulator ring slot; the stage after
+    // it is found first (its block scales load while this stage's
+    // accumulator is awaited), reading the shared-tail units as they come
+    StageCursor<DR> c(s_begin, KB);
+    int cs = s_begin, cend = s_end, uj = 0;
+    bool ok = true;
+    bool have = cs < cend;
+    if (!have && tail && unit_next(s_units, uj, total, cs, cend, true, p.wait_ns, &s_abort, &ok)) {
+      c.seek(cs);
+      have = true;
+    }
+    if (have) {
       inf = decode_item(c.it, rtiles, pl, p, NT);
       scales(inf, c.kb, bs0, bs1);
     }
-    for (int i = 0; i < nst && !dead; ++i) {
-      // the next stage's scales, loaded while this stage's accumulator is awaited
+    while (have && !dead) {
+      // the next stage: the following one in this segment, or the first of
+      // the next unit (a new accumulation even within the same item)
+      int ns = cs + 1, nend = cend;
+      StageCursor<DR> nc = c;  // its accumulator slot is the next one in any case
+      nc.next();
+      bool have_next = ns < nend, jump = false;
+      if (!have_next && tail) {
+        have_next = unit_next(s_units, uj, total, ns, nend, true, p.wait_ns, &s_abort, &ok);
+        jump = true;
+        if (have_next) nc.seek(ns);
+      }
       float nb0 = 0.f, nb1 = 0.f;
       ItemInfo ninf = inf;
-      const bool closes = (i + 1 == nst) || (c.kb + 1 == KB);
-      if (i + 1 < nst) {
-        if (c.kb + 1 == KB) ninf = decode_item(c.it + 1, rtiles, pl, p, NT);
-        scales(ninf, c.kb + 1 == KB ? 0 : c.kb + 1, nb0, nb1);
+      const bool closes = !have_next || jump || (c.kb + 1 == KB);
+      if (have_next) {
+        if (nc.it != c.it) ninf = decode_item(nc.it, rtiles, pl, p, NT);
+        scales(ninf, nc.kb, nb0, nb1);
       }
       const int db = c.slot;
       if (!mbar_wait_bounded(&dfull_bar[db], c.par, p.wait_ns, &s_abort)) {
@@ -356,7 +429,14 @@ __global__ void __launch_bounds__(kF8Threads, 1)
       inf = ninf;
       bs0 = nb0;
       bs1 = nb1;
-      c.next();
+      c = nc;
+      cs = ns;
+      cend = nend;
+      have = have_next;
+    }
+    if (!ok) {
+      set_status(p.status, timeout_bit);
+      s_abort = 1;
     }
     tc_fence_before();
     asm volatile("bar.sync 2, %0;" ::"n"(kTeardown) : "memory");
