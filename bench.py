@@ -414,10 +414,14 @@ def run_ours(args):
                 body(s_ % n_rot)
         return g
 
-    def timed(g_full, g_rem, steps):
-        """Replays that run exactly `steps` steps."""
+    def timed(g_full, g_rem, steps, marks=None):
+        """Replays that run exactly `steps` steps; `marks` gets an event after
+        every full replay (the spread over repetitions)."""
         for _ in range(steps // G):
             g_full.replay()
+            if marks is not None:
+                marks.append(torch.cuda.Event(enable_timing=True))
+                marks[-1].record(stream)
         if g_rem is not None:
             g_rem.replay()
 
@@ -449,13 +453,40 @@ def run_ours(args):
     barrier(world)
     h_beg = time.perf_counter()
     t_beg.record(stream)
-    timed(g_step, g_rem, args.steps)
+    marks = []
+    timed(g_step, g_rem, args.steps, marks)
     t_end.record(stream)
     torch.cuda.synchronize()
     h_end = time.perf_counter()
     ms_total = t_beg.elapsed_time(t_end)
     ms_step = barrier_max(ms_total / args.steps, world)
     tok_s = job_throughput(ms_step, T, world)
+    # per-step time of each repetition (one graph replay of G steps)
+    reps = [a.elapsed_time(b) / G for a, b in zip([t_beg] + marks[:-1], marks)]
+    repeats = None
+    if reps:
+        repeats = {"n": len(reps), "steps_each": G, "median_ms": float(np.median(reps)),
+                   "p10_ms": float(np.percentile(reps, 10)),
+                   "p90_ms": float(np.percentile(reps, 90))}
+
+    # single-call latency: one step, eager (host launches included) and as a
+    # one-step graph, each timed alone on an idle GPU
+    lat_eager, lat_graph = [], []
+    g_one = capture(1, lambda r: run_layers(xs[r]))
+    for i_ in range(12):
+        a_, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        a_.record(stream)
+        if i_ % 2:
+            g_one.replay()
+        else:
+            run_layers(xs[0])
+        b_.record(stream)
+        torch.cuda.synchronize()
+        (lat_graph if i_ % 2 else lat_eager).append(a_.elapsed_time(b_) * 1e3)
+    latency = {"eager_us": statistics.median(lat_eager[1:]),
+               "graph_us": statistics.median(lat_graph[1:]),
+               "per": "layer call" if L == 1 else f"{L}-layer step"}
 
     # ---- energy per token (NVML counter over >= 2 s of back-to-back steps)
     energy = None
@@ -582,6 +613,8 @@ def run_ours(args):
                 "h2d_bytes_per_step": T * H * 2, "d2h_bytes_per_step": T * H * 2},
         "gpu_launches": 5 * L * args.steps,
         "timing": f"CUDA-graph replay, {G} steps (layer calls) per graph",
+        "repeats": repeats,
+        "latency": latency,
         "clocks": clk,
         "energy": energy,
     }
