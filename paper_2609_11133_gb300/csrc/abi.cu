@@ -142,8 +142,15 @@ int nt_for(int T, int eng) {
 // Experts per router CTA: small batches spread the router rows over more
 // CTAs (one expert per CTA, its row split over 8 warps); larger ones keep
 // four experts per CTA so that the token rows staged in shared memory are
-// reused.
-int route_epb(int T) { return T <= 16 ? 1 : 4; }
+// reused, and eight (two rounds of four) once the grid would not fit two CTAs
+// per SM: fewer waves of each CTA's fixed work (staging, activation terms,
+// ticket).  Measured: 235B-shaped layer at 128 tokens 25 -> 19 us; more
+// experts per CTA (16, 32) made the 480B-shaped router at 256 tokens slower.
+int route_epb(int T, int E, int sms) {
+  if (T <= 16) return 1;
+  const int chunks = (T + kRouteTok - 1) / kRouteTok;
+  return (long long)((E + 3) / 4) * chunks > 2LL * sms ? 8 : 4;
+}
 
 // ------------------------------------------------------------------ validation
 int check_weights(const moe_expert_weights_t* w) {
@@ -413,7 +420,7 @@ int moe_route_topk(const void* x, const float* router_w, const float* router_bia
   p.ids = topk_ids;
   p.gates = topk_w;
   p.chunk_cnt = ws_ptr<unsigned>(ws, L.route_chunk);
-  p.epb = route_epb(T);
+  p.epb = route_epb(T, E, sms);
   return launch_route(p, (cudaStream_t)stream) == cudaSuccess ? MOE_OK : MOE_ERR_CUDA;
 }
 
@@ -543,7 +550,7 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
   p.prenorm = (flags & MOE_FLAG_PRENORM_RMS) ? 1 : 0;
   p.fmt = w->fmt;
   p.fused = 1;
-  p.epb = route_epb(T);
+  p.epb = route_epb(T, E, sms);
   p.act = act_for(w->fmt, eng);
   p.logits = logits_out ? logits_out : ws_ptr<float>(ws, L.logits);
   p.ids = ws_ptr<int>(ws, L.ids);

@@ -440,82 +440,90 @@ __global__ void __launch_bounds__(256) route_kernel(const RouteParams p) {
     }
   }
 
-  // router GEMV: warp w covers one eighth of H for all epb experts of this
-  // CTA (each staged x value is read once per warp), lanes -> 4 consecutive
-  // h per 128.  The 4 x 8 partial sums of a lane meet across the warp in a
-  // butterfly (lane l ends with sum l = expert slot l/8, token l%8), then
-  // across the warps in shared memory in warp order.
+  // router GEMV, in rounds of up to four of the CTA's experts: warp w covers
+  // one eighth of H for the round's experts (each staged x value is read once
+  // per warp and round), lanes -> 4 consecutive h per 128.  The 4 x 8 partial
+  // sums of a lane meet across the warp in a butterfly (lane l ends with sum
+  // l = expert slot l/8, token l%8), then across the warps in shared memory
+  // in warp order.
   __shared__ float s_part[kRouteWarps][32];
-  {
+  const int nexp = min(p.epb, E - eb * p.epb);  // experts of this CTA
+  for (int q0 = 0; q0 < nexp; q0 += 4) {
     constexpr int MAXEPB = 4;
-    const int nexp = min(p.epb, E - eb * p.epb);  // experts of this CTA
-    const int hpart = H / kRouteWarps;
-    const int hbeg = warp * hpart;
-    float acc[MAXEPB][kRouteTok];
+    const int e0 = eb * p.epb + q0;
+    const int nq = min(MAXEPB, nexp - q0);  // experts of this round
+    {
+      const int hpart = H / kRouteWarps;
+      const int hbeg = warp * hpart;
+      float acc[MAXEPB][kRouteTok];
 #pragma unroll
-    for (int x = 0; x < MAXEPB; ++x)
+      for (int x = 0; x < MAXEPB; ++x)
 #pragma unroll
-      for (int t = 0; t < kRouteTok; ++t) acc[x][t] = 0.f;
-    constexpr int DEPTH = 4;  // 128-element steps whose router loads are in flight together
-    for (int h0 = hbeg + lane * 4; h0 < hbeg + hpart; h0 += 128 * DEPTH) {
-      float4 w[DEPTH][MAXEPB];
+        for (int t = 0; t < kRouteTok; ++t) acc[x][t] = 0.f;
+      constexpr int DEPTH = 4;  // 128-element steps whose router loads are in flight together
+      for (int h0 = hbeg + lane * 4; h0 < hbeg + hpart; h0 += 128 * DEPTH) {
+        float4 w[DEPTH][MAXEPB];
 #pragma unroll
-      for (int q = 0; q < DEPTH; ++q)
+        for (int q = 0; q < DEPTH; ++q)
 #pragma unroll
-        for (int x = 0; x < MAXEPB; ++x)
-          w[q][x] = (x < nexp && h0 + 128 * q < hbeg + hpart)
-                        ? __ldg(reinterpret_cast<const float4*>(
-                              p.wr + (size_t)(eb * p.epb + x) * H + h0 + 128 * q))
-                        : make_float4(0.f, 0.f, 0.f, 0.f);
+          for (int x = 0; x < MAXEPB; ++x)
+            w[q][x] = (x < nq && h0 + 128 * q < hbeg + hpart)
+                          ? __ldg(reinterpret_cast<const float4*>(p.wr + (size_t)(e0 + x) * H +
+                                                                  h0 + 128 * q))
+                          : make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-      for (int q = 0; q < DEPTH; ++q) {
-        const int h = h0 + 128 * q;
-        if (h >= hbeg + hpart) break;
+        for (int q = 0; q < DEPTH; ++q) {
+          const int h = h0 + 128 * q;
+          if (h >= hbeg + hpart) break;
 #pragma unroll
-        for (int t = 0; t < kRouteTok; ++t) {
-          if (t < nt) {
-            const uint2 xv = *reinterpret_cast<const uint2*>(xs + (size_t)t * H + h);
-            const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&xv.x));
-            const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&xv.y));
+          for (int t = 0; t < kRouteTok; ++t) {
+            if (t < nt) {
+              const uint2 xv = *reinterpret_cast<const uint2*>(xs + (size_t)t * H + h);
+              const float2 a =
+                  __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&xv.x));
+              const float2 b =
+                  __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&xv.y));
 #pragma unroll
-            for (int x = 0; x < MAXEPB; ++x) {
-              float sacc = acc[x][t];
-              sacc = fmaf(a.x, w[q][x].x, sacc);
-              sacc = fmaf(a.y, w[q][x].y, sacc);
-              sacc = fmaf(b.x, w[q][x].z, sacc);
-              sacc = fmaf(b.y, w[q][x].w, sacc);
-              acc[x][t] = sacc;
+              for (int x = 0; x < MAXEPB; ++x) {
+                float sacc = acc[x][t];
+                sacc = fmaf(a.x, w[q][x].x, sacc);
+                sacc = fmaf(a.y, w[q][x].y, sacc);
+                sacc = fmaf(b.x, w[q][x].z, sacc);
+                sacc = fmaf(b.y, w[q][x].w, sacc);
+                acc[x][t] = sacc;
+              }
             }
           }
         }
       }
+      float v[32];
+#pragma unroll
+      for (int i = 0; i < 32; ++i) v[i] = acc[i / kRouteTok][i % kRouteTok];
+#pragma unroll
+      for (int sft = 16; sft >= 1; sft >>= 1) {
+        const bool upper = (lane & sft) != 0;
+#pragma unroll
+        for (int i = 0; i < sft; ++i) {
+          const float send = upper ? v[i] : v[i + sft];
+          const float keep = upper ? v[i + sft] : v[i];
+          v[i] = keep + __shfl_xor_sync(0xffffffffu, send, sft);
+        }
+      }
+      s_part[warp][lane] = v[0];
     }
-    float v[32];
+    __syncthreads();
+    if (threadIdx.x < 32) {
+      const int x = threadIdx.x / kRouteTok, t = threadIdx.x % kRouteTok;
+      const int e = e0 + x;
+      if (x < nq && t < nt) {
+        float sum = s_part[0][threadIdx.x];
 #pragma unroll
-    for (int i = 0; i < 32; ++i) v[i] = acc[i / kRouteTok][i % kRouteTok];
-#pragma unroll
-    for (int sft = 16; sft >= 1; sft >>= 1) {
-      const bool upper = (lane & sft) != 0;
-#pragma unroll
-      for (int i = 0; i < sft; ++i) {
-        const float send = upper ? v[i] : v[i + sft];
-        const float keep = upper ? v[i + sft] : v[i];
-        v[i] = keep + __shfl_xor_sync(0xffffffffu, send, sft);
+        for (int w = 1; w < kRouteWarps; ++w) sum += s_part[w][threadIdx.x];
+        const float b = p.bias ? __ldg(p.bias + e) : 0.f;
+        p.logits[(size_t)(t0 + t) * E + e] = sum + b;
       }
     }
-    s_part[warp][lane] = v[0];
-  }
-  __syncthreads();
-  if (threadIdx.x < 32) {
-    const int x = threadIdx.x / kRouteTok, t = threadIdx.x % kRouteTok;
-    const int e = eb * p.epb + x;
-    if (x < p.epb && e < E && t < nt) {
-      float sum = s_part[0][threadIdx.x];
-#pragma unroll
-      for (int w = 1; w < kRouteWarps; ++w) sum += s_part[w][threadIdx.x];
-      const float b = p.bias ? __ldg(p.bias + e) : 0.f;
-      p.logits[(size_t)(t0 + t) * E + e] = sum + b;
-    }
+    __syncthreads();  // s_part is reused by the next round
   }
 
   // accumulators and counters of the later kernels start from zero
