@@ -277,15 +277,40 @@ class OracleSample:
         return time.perf_counter() - t0
 
 
+def _omp_threads(n=None):
+    """The OpenMP thread count of this process (the oracle's), set if n is given."""
+    try:
+        gomp = ctypes.CDLL("libgomp.so.1")
+    except OSError:
+        return None
+    if n is not None:
+        gomp.omp_set_num_threads(int(n))
+    return gomp.omp_get_max_threads()
+
+
 def cpu_oracle_sample(wl, seed, w=None, budget_s=10.0):
     s = OracleSample(wl, seed, budget_s=budget_s, w=w)
     dt = s.run()
     L = wl["layers"]
     per_layer = f", x{L} layers (layer 0 timed)" if L > 1 else ""
-    return {"value": s.n / (dt * L), "unit": "tokens/s", "cores": s.cores, "kind": "oracle",
-            "sample": f"first {s.n} of {wl['T']} tokens ({s.experts} experts): "
-                      f"{'RMS pre-norm, ' if wl['prenorm'] else ''}router, top-k, experts and "
-                      f"combine in float64, {dt:.2f} s{per_layer}"}
+    res = {"value": s.n / (dt * L), "unit": "tokens/s", "cores": s.cores, "kind": "oracle",
+           "sample": f"first {s.n} of {wl['T']} tokens ({s.experts} experts): "
+                     f"{'RMS pre-norm, ' if wl['prenorm'] else ''}router, top-k, experts and "
+                     f"combine in float64, {dt:.2f} s{per_layer}"}
+    # the same oracle on one core, on the first token of the sample
+    prev = _omp_threads()
+    if prev:
+        n_all = s.n
+        try:
+            _omp_threads(1)
+            s.n = 1
+            dt1 = s.run()
+        finally:
+            s.n = n_all
+            _omp_threads(prev)
+        res["one_core"] = {"value": 1.0 / (dt1 * L), "unit": "tokens/s",
+                           "sample": f"first token, {dt1:.2f} s{per_layer}"}
+    return res
 
 
 def expert_bytes(w):
