@@ -101,6 +101,64 @@ __device__ __forceinline__ void encode_terms16(float (&r)[16], uint2 (&codes)[kT
   }
 }
 
+// encode_terms16 spread over the four lanes of a quad (lanes 4j..4j+3 of a
+// warp): lane q of the quad holds elements 4q..4q+3 of the block (already
+// scaled by the row's power of two) in r.  Every step is the serial one's,
+// element by element, so the codes are the same; the block maximum takes two
+// shuffles.  All 32 lanes of the warp call it together (lanes whose quad has
+// no block pass zeros).  part[t] gets this lane's 16 bits of term t's codes
+// (elements 4q..4q+3, element 4q in the low nibble), sf[t] the term's scale.
+__device__ __forceinline__ void encode_terms16_quad(float (&r)[4], uint32_t (&part)[kTerms],
+                                                    uint32_t (&sf)[kTerms]) {
+#pragma unroll
+  for (int t = 0; t < kTerms; ++t) {
+    float m = fmaxf(fmaxf(fabsf(r[0]), fabsf(r[1])), fmaxf(fabsf(r[2]), fabsf(r[3])));
+    m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 1));
+    m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 2));
+    float s = 0.f;
+    const uint32_t c = ue4m3_ceil(m * (1.f / 6.f), &s);
+    sf[t] = (m > 0.f) ? c : 0u;
+    part[t] = 0u;
+    if (m > 0.f) {
+      const float inv = 1.f / s;
+      uint32_t w;
+      asm("{\n .reg .b8 b0, b1;\n"
+          " cvt.rn.satfinite.e2m1x2.f32 b0, %2, %1;\n"
+          " cvt.rn.satfinite.e2m1x2.f32 b1, %4, %3;\n"
+          " mov.b32 %0, {b0, b1, b0, b1};\n}\n"
+          : "=r"(w)
+          : "f"(r[0] * inv), "f"(r[1] * inv), "f"(r[2] * inv), "f"(r[3] * inv));
+      part[t] = w & 0xffffu;
+      uint32_t d[4];
+      e2m1x8_to_f16x8(part[t], d);  // d[0], d[1]: elements 0-1, 2-3
+#pragma unroll
+      for (int i = 0; i < 2; ++i) {
+        const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&d[i]));
+        r[2 * i] = fmaf(-f.x, s, r[2 * i]);  // exact
+        r[2 * i + 1] = fmaf(-f.y, s, r[2 * i + 1]);
+      }
+    }
+  }
+}
+
+// Store the quad's block b: lanes q = 0 and 2 write the two 32-bit halves of
+// each term's codes, lane 0 the scale bytes.  All lanes of the warp call it;
+// `valid` is false on lanes whose quad has no block.
+__device__ __forceinline__ void store_terms16_quad(const uint32_t (&part)[kTerms],
+                                                   const uint32_t (&sf)[kTerms], bool valid,
+                                                   uint8_t* q, uint8_t* sfp, size_t row4, int K,
+                                                   int b) {
+  const int lq = threadIdx.x & 3;
+#pragma unroll
+  for (int t = 0; t < kTerms; ++t) {
+    uint32_t w = part[t] << (16 * (lq & 1));
+    w |= __shfl_xor_sync(0xffffffffu, w, 1);  // lanes 0,1: elements 0-7; 2,3: 8-15
+    if (valid && (lq & 1) == 0)
+      *reinterpret_cast<uint32_t*>(q + (row4 + t) * (size_t)(K / 2) + 8 * b + 2 * lq) = w;
+    if (valid && lq == 0) sfp[(row4 + t) * (size_t)(K / 16) + b] = (uint8_t)sf[t];
+  }
+}
+
 // Write block b of a row's terms: row r of the term arrays is token/assignment
 // `row4 / kTerms`, term `row4 % kTerms`; q rows are K/2 bytes, sf rows K/16.
 __device__ __forceinline__ void store_terms16(const uint2 (&codes)[kTerms],

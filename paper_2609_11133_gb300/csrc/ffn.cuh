@@ -389,8 +389,10 @@ template <int FMT>
 __global__ void __launch_bounds__(256) swiglu_kernel(const FfnParams p, int rows, int perm) {
   constexpr int G = 8;  // float4 groups per thread
   __shared__ float s_max[8];
-  pdl_wait();
+  // the down step may launch now: what it does before its own wait (plan,
+  // weight copies) does not read this kernel's output
   pdl_launch_dependents();
+  pdl_wait();
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int n4 = p.I / 4;
   for (int row = blockIdx.x; row < rows; row += gridDim.x) {

@@ -46,6 +46,7 @@ constexpr int kBsSfWarp0 = 0, kBsEpiWarp0 = 4, kBsProducerWarp = 8, kBsMmaWarp =
 constexpr int kBsProducerWarp2 = 10;
 constexpr uint32_t kBsTmemCols = 512;
 constexpr int kBsSfCols = 48;  // per stage: A scales 2 x 16 columns, B scales 16
+constexpr int kSwigluThreads = 384;  // swiglu_terms_kernel: 96 quads of lanes
 
 template <int NT>
 struct BsGeom {
@@ -479,52 +480,64 @@ __global__ void __launch_bounds__(kBsThreads, 1)
 
 // SwiGLU of every assignment row into four NVFP4 terms (the B operand of the
 // down step): h = silu(g) * u from the fp32 gate|up accumulators, a per-row
-// power of two, then encode_terms16 per 16-column block.  One CTA per row,
-// one thread per block (I <= 8192: at most 4 blocks per thread).
-__global__ void __launch_bounds__(128) swiglu_terms_kernel(const FfnParams p, int rows) {
-  constexpr int G = 4;  // blocks per thread
-  __shared__ float s_max[4];
-  pdl_wait();
+// power of two, then the terms of each 16-column block by a quad of lanes
+// (four columns each).  One CTA per row, one pass over the row when I <= 1536
+// (96 blocks); every load of the row is issued before the first is used.
+__global__ void __launch_bounds__(kSwigluThreads, 2) swiglu_terms_kernel(const FfnParams p, int rows) {
+  constexpr int BPP = kSwigluThreads / 4;          // blocks per pass
+  constexpr int PMAX = (8192 / 16 + BPP - 1) / BPP;  // passes for I <= 8192
+  __shared__ float s_max[kSwigluThreads / 32];
+  // the down step may launch now: what it does before its own wait (plan,
+  // weight copies) does not read this kernel's output
   pdl_launch_dependents();
+  pdl_wait();
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int lq = threadIdx.x & 3, quad = threadIdx.x >> 2;
   const int nb = p.I / 16;
+  const int np = (nb + BPP - 1) / BPP;
   for (int row = blockIdx.x; row < rows; row += gridDim.x) {
     const float* g = p.gu + (size_t)row * 2 * p.I;
     const float* u = g + p.I;
-    float h[G][16];
+    float h[PMAX][4];
     float amax = 0.f;
+    float4 gv[PMAX], uv[PMAX];
 #pragma unroll
-    for (int q = 0; q < G; ++q) {
-      const int b = threadIdx.x + 128 * q;
-      if (b < nb) {
+    for (int ps = 0; ps < PMAX; ++ps) {
+      const int b = quad + BPP * ps;
+      gv[ps] = uv[ps] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (ps < np && b < nb) {
+        gv[ps] = __ldcg(reinterpret_cast<const float4*>(g + 16 * b + 4 * lq));
+        uv[ps] = __ldcg(reinterpret_cast<const float4*>(u + 16 * b + 4 * lq));
+      }
+    }
 #pragma unroll
-        for (int i = 0; i < 16; i += 4) {
-          const float4 gv = __ldcg(reinterpret_cast<const float4*>(g + 16 * b + i));
-          const float4 uv = __ldcg(reinterpret_cast<const float4*>(u + 16 * b + i));
-          h[q][i + 0] = gv.x / (1.f + expf(-gv.x)) * uv.x;
-          h[q][i + 1] = gv.y / (1.f + expf(-gv.y)) * uv.y;
-          h[q][i + 2] = gv.z / (1.f + expf(-gv.z)) * uv.z;
-          h[q][i + 3] = gv.w / (1.f + expf(-gv.w)) * uv.w;
-        }
+    for (int ps = 0; ps < PMAX; ++ps) {
+      if (ps < np) {  // the same on every thread
+        h[ps][0] = gv[ps].x / (1.f + expf(-gv[ps].x)) * uv[ps].x;
+        h[ps][1] = gv[ps].y / (1.f + expf(-gv[ps].y)) * uv[ps].y;
+        h[ps][2] = gv[ps].z / (1.f + expf(-gv[ps].z)) * uv[ps].z;
+        h[ps][3] = gv[ps].w / (1.f + expf(-gv[ps].w)) * uv[ps].w;
 #pragma unroll
-        for (int i = 0; i < 16; ++i) amax = fmaxf(amax, fabsf(h[q][i]));
+        for (int i = 0; i < 4; ++i) amax = fmaxf(amax, fabsf(h[ps][i]));
       }
     }
     amax = warp_max(amax);
     if (lane == 0) s_max[warp] = amax;
     __syncthreads();
-    amax = fmaxf(fmaxf(s_max[0], s_max[1]), fmaxf(s_max[2], s_max[3]));
+    amax = s_max[0];
+#pragma unroll
+    for (int i = 1; i < kSwigluThreads / 32; ++i) amax = fmaxf(amax, s_max[i]);
     const float sc = pow2_scale_terms(amax);
 #pragma unroll
-    for (int q = 0; q < G; ++q) {
-      const int b = threadIdx.x + 128 * q;
-      if (b < nb) {
+    for (int ps = 0; ps < PMAX; ++ps) {
+      if (ps < np) {  // the same on every thread
+        const int b = quad + BPP * ps;
+        float r[4];
 #pragma unroll
-        for (int i = 0; i < 16; ++i) h[q][i] *= sc;
-        uint2 codes[kTerms];
-        uint32_t sf[kTerms];
-        encode_terms16(h[q], codes, sf);
-        store_terms16(codes, sf, p.hq, p.hsf, (size_t)row * kTerms, p.I, b);
+        for (int i = 0; i < 4; ++i) r[i] = h[ps][i] * sc;
+        uint32_t part[kTerms], sf[kTerms];
+        encode_terms16_quad(r, part, sf);
+        store_terms16_quad(part, sf, b < nb, p.hq, p.hsf, (size_t)row * kTerms, p.I, b);
       }
     }
     if (threadIdx.x == 0) p.hinv[row] = 1.f / sc;

@@ -450,8 +450,10 @@ __global__ void __launch_bounds__(kF8Threads, 1)
 __global__ void __launch_bounds__(128) swiglu_e4m3_kernel(const FfnParams p, int rows) {
   constexpr int G = 8;
   __shared__ float s_max[4];
-  pdl_wait();
+  // the down step may launch now: what it does before its own wait (plan,
+  // weight copies) does not read this kernel's output
   pdl_launch_dependents();
+  pdl_wait();
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int n8 = p.I / 8;
   for (int row = blockIdx.x; row < rows; row += gridDim.x) {

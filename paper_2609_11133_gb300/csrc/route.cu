@@ -80,15 +80,27 @@ __device__ void convert_chunk_terms(const __nv_bfloat16* xs, int nt, int H, int 
     }
   }
   __syncthreads();
-  const int nb = H / 16;
-  for (int idx = part * blockDim.x + threadIdx.x; idx < nt * nb; idx += nparts * blockDim.x) {
-    const int j = idx / nb, b = idx - j * nb;
-    float r[16];
-    load_bf16x16_scaled(xs + (size_t)j * H + 16 * b, s_sc[j], r);
-    uint2 codes[kTerms];
-    uint32_t sf[kTerms];
-    encode_terms16(r, codes, sf);
-    store_terms16(codes, sf, xq, xsf, (size_t)(t0 + j) * kTerms, H, b);
+  // a quad of lanes per 16-element block, four elements each; every warp runs
+  // the same number of rounds (the quads' shuffles need all its lanes)
+  const int nb = H / 16, total = nt * nb;
+  const int nq = blockDim.x >> 2, lq = threadIdx.x & 3;
+  for (int base = part * nq; base < total; base += nparts * nq) {
+    const int idx = base + (threadIdx.x >> 2);
+    const bool valid = idx < total;
+    const int j = valid ? idx / nb : 0, b = valid ? idx - j * nb : 0;
+    float r[4] = {0.f, 0.f, 0.f, 0.f};
+    if (valid) {
+      const uint2 v = *reinterpret_cast<const uint2*>(xs + (size_t)j * H + 16 * b + 4 * lq);
+      const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&v.x));
+      const float2 c = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&v.y));
+      r[0] = a.x * s_sc[j];
+      r[1] = a.y * s_sc[j];
+      r[2] = c.x * s_sc[j];
+      r[3] = c.y * s_sc[j];
+    }
+    uint32_t pt[kTerms], sf[kTerms];
+    encode_terms16_quad(r, pt, sf);
+    store_terms16_quad(pt, sf, valid, xq, xsf, (size_t)(t0 + j) * kTerms, H, b);
   }
 }
 
