@@ -40,6 +40,8 @@ cudaError_t launch_swiglu_terms(int rows, int sms, const FfnParams& p, cudaStrea
   int blocks = rows;
   if (blocks > 8 * sms) blocks = 8 * sms;
   if (blocks < 1) blocks = 1;
+  if (rows > kSwigluQuadMaxRows)
+    return launch_pdl(swiglu_terms_rows_kernel, dim3(blocks), dim3(128), 0, st, p, rows);
   return launch_pdl(swiglu_terms_kernel, dim3(blocks), dim3(kSwigluThreads), 0, st, p, rows);
 }
 

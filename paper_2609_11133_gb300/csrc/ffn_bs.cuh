@@ -47,6 +47,8 @@ constexpr int kBsProducerWarp2 = 10;
 constexpr uint32_t kBsTmemCols = 512;
 constexpr int kBsSfCols = 48;  // per stage: A scales 2 x 16 columns, B scales 16
 constexpr int kSwigluThreads = 384;  // swiglu_terms_kernel: 96 quads of lanes
+// above this many rows the 128-thread kernel (more rows in flight per SM) runs
+constexpr int kSwigluQuadMaxRows = 512;
 
 template <int NT>
 struct BsGeom {
@@ -538,6 +540,63 @@ __global__ void __launch_bounds__(kSwigluThreads, 2) swiglu_terms_kernel(const F
         uint32_t part[kTerms], sf[kTerms];
         encode_terms16_quad(r, part, sf);
         store_terms16_quad(part, sf, b < nb, p.hq, p.hsf, (size_t)row * kTerms, p.I, b);
+      }
+    }
+    if (threadIdx.x == 0) p.hinv[row] = 1.f / sc;
+    __syncthreads();  // s_max is reused by the next row
+  }
+}
+
+// The same SwiGLU with one thread per 16-column block (encode_terms16 run
+// serially by that thread) in 128-thread CTAs: more rows in flight per SM
+// (five CTAs), which pays when there are many rows.  Same codes as the quad
+// kernel.
+__global__ void __launch_bounds__(128) swiglu_terms_rows_kernel(const FfnParams p, int rows) {
+  constexpr int G = 4;  // blocks per thread (I <= 8192)
+  __shared__ float s_max[4];
+  // the down step may launch now: what it does before its own wait (plan,
+  // weight copies) does not read this kernel's output
+  pdl_launch_dependents();
+  pdl_wait();
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int nb = p.I / 16;
+  for (int row = blockIdx.x; row < rows; row += gridDim.x) {
+    const float* g = p.gu + (size_t)row * 2 * p.I;
+    const float* u = g + p.I;
+    float h[G][16];
+    float amax = 0.f;
+#pragma unroll
+    for (int q = 0; q < G; ++q) {
+      const int b = threadIdx.x + 128 * q;
+      if (b < nb) {
+#pragma unroll
+        for (int i = 0; i < 16; i += 4) {
+          const float4 gv = __ldcg(reinterpret_cast<const float4*>(g + 16 * b + i));
+          const float4 uv = __ldcg(reinterpret_cast<const float4*>(u + 16 * b + i));
+          h[q][i + 0] = gv.x / (1.f + expf(-gv.x)) * uv.x;
+          h[q][i + 1] = gv.y / (1.f + expf(-gv.y)) * uv.y;
+          h[q][i + 2] = gv.z / (1.f + expf(-gv.z)) * uv.z;
+          h[q][i + 3] = gv.w / (1.f + expf(-gv.w)) * uv.w;
+        }
+#pragma unroll
+        for (int i = 0; i < 16; ++i) amax = fmaxf(amax, fabsf(h[q][i]));
+      }
+    }
+    amax = warp_max(amax);
+    if (lane == 0) s_max[warp] = amax;
+    __syncthreads();
+    amax = fmaxf(fmaxf(s_max[0], s_max[1]), fmaxf(s_max[2], s_max[3]));
+    const float sc = pow2_scale_terms(amax);
+#pragma unroll
+    for (int q = 0; q < G; ++q) {
+      const int b = threadIdx.x + 128 * q;
+      if (b < nb) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) h[q][i] *= sc;
+        uint2 codes[kTerms];
+        uint32_t sf[kTerms];
+        encode_terms16(h[q], codes, sf);
+        store_terms16(codes, sf, p.hq, p.hsf, (size_t)row * kTerms, p.I, b);
       }
     }
     if (threadIdx.x == 0) p.hinv[row] = 1.f / sc;
