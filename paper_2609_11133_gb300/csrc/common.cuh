@@ -290,9 +290,6 @@ __device__ __forceinline__ void red_add_f32(float* p, float v) {
   asm volatile("red.global.add.f32 [%0], %1;" ::"l"(p), "f"(v) : "memory");
 }
 
-__device__ __forceinline__ float ld_cg_f32(const float* p) { return __ldcg(p); }
-__device__ __forceinline__ int ld_cg_i32(const int* p) { return __ldcg(p); }
-
 // Power-of-two factor that maps max|v| into [2^14, 2^15): f16 holds the
 // scaled value exactly for every bf16 input and leaves headroom for sums.
 __device__ __forceinline__ float pow2_scale_for(float amax) {
@@ -355,15 +352,6 @@ __device__ __forceinline__ void tc_commit(uint64_t* bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
                    smem_u32(bar))
                : "memory");
-}
-// D[tmem] (+)= A[tmem] * B[smem];  kind::f16 (f16 inputs, f32 accumulate).
-__device__ __forceinline__ void tc_mma_f16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
-                                              uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n .reg .pred p;\n setp.ne.u32 p, %4, 0;\n"
-      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d_tmem),
-      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
-      : "memory");
 }
 // 16 consecutive 32-bit columns of this thread's lane.
 __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&v)[16]) {
