@@ -107,6 +107,25 @@ int moe_workspace_size(const moe_expert_weights_t* w, int T, int k, size_t* byte
 /* Bytes of device workspace needed by moe_route_topk for T tokens, E experts. */
 int moe_route_workspace_size(int T, int E, size_t* bytes);
 
+/* How the tensor-core expert kernels divide their stages between CTAs: the
+ * first stage that begins at or after the fraction num / den of the layer's
+ * total cost.  Runs the kernels' own split function on the host, on the plan
+ * the kernels build from the per-expert token counts.  Pure host computation;
+ * a diagnostic for tests and tuning, not a step of the decode layer.
+ *   counts [E] int32, host: tokens per expert (the plan lists the experts with
+ *     tokens in increasing id order).
+ *   Stage order: active expert, row tile (rtiles of them), chunk of NT tokens,
+ *     K-block (KB of them).  A stage of a chunk with n tokens costs a + b * n.
+ *   *stage (host): the first stage s whose preceding stages cost at least
+ *     floor(C * num / den), C the total cost; 0 for num = 0, every stage for
+ *     num = den.
+ *   MOE_ERR_INVALID_ARG: null pointer, negative count, NT outside [1, 256],
+ *     rtiles, KB or a below 1, b below 0, den below 1, num outside [0, den].
+ *   MOE_ERR_UNSUPPORTED_SHAPE: E outside [1, 512], 2^31 stages or more, more
+ *     than 2^24 tokens, a or b above 2^16, or C * num above 2^62. */
+int moe_cost_split_stage(const int32_t* counts, int E, int NT, int rtiles, int KB, int a, int b,
+                         long long num, long long den, int* stage);
+
 /* Zero a workspace (cudaMemsetAsync).  A workspace must be zeroed once
  * before its first use; the library keeps it consistent afterwards (its
  * counters are reset by their last user).  After moe_read_status() reports

@@ -55,6 +55,8 @@ _SIGS = {
     "moe_version": [],
     "moe_workspace_size": [ctypes.POINTER(ExpertWeightsC), _I, _I, ctypes.POINTER(_SZ)],
     "moe_route_workspace_size": [_I, _I, ctypes.POINTER(_SZ)],
+    "moe_cost_split_stage": [_P, _I, _I, _I, _I, _I, _I, ctypes.c_longlong, ctypes.c_longlong,
+                             ctypes.POINTER(_I)],
     "moe_workspace_init": [_P, _SZ, _P],
     "moe_read_status": [_P, _SZ, ctypes.POINTER(_I), _P],
     "moe_route_topk": [_P, _P, _P, _I, _I, _I, _I, _I, _P, _P, _P, _P, _SZ, _P],
@@ -140,6 +142,17 @@ def moe_route_workspace_size(T: int, E: int) -> int:
     n = _SZ(0)
     _check(load().moe_route_workspace_size(T, E, ctypes.byref(n)), "moe_route_workspace_size")
     return n.value
+
+
+def moe_cost_split_stage(counts, NT: int, rtiles: int, KB: int, a: int, b: int, num: int,
+                         den: int) -> int:
+    """The expert kernels' stage split for num / den of the total cost, run on the host
+    (counts: tokens per expert, any int sequence)."""
+    arr = (ctypes.c_int32 * len(counts))(*[int(c) for c in counts])
+    out = _I(0)
+    _check(load().moe_cost_split_stage(arr, len(counts), NT, rtiles, KB, a, b, num, den,
+                                       ctypes.byref(out)), "moe_cost_split_stage")
+    return out.value
 
 
 def alloc_workspace(nbytes: int, device=None) -> torch.Tensor:

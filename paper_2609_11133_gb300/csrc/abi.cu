@@ -362,6 +362,41 @@ int moe_route_workspace_size(int T, int E, size_t* bytes) {
   return MOE_OK;
 }
 
+int moe_cost_split_stage(const int32_t* counts, int E, int NT, int rtiles, int KB, int a, int b,
+                         long long num, long long den, int* stage) {
+  if (!counts || !stage || NT < 1 || NT > 256 || rtiles < 1 || KB < 1) return MOE_ERR_INVALID_ARG;
+  if (a < 1 || b < 0 || den < 1 || num < 0 || num > den) return MOE_ERR_INVALID_ARG;
+  if (E < 1 || E > kMaxE) return MOE_ERR_UNSUPPORTED_SHAPE;
+  // the plan the kernels build in shared memory, built here by a plain scan
+  PlanSmem pl;
+  long long off = 0, ch = 0;
+  int n = 0;
+  for (int e = 0; e < E; ++e) {
+    const int c = counts[e];
+    if (c < 0) return MOE_ERR_INVALID_ARG;
+    if (c == 0) continue;
+    pl.act[n] = e;
+    pl.acnt[n] = c;
+    pl.aoff[n] = (int)off;
+    pl.cpre[n] = (int)ch;
+    off += c;
+    ch += (c + NT - 1) / NT;
+    ++n;
+    if (off > (1 << 24)) return MOE_ERR_UNSUPPORTED_SHAPE;
+  }
+  pl.nA = n;
+  pl.aoff[n] = (int)off;
+  pl.cpre[n] = (int)ch;
+  // stage indices are int; the scaled cost prefix C * num is long long
+  const long long stages = ch * rtiles * KB;
+  if (stages >= (1ll << 31)) return MOE_ERR_UNSUPPORTED_SHAPE;
+  if (a > (1 << 16) || b > (1 << 16)) return MOE_ERR_UNSUPPORTED_SHAPE;
+  const long long C = (long long)rtiles * KB * ((long long)a * ch + (long long)b * off);
+  if (C > 0 && num > (1ll << 62) / C) return MOE_ERR_UNSUPPORTED_SHAPE;
+  *stage = cost_split_stage(pl, rtiles, KB, NT, a, b, num, den);
+  return MOE_OK;
+}
+
 int moe_workspace_init(void* ws, size_t ws_bytes, void* stream) {
   if (!ws) return MOE_ERR_INVALID_ARG;
   return cudaMemsetAsync(ws, 0, ws_bytes, (cudaStream_t)stream) == cudaSuccess ? MOE_OK

@@ -212,8 +212,9 @@ __host__ __device__ constexpr int stage_cost_base(bool per_token_rows) {
 // the fraction num / den of the total cost.  The cost prefix over active
 // experts follows from the chunk and token prefixes: sum of (a * chunks + b *
 // tokens) per row tile and K-stage.  f(0) = 0, f(den) = every stage, f
-// increasing in num.
-__device__ __forceinline__ int cost_split_stage(const PlanSmem& pl, int rtiles, int KB, int NT,
+// increasing in num.  Host-callable so that the library can run the same code
+// on a plan built from counts (moe_cost_split_stage).
+__host__ __device__ __forceinline__ int cost_split_stage(const PlanSmem& pl, int rtiles, int KB, int NT,
                                                 int a, int b, long long num, long long den) {
   const long long per = (long long)rtiles * KB;
   auto prefix = [&](int s) {

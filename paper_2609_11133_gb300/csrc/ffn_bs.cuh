@@ -161,9 +161,9 @@ __global__ void __launch_bounds__(kBsThreads, 1)
   const int K = (PHASE == 1) ? p.H : p.I;  // contraction length
   const int rtiles = (PHASE == 1) ? p.I / kRowsHalf : p.H / (2 * kRowsHalf);
   const int KB = K / KEL;
-  // stages of all items (< 2^31 for every supported shape), this CTA's share
-  // this CTA's share of the stages, divided by cost (items of many tokens
-  // cost more per stage when their rows come token by token)
+  // this CTA's share of the stages of all items (< 2^31 for every supported
+  // shape), divided by cost (items of many tokens cost more per stage when
+  // their rows come token by token)
   const int cost_a = stage_cost_base((PHASE == 1) && !p.b_compact);
   const int s_begin = cost_split_stage(pl, rtiles, KB, NT, cost_a, kTokenCost, blockIdx.x, gridDim.x);
   const int s_end = cost_split_stage(pl, rtiles, KB, NT, cost_a, kTokenCost, blockIdx.x + 1,
