@@ -636,7 +636,7 @@ def run_ours(args):
                      "peak_source": peak_src},
         "e2e": {"value": job_throughput(ms_e2e, T, world), "unit": "tokens/s",
                 "h2d_bytes_per_step": T * H * 2, "d2h_bytes_per_step": T * H * 2},
-        "gpu_launches": 5 * L * args.steps,
+        "gpu_launches": binding.moe_layer_kernel_count(layers[0][0], T, k) * L * args.steps,
         "timing": f"CUDA-graph replay, {G} steps (layer calls) per graph",
         "repeats": repeats,
         "latency": latency,

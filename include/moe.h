@@ -104,6 +104,13 @@ int moe_version(void);
  * Pure host computation. */
 int moe_workspace_size(const moe_expert_weights_t* w, int T, int k, size_t* bytes);
 
+/* Kernels one moe_decode_layer call launches for these weights and T tokens
+ * with k experts each (*count, host pointer): the router, the gather of the
+ * activation terms (tensor-core engines, T > 64), gate/up, SwiGLU, down and
+ * the bf16 finalize.  0 for T = 0.  Pure host computation; errors as
+ * moe_workspace_size. */
+int moe_layer_kernel_count(const moe_expert_weights_t* w, int T, int k, int* count);
+
 /* Bytes of device workspace needed by moe_route_topk for T tokens, E experts. */
 int moe_route_workspace_size(int T, int E, size_t* bytes);
 

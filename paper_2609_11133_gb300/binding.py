@@ -55,6 +55,7 @@ _SIGS = {
     "moe_version": [],
     "moe_workspace_size": [ctypes.POINTER(ExpertWeightsC), _I, _I, ctypes.POINTER(_SZ)],
     "moe_route_workspace_size": [_I, _I, ctypes.POINTER(_SZ)],
+    "moe_layer_kernel_count": [ctypes.POINTER(ExpertWeightsC), _I, _I, ctypes.POINTER(_I)],
     "moe_cost_split_stage": [_P, _I, _I, _I, _I, _I, _I, ctypes.c_longlong, ctypes.c_longlong,
                              ctypes.POINTER(_I)],
     "moe_workspace_init": [_P, _SZ, _P],
@@ -135,6 +136,14 @@ def moe_workspace_size(w, T: int, k: int) -> int:
     ws = weights_struct(w)
     _check(load().moe_workspace_size(ctypes.byref(ws), T, k, ctypes.byref(n)),
            "moe_workspace_size")
+    return n.value
+
+
+def moe_layer_kernel_count(w, T: int, k: int) -> int:
+    n = _I(0)
+    ws = weights_struct(w)
+    _check(load().moe_layer_kernel_count(ctypes.byref(ws), T, k, ctypes.byref(n)),
+           "moe_layer_kernel_count")
     return n.value
 
 

@@ -355,6 +355,17 @@ int moe_workspace_size(const moe_expert_weights_t* w, int T, int k, size_t* byte
   return MOE_OK;
 }
 
+int moe_layer_kernel_count(const moe_expert_weights_t* w, int T, int k, int* count) {
+  if (!count) return MOE_ERR_INVALID_ARG;
+  int rc = check_weights(w);
+  if (rc) return rc;
+  rc = check_tk(T, k, w->E);
+  if (rc) return rc;
+  // route, (gather), gate/up, SwiGLU, down, finalize
+  *count = (T == 0) ? 0 : 5 + (gather_terms(T, act_for(w->fmt, engine_for(w->fmt))) ? 1 : 0);
+  return MOE_OK;
+}
+
 int moe_route_workspace_size(int T, int E, size_t* bytes) {
   if (!bytes || T < 0) return MOE_ERR_INVALID_ARG;
   if (E < 1 || E > kMaxE) return MOE_ERR_UNSUPPORTED_SHAPE;

@@ -104,3 +104,21 @@ def test_other_entry_points_validate(lib):
     assert lib.moe_route_workspace_size(4, 8, ctypes.byref(n)) == 0 and n.value > 0
     assert lib.moe_route_topk(P(16), P(16), None, 4, 512, 8, 2, 1, P(16), P(16), None,
                               P(256), n.value - 1, None) == -3
+
+
+def test_layer_kernel_count(lib):
+    def count(c, T, k):
+        n = ctypes.c_int(-1)
+        rc = lib.moe_layer_kernel_count(ctypes.byref(c), T, k, ctypes.byref(n))
+        return rc, n.value
+
+    # route, gate/up, SwiGLU, down and finalize; the gather of the activation
+    # terms joins above 64 tokens
+    for fmt in (1, 2):
+        assert count(fake_weights(fmt=fmt), 0, 2) == (0, 0)
+        assert count(fake_weights(fmt=fmt), 64, 2) == (0, 5)
+        assert count(fake_weights(fmt=fmt), 65, 2) == (0, 6)
+    assert count(fake_weights(), 4, 0)[0] == -1
+    assert count(fake_weights(fmt=3), 4, 2)[0] == -1
+    assert count(fake_weights(E=600), 4, 2)[0] == -2
+    assert lib.moe_layer_kernel_count(ctypes.byref(fake_weights()), 4, 2, None) == -1
