@@ -184,7 +184,12 @@ __global__ void __launch_bounds__(kBsThreads, 1)
       tma_prefetch_desc(&tmS0);
       tma_prefetch_desc(&tmS1);
       tma_prefetch_desc(&tmB);
+      // weights stream through L2 once (evict first), except the tile of an
+      // item whose expert has tokens in a later chunk: that chunk's item,
+      // next in the order, reads the same tile again (evict last)
       const uint64_t pol_w = policy_evict_first();
+      const uint64_t pol_keep = policy_evict_last();
+      uint64_t pol_item = pol_w;
       const uint64_t pol_a = policy_evict_last();
       int cur_item = -1;
       ItemInfo inf{};
@@ -195,6 +200,7 @@ __global__ void __launch_bounds__(kBsThreads, 1)
         if (it != cur_item) {
           cur_item = it;
           inf = decode_item(it, rtiles, pl, p, NT);
+          pol_item = (inf.arow0 + NT < pl.aoff[inf.slot] + pl.acnt[inf.slot]) ? pol_keep : pol_w;
           if (!lead && btok)
             for (int j = 0; j < inf.nvalid; ++j) s_tok[j] = __ldg(p.sorted + inf.lrow0 + j) / p.k;
         }
@@ -226,17 +232,17 @@ __global__ void __launch_bounds__(kBsThreads, 1)
         // stages, whose weights the lead copies before the SwiGLU kernel ends.
         const bool a1_lead = early && issued < S;
         if (lead) {
-          tma_load_2d(st + G::A0, &tmA0, &full_bar[slot], kb * kRowBytes, rowA0, pol_w);
-          tma_load_2d(st + G::S0, &tmS0, &full_bar[slot], kb * 16, rowA0, pol_w);
+          tma_load_2d(st + G::A0, &tmA0, &full_bar[slot], kb * kRowBytes, rowA0, pol_item);
+          tma_load_2d(st + G::S0, &tmS0, &full_bar[slot], kb * 16, rowA0, pol_item);
           if (a1_lead) {
-            tma_load_2d(st + G::A1, &tmA1, &full_bar[slot], kb * kRowBytes, rowA1, pol_w);
-            tma_load_2d(st + G::S1, &tmS1, &full_bar[slot], kb * 16, rowA1, pol_w);
+            tma_load_2d(st + G::A1, &tmA1, &full_bar[slot], kb * kRowBytes, rowA1, pol_item);
+            tma_load_2d(st + G::S1, &tmS1, &full_bar[slot], kb * 16, rowA1, pol_item);
           }
           continue;
         }
         if (!a1_lead) {
-          tma_load_2d(st + G::A1, &tmA1, &full_bar[slot], kb * kRowBytes, rowA1, pol_w);
-          tma_load_2d(st + G::S1, &tmS1, &full_bar[slot], kb * 16, rowA1, pol_w);
+          tma_load_2d(st + G::A1, &tmA1, &full_bar[slot], kb * kRowBytes, rowA1, pol_item);
+          tma_load_2d(st + G::S1, &tmS1, &full_bar[slot], kb * 16, rowA1, pol_item);
         }
         // activation terms: token j's four rows land at B rows 4j..4j+3
         if (btok) {

@@ -161,7 +161,12 @@ __global__ void __launch_bounds__(kF8Threads, 1)
       tma_prefetch_desc(&tmA0);
       tma_prefetch_desc(&tmA1);
       if (!lead) tma_prefetch_desc(&tmB);
+      // weights stream through L2 once (evict first), except the tile of an
+      // item whose expert has tokens in a later chunk: that chunk's item,
+      // next in the order, reads the same tile again (evict last)
       const uint64_t pol_w = policy_evict_first();
+      const uint64_t pol_keep = policy_evict_last();
+      uint64_t pol_item = pol_w;
       const uint64_t pol_a = policy_evict_last();
       int cur_item = -1;
       ItemInfo inf{};
@@ -177,6 +182,7 @@ __global__ void __launch_bounds__(kF8Threads, 1)
           if (it != cur_item) {
             cur_item = it;
             inf = decode_item(it, rtiles, pl, p, NT);
+            pol_item = (inf.arow0 + NT < pl.aoff[inf.slot] + pl.acnt[inf.slot]) ? pol_keep : pol_w;
             if (!lead && btok)
               for (int j = 0; j < inf.nvalid; ++j) s_tok[j] = __ldg(p.sorted + inf.lrow0 + j) / p.k;
           }
@@ -205,13 +211,13 @@ __global__ void __launch_bounds__(kF8Threads, 1)
             mbar_arrive_expect_tx(&full_bar[slot], bytes);
             // box A0 always; box A1 too for the down step's first ring of
             // stages, copied before the SwiGLU kernel ends
-            tma_load_2d(st + G::A0, &tmA0, &full_bar[slot], kb * kRowBytes, rowA0, pol_w);
+            tma_load_2d(st + G::A0, &tmA0, &full_bar[slot], kb * kRowBytes, rowA0, pol_item);
             if (early && issued < S)
-              tma_load_2d(st + G::A1, &tmA1, &full_bar[slot], kb * kRowBytes, rowA1, pol_w);
+              tma_load_2d(st + G::A1, &tmA1, &full_bar[slot], kb * kRowBytes, rowA1, pol_item);
             continue;
           }
           if (!(early && issued < S))
-            tma_load_2d(st + G::A1, &tmA1, &full_bar[slot], kb * kRowBytes, rowA1, pol_w);
+            tma_load_2d(st + G::A1, &tmA1, &full_bar[slot], kb * kRowBytes, rowA1, pol_item);
           // activation terms: token j's two rows land at B rows 2j, 2j+1
           if (btok) {
             for (int j = 0; j < inf.nvalid; ++j)
