@@ -32,13 +32,19 @@
  *   with moe_read_status().  No exception or abort crosses the ABI.
  *
  * Arithmetic of the GPU path: fp32 router and gates; expert products
- * accumulate in fp32.  FP8 weights are decoded exactly to f16 and multiplied
- * with the f16 activations (exact for bf16 inputs after a power-of-two row
- * scale).  NVFP4 weights are fed to the tensor cores as stored (block-scaled
- * MMA, E2M1 x UE4M3 per 16 K); the activations (x, and h between the gate/up
- * and down steps) are encoded as sums of four NVFP4 terms per row, each term
- * coding the previous terms' residual, which leaves less than 2^-9.5 of each
- * 16-element block's maximum uncoded.
+ * accumulate in fp32.  Both formats feed their weights to the tensor cores
+ * as stored, and the activations (x, and h between the gate/up and down
+ * steps) are encoded in the weights' format family:
+ * - NVFP4: block-scaled MMA (E2M1 x UE4M3 per 16 K); each activation row is
+ *   a sum of four NVFP4 terms, each term coding the previous terms'
+ *   residual, which leaves less than 2^-9.5 of each 16-element block's
+ *   maximum uncoded.
+ * - FP8: E4M3 x E4M3 MMA per 128-K block, the block scales applied in fp32;
+ *   each activation row is two E4M3 terms, hi = e4m3(v) and lo = e4m3(v -
+ *   hi), after a power-of-two row scale.
+ * The environment variable MOE_ENGINE=mma selects instead a warp-MMA engine
+ * that decodes the weights exactly to f16 and multiplies them with exact f16
+ * activations (bf16 inputs after a power-of-two row scale).
  *
  * Expert weight formats (moe_expert_weights_t)
  *   gate and up are [E, I, H]-shaped (N = I rows, K = H contiguous),
