@@ -1,11 +1,12 @@
 """ctypes binding of libmoe.so (the C ABI in include/moe.h).
 
-Argument marshalling only: every function here takes torch tensors that
-already live on the GPU, passes their device pointers and the current CUDA
-stream to the C function of the same name, and raises ``MoeError`` on a
-non-zero status.  No computation happens in Python, and there is no
-fallback: if the library cannot be loaded, importing this module's
-functions raises.
+Argument marshalling only: every function here calls the C function of the
+same name and raises ``MoeError`` on a non-zero status.  The layer's steps
+take torch tensors that already live on the GPU and pass their device
+pointers and the current CUDA stream; the host-only calls (workspace sizes,
+the kernel count of a layer call, the expert kernels' stage split) take host
+values.  No computation happens in Python, and there is no fallback: if the
+library cannot be loaded, calling this module's functions raises.
 """
 from __future__ import annotations
 
