@@ -1,5 +1,9 @@
 // Expert FFN kernels of the MoE decode layer (gate/up + SwiGLU, and down +
-// combine), for FP8 E4M3 with 128x128 fp32 block scales and NVFP4.
+// combine), for FP8 E4M3 with 128x128 fp32 block scales and NVFP4: what the
+// three engines share (parameters, work plan, stage split and cursors, the
+// FP8 engine's shared tail, SwiGLU and finalize kernels), and the warp-MMA
+// engine itself (ffn_kernel).  The tensor-core engines are in ffn_bs.cuh
+// (NVFP4) and ffn_f8.cuh (FP8).
 //
 // Shape of the work.  Per active expert e with n_e routed tokens, the
 // gate/up step streams 2*I*H weights and the down step H*I weights, each
@@ -7,29 +11,32 @@
 // HBM-bound weight streams (the decode-lane regime of the paper's
 // Section 2.1).  The kernels are built around keeping HBM busy:
 //
-// * Work list.  Items are (active expert, token chunk of <= NT tokens,
-//   row tile); each item is a run of K-blocks ("stages").  The stages of
-//   all items are laid end to end and every CTA of a persistent grid takes
-//   an equal contiguous share of them (stream-K), so every SM streams the
-//   same number of bytes whatever the routing.  Partial sums of an item
-//   split between CTAs meet in fp32 accumulators through red.global.add.
-// * Pipeline.  One producer thread issues 2-D TMA tensor copies of each
-//   stage (two 128-row x 128-byte weight boxes with 128B swizzle, the NVFP4
-//   scale boxes, and the stage's token rows) into a ring of shared-memory
-//   stages guarded by mbarriers; consumer warps (eight per 128-row box, or
-//   sixteen with each stage's K split in two) decode and multiply.
-// * Decode.  E4M3 and E2M1*E4M3 values are exact in f16, so weights are
-//   converted exactly in registers (cvt e4m3x2/e2m1x2 -> f16x2; the NVFP4
-//   per-16 scale multiplied in f16, still exact).  Activations are stored
-//   as f16 after a per-row power-of-two scaling (exact for bf16 inputs).
-//   The tensor pipe (mma m16n8k16, fp32 accumulate) does the multiply-adds
-//   with the tokens as the n=8 side; FP8 block scales and NVFP4 tensor
-//   scales are applied to the fp32 accumulators.
+// * Work list.  Items are (active expert, row tile, token chunk of <= NT
+//   tokens); each item is a run of K-blocks ("stages").  The stages of all
+//   items are laid end to end and every CTA of a persistent grid takes a
+//   contiguous share of them (stream-K): an equal share in the warp-MMA
+//   engine, a share of equal cost in the tensor-core engines
+//   (cost_split_stage), where the FP8 engine also leaves a shared tail of
+//   units to whichever CTA is free.  Partial sums of an item split between
+//   CTAs meet in fp32 accumulators through red.global.add.
+// * Pipeline.  Producer threads issue 2-D TMA tensor copies of each stage
+//   (weight boxes of 128 rows x 128 bytes with 128B swizzle, the NVFP4 scale
+//   boxes, and the stage's token rows) into a ring of shared-memory stages
+//   guarded by mbarriers.  In the warp-MMA engine consumer warps (eight per
+//   128-row box, or sixteen with each stage's K split in two) decode and
+//   multiply.
+// * Decode (warp-MMA engine).  E4M3 and E2M1*E4M3 values are exact in f16,
+//   so weights are converted exactly in registers (cvt e4m3x2/e2m1x2 ->
+//   f16x2; the NVFP4 per-16 scale multiplied in f16, still exact).
+//   Activations are stored as f16 after a per-row power-of-two scaling
+//   (exact for bf16 inputs).  mma m16n8k16 (fp32 accumulate) does the
+//   multiply-adds with the tokens as the n=8 side; FP8 block scales and
+//   NVFP4 tensor scales are applied to the fp32 accumulators.
 // * Fusion.  The gate/up step adds fp32 pre-activations into [T*k, 2I]
-//   accumulators; swiglu_kernel turns them into the f16 input of the down
-//   step.  The down step multiplies by the gate weight and adds straight into
-//   a [T, H] fp32 accumulator (the scatter-combine); finalize_kernel writes
-//   bf16 (+ residual).  No wait depends on another CTA.
+//   accumulators; a SwiGLU kernel turns them into the down step's input.
+//   The down step multiplies by the gate weight and adds straight into a
+//   [T, H] fp32 accumulator (the scatter-combine); finalize_kernel writes
+//   bf16 (+ residual).
 #pragma once
 
 #include "common.cuh"
