@@ -1,5 +1,7 @@
-// Activations as sums of NVFP4-coded terms, the B operand of the block-scaled
-// tensor-core engine (ffn_bs.cuh).
+// Activations as sums of low-precision terms, the B operand of the
+// tensor-core engines: four NVFP4 terms per row for the block-scaled engine
+// (ffn_bs.cuh, below), two E4M3 terms per row for the FP8 engine (ffn_f8.cuh,
+// at the end of this file).
 //
 // The tcgen05 kind::mxf4nvf4 MMA multiplies E2M1 codes with one UE4M3 scale
 // per 16 K elements on BOTH operands.  The weights are stored that way; the
