@@ -6,7 +6,8 @@ also after an error; caps outside the GPU's range are refused; the acceptance ga
 throughput and the latency criterion (Algorithm 2); the mode ladder from a flat-then-cliff sweep
 (Section 3.2, Figure 3's shape); the median reference resists one noisy repetition; a changed
 engine fingerprint invalidates the result; the command line changes nothing without
---set-power-limits."""
+--set-power-limits; static clock locks need permission and are released, also after an error;
+the actuator A/B picks its lock arms by the rules of Section 5.3."""
 import pytest
 
 from paper_2609_11133_gb300 import capsweep as cs
@@ -193,3 +194,70 @@ def test_command_line_changes_nothing_without_the_flag(capsys):
     assert cs.main(["--caps", "800,600", "--slo-ms", "1"], nvml=nv) is None
     assert nv.sets == []
     assert "dry run" in capsys.readouterr().out
+
+
+class FakeClocks(FakeNvml):
+    def __init__(self, max_mhz=2070, **kw):
+        super().__init__(**kw)
+        self.max_mhz = max_mhz
+        self.locked = None
+        self.lock_calls = []
+
+    def max_sm_clock_mhz(self):
+        return self.max_mhz
+
+    def set_locked_clocks(self, lo, hi):
+        self.lock_calls.append((lo, hi))
+        self.locked = (lo, hi)
+
+    def reset_locked_clocks(self):
+        self.lock_calls.append("reset")
+        self.locked = None
+
+
+def lock_curve(nv, knee_mhz=1400.0, t0=270000.0, p_idle=300.0, p_max=900.0, slow_below=0.0):
+    """A memory-bound step under a static lock: throughput flat above the knee and falling with
+    the clock below it; draw rising with the clock squared; p99 inflated below `slow_below`."""
+    def run(reps):
+        f = nv.locked[0] if nv.locked else nv.max_mhz
+        t = t0 * min(1.0, f / knee_mhz)
+        draw = p_idle + (p_max - p_idle) * (f / nv.max_mhz) ** 2
+        p99 = 0.3 * (3.0 if f < slow_below else 1.0)
+        return cs.CapPoint(None, [t] * reps, p99, draw / t, draw)
+    return run
+
+
+def test_clock_locks_need_permission_and_are_released():
+    nv = FakeClocks()
+    with cs.ClockGuard(nv) as g:
+        with pytest.raises(PermissionError):
+            g.lock(1200)
+    assert nv.lock_calls == []
+    with pytest.raises(RuntimeError, match="failed"):
+        with cs.ClockGuard(nv, allow_set=True) as g:
+            g.lock(1200)
+            raise RuntimeError("measurement failed")
+    assert nv.locked is None and nv.lock_calls == [(1200, 1200), "reset"]
+    with cs.ClockGuard(nv, allow_set=True) as g:
+        with pytest.raises(ValueError):
+            g.lock(2100)  # above the GPU's maximum SM clock
+
+
+def test_actuator_ab_arms():
+    nv = FakeClocks()
+    run = lock_curve(nv, slow_below=800)
+    ref = run(3)
+    with cs.ClockGuard(nv, allow_set=True) as g:
+        locks = cs.lock_sweep(g, [2070, 1800, 1400, 1200, 1000, 800, 600], run, 3)
+    assert nv.locked is None and [p.lock_mhz for p in locks] == [2070, 1800, 1400, 1200, 1000, 800, 600]
+    # a cap that keeps the full throughput at 600 W (the power manager's own DVFS under it)
+    cap = cs.CapPoint(600.0, [270000.0] * 3, 0.3, 600.0 / 270000.0, 600.0)
+    rows = {r["arm"]: r for r in cs.actuator_ab(ref, cap, locks, 0.5)}
+    assert rows["clock lock, throughput-optimal"]["setting"] == "1400 MHz lock"  # lowest flat clock
+    assert rows["clock lock, aggressive"]["setting"] == "800 MHz lock"  # 600 MHz breaks the SLO
+    assert rows["power cap"]["d_throughput"] == 0.0
+    assert rows["power cap"]["d_power"] == pytest.approx(600.0 / 900.0 - 1.0)
+    assert rows["clock lock, aggressive"]["d_throughput"] == pytest.approx(800 / 1400 - 1.0)
+    # tokens/J against the default: (270000 / 600) / (270000 / 900) - 1
+    assert rows["power cap"]["d_tokens_per_j"] == pytest.approx(0.5)
+    assert all(r["slo"] for r in rows.values())
