@@ -357,6 +357,33 @@ def kernel_sources_sha256():
 
 
 # ---------------------------------------------------------------- our arm
+def gateup_roofline(wl, fmt, T, k, H, I, gu_ms, gu_gbs, peaks, traffic):
+    """The `roofline` object of the dominant kernel, gate/up.  Decode batches:
+    algorithmic bytes per launch / its CUDA-event time against the measured
+    copy rate.  A prefill-shaped batch reuses each weight tile for ~T*k/E
+    tokens, so its roofline is the tensor cores': useful gate/up FLOPs (2
+    matrices x 2 x H x I per assignment; the activation terms' extra MMA work
+    is not counted) against the dense rate of the weights' format, the
+    measured sustained bf16 rate times the nominal ratio (NVFP4 13.5 / 2.25 =
+    6, FP8 4.5 / 2.25 = 2)."""
+    hbm = float(peaks.get("hbm_gbs", 6800.0))
+    hbm_src = "measured" if "hbm_gbs" in peaks else "fallback"
+    if not wl["prefill"]:
+        return {"bound": "hbm", "achieved": gu_gbs, "peak": hbm, "unit": "GB/s",
+                "frac": gu_gbs / hbm, "traffic": traffic, "kernel": "ffn gate/up",
+                "peak_source": hbm_src}
+    ratio, name = (6.0, "NVFP4") if fmt == 2 else (2.0, "FP8")
+    tflops = 4.0 * T * k * H * I / (gu_ms * 1e-3) / 1e12
+    bf16 = peaks.get("bf16_tflops_sustained")
+    peak = ratio * (float(bf16) if bf16 else 1700.0)
+    src = (f"measured bf16 sustained x {ratio:g} ({name})" if bf16 else
+           f"fallback 1.7 PFLOP/s bf16 sustained x {ratio:g} ({name})")
+    return {"bound": "tensor", "achieved": tflops, "peak": peak, "unit": "TFLOP/s",
+            "frac": tflops / peak, "traffic": traffic, "kernel": "ffn gate/up",
+            "peak_source": src,
+            "hbm": {"achieved": gu_gbs, "peak": hbm, "unit": "GB/s", "frac": gu_gbs / hbm}}
+
+
 def run_ours(args):
     import numpy as np
     import torch
@@ -583,7 +610,6 @@ def run_ours(args):
     if os.path.exists(pp):
         peaks = json.load(open(pp))
     hbm = float(peaks.get("hbm_gbs", 6800.0))
-    peak_src = "measured" if "hbm_gbs" in peaks else "fallback"
     gu_ms = statistics.mean(kern[1]) / L
     dn_ms = statistics.mean(kern[2]) / L
     rt_ms = statistics.mean(kern[0]) / L
@@ -614,24 +640,7 @@ def run_ours(args):
     if wl["zipf"]:
         cfg["router_bias"] = f"zipf s={wl['zipf']}"
         cfg["popularity"] = zipf_stats(ids[0].cpu().numpy(), E)
-    roofline = {"bound": "hbm", "achieved": gu_gbs, "peak": hbm, "unit": "GB/s",
-                "frac": gu_gbs / hbm, "traffic": traffic, "kernel": "ffn gate/up",
-                "peak_source": peak_src}
-    if wl["prefill"]:
-        # A prefill-shaped batch reuses each weight tile for ~T*k/E tokens: the
-        # tensor-core roofline.  Useful FLOPs of gate/up: 2 matrices x 2 x H x I
-        # per assignment (the activation terms' extra MMA work is not counted).
-        # Peak: the dense NVFP4 rate, the measured sustained bf16 rate x 6 (the
-        # nominal 13.5 / 2.25 PFLOP/s ratio).
-        gu_tflops = 4.0 * T * k * H * I / (gu_ms * 1e-3) / 1e12
-        bf16 = peaks.get("bf16_tflops_sustained")
-        tpk = 6.0 * float(bf16) if bf16 else 6.0 * 1700.0
-        roofline = {"bound": "tensor", "achieved": gu_tflops, "peak": tpk, "unit": "TFLOP/s",
-                    "frac": gu_tflops / tpk, "traffic": traffic, "kernel": "ffn gate/up",
-                    "peak_source": ("measured bf16 sustained x 6" if bf16 else
-                                    "fallback 1.7 PFLOP/s bf16 sustained x 6"),
-                    "hbm": {"achieved": gu_gbs, "peak": hbm, "unit": "GB/s",
-                            "frac": gu_gbs / hbm}}
+    roofline = gateup_roofline(wl, fmt, T, k, H, I, gu_ms, gu_gbs, peaks, traffic)
     kind = "prefill-shaped layer" if wl["prefill"] else "decode-layer"
     res = {
         "metric": f"MoE {kind} tokens/s" if L == 1 else f"MoE {L}-layer decode-step tokens/s",
