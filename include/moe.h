@@ -46,6 +46,14 @@
  * that decodes the weights exactly to f16 and multiplies them with exact f16
  * activations (bf16 inputs after a power-of-two row scale).
  *
+ * Environment (read by the library; none is needed):
+ *   MOE_ENGINE=mma        the warp-MMA engine above (read once per process)
+ *   MOE_NT=8|16|32        token-chunk width of the expert kernels instead of
+ *                         the default (8 up to 64 tokens, else 16 for NVFP4
+ *                         and 32 for FP8); 32 is not taken for NVFP4
+ *   MOE_WAIT_LIMIT_MS=n   limit in ms of every bounded device wait, 1-60000
+ *                         (default 1000; read once per process)
+ *
  * Expert weight formats (moe_expert_weights_t)
  *   gate and up are [E, I, H]-shaped (N = I rows, K = H contiguous),
  *   down is [E, H, I]-shaped (N = H rows, K = I contiguous).
