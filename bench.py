@@ -357,6 +357,13 @@ def kernel_sources_sha256():
 
 
 # ---------------------------------------------------------------- our arm
+def metric_name(wl):
+    """The metric both arms report for a workload."""
+    if wl["layers"] > 1:
+        return f"MoE {wl['layers']}-layer decode-step tokens/s"
+    return "MoE prefill-shaped layer tokens/s" if wl["prefill"] else "MoE decode-layer tokens/s"
+
+
 def gateup_roofline(wl, fmt, T, k, H, I, gu_ms, gu_gbs, peaks, traffic):
     """The `roofline` object of the dominant kernel, gate/up.  Decode batches:
     algorithmic bytes per launch / its CUDA-event time against the measured
@@ -641,9 +648,8 @@ def run_ours(args):
         cfg["router_bias"] = f"zipf s={wl['zipf']}"
         cfg["popularity"] = zipf_stats(ids[0].cpu().numpy(), E)
     roofline = gateup_roofline(wl, fmt, T, k, H, I, gu_ms, gu_gbs, peaks, traffic)
-    kind = "prefill-shaped layer" if wl["prefill"] else "decode-layer"
     res = {
-        "metric": f"MoE {kind} tokens/s" if L == 1 else f"MoE {L}-layer decode-step tokens/s",
+        "metric": metric_name(wl),
         "value": tok_s,
         "unit": "tokens/s",
         "n_gpus": world,
@@ -699,7 +705,7 @@ def run_reference(args):
         s.run()
     dt = sum(s.run() for _ in range(steps)) / steps
     v = s.n / (dt * L)
-    res = {"metric": "MoE decode-layer tokens/s" if L == 1 else f"MoE {L}-layer decode-step tokens/s",
+    res = {"metric": metric_name(wl),
            "value": v, "unit": "tokens/s", "n_gpus": world,
            "steps": steps, "warmup": warm, "ms_per_step": dt * L * 1e3 * T / s.n,
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",

@@ -45,3 +45,11 @@ def test_every_workload_parses():
     for name in bench.WORKLOADS:
         wl = bench.workload(bench.parse(["--workload", name]))
         assert wl["name"].startswith(name) and wl["T"] >= 1
+
+
+def test_both_arms_name_the_same_metric():
+    names = {n: bench.metric_name(bench.workload(bench.parse(["--workload", n])))
+             for n in bench.WORKLOADS}
+    assert names["qwen3_235b_nvfp4"] == "MoE decode-layer tokens/s"
+    assert names["qwen3_235b_nvfp4_prefill"] == "MoE prefill-shaped layer tokens/s"
+    assert names["qwen3_235b_nvfp4_x94"] == "MoE 94-layer decode-step tokens/s"
