@@ -261,3 +261,11 @@ def test_actuator_ab_arms():
     # tokens/J against the default: (270000 / 600) / (270000 / 900) - 1
     assert rows["power cap"]["d_tokens_per_j"] == pytest.approx(0.5)
     assert all(r["slo"] for r in rows.values())
+
+
+def test_engine_fingerprint_names_the_library_and_its_kernels():
+    fp = cs.engine_fingerprint({"gpu": "GB300", "launch": "one CUDA graph per step"})
+    assert int(fp["abi_version"]) >= 100
+    assert len(fp["kernel_sources"]) == 64 and int(fp["kernel_sources"], 16) >= 0
+    assert fp["gpu"] == "GB300" and fp == cs.engine_fingerprint(
+        {"gpu": "GB300", "launch": "one CUDA graph per step"})
