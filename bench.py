@@ -640,6 +640,10 @@ def run_ours(args):
                   f"{n_rot} resident input batches rotated step by step: {B / 1e9:.3f} GB "
                   f"touched per step, {n_rot * B / 1e9:.2f} GB per rotation (L2 {l2 / 1e6:.0f} MB)"),
            "steps_per_graph": G,
+           "arithmetic": ("e2m1 x e2m1 block-scaled MMA (ue4m3 per 16), activations as 4 nvfp4 "
+                          "terms, fp32 accumulate" if fmt == 2 else
+                          "e4m3 x e4m3 MMA, 128x128 fp32 block scales applied per stage, "
+                          "activations as 2 e4m3 terms, fp32 accumulate"),
            "parallelism": f"replicas x{world}"}
     if L > 1:
         cfg.update(layers=L, prenorm="rms, eps 1e-6, unit weight", residual="threaded",
@@ -659,9 +663,7 @@ def run_ours(args):
         "higher_is_better": True,
         "scaling": "weak",
         "vs_baseline": None,
-        "dtype": "nvfp4 (e2m1 x e2m1 block-scaled MMA, activations as 4 nvfp4 terms, fp32 accumulate)"
-                 if fmt == 2 else
-                 "fp8 e4m3 (e4m3 x e4m3 MMA, activations as 2 e4m3 terms, fp32 accumulate)",
+        "dtype": "nvfp4" if fmt == 2 else "fp8_e4m3",
         "data": "synthetic (seeded N(0,1) activations, N(0,0.02) weights quantised)",
         "config": cfg,
         "hbm_gbs": layer_gbs,
