@@ -380,16 +380,6 @@ __device__ __forceinline__ void tmem_ld_wait() {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
-// Instruction descriptor of tcgen05.mma kind::f16: f32 D, f16 A and B, both
-// K-major, shape M x N.
-__host__ __device__ constexpr uint32_t tc_idesc_f16(int M, int N) {
-  return (1u << 4)                               // D format: f32
-         | (0u << 7) | (0u << 10)                // A, B: f16
-         | (0u << 15) | (0u << 16)               // A, B K-major
-         | ((uint32_t)(N >> 3) << 17)            // N / 8
-         | ((uint32_t)(M >> 4) << 24);           // M / 16
-}
-
 // Shared-memory matrix descriptor: K-major operand stored in 128-byte rows
 // with the 128B swizzle, 8-row atoms 1024 bytes apart.
 __device__ __forceinline__ uint64_t tc_desc_sw128(uint32_t smem_addr) {
