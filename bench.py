@@ -7,10 +7,11 @@ One step = one decode step (router GEMV + top-k + permute + gate/up SwiGLU
 + down + combine, for each layer of the workload) over a batch of T tokens,
 on synthetic seeded inputs.  Workloads:
 
-  qwen3_235b_nvfp4      Qwen3-235B-A22B-shaped NVFP4 layer (H=4096, E=128,
-                        top-8, I=1536), T=64 by default (the headline line)
   qwen3_480b_fp8        Qwen3-Coder-480B-shaped FP8 layer (H=6144, E=160,
-                        top-8, I=2560), T=64
+                        top-8, I=2560), T=64 (the default: the largest
+                        single-GPU decode layer of the two served models)
+  qwen3_235b_nvfp4      Qwen3-235B-A22B-shaped NVFP4 layer (H=4096, E=128,
+                        top-8, I=1536), T=64 by default
   qwen3_480b_fp8_zipf   the 480B layer with a router bias that makes expert
                         popularity follow Zipf(1.1); sweep --tokens
   qwen3_235b_nvfp4_x94  94 235B-shaped NVFP4 layers with fresh weights per
@@ -24,7 +25,11 @@ on synthetic seeded inputs.  Workloads:
 
 The metric is decode tokens/s; achieved HBM GB/s, the roofline fraction of
 the dominant kernel (gate/up) and J/token (NVML energy counter) are reported
-beside it.  Under torchrun each rank runs an independent replica on its own
+beside it.  The default run (N=1) adds a "sweep" key: the 235B-shaped NVFP4
+layer at T = 1, 8, 32, 64 and the 480B-shaped FP8 layer with Zipf-skewed
+routing at T = 1, 8, 32, 128, 256, each with its time per step, layer and
+gate/up HBM fractions against the measured copy rate and 8 TB/s, J/token and
+the SM clock over its own window (--no-sweep skips it).  Under torchrun each rank runs an independent replica on its own
 GPU (the layer does not shard across GPUs); the timed region is bracketed by
 a barrier and the slowest rank's time is reported.
 
@@ -78,7 +83,7 @@ def parse(argv=None):
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--workload", default="qwen3_235b_nvfp4", choices=sorted(WORKLOADS))
+    ap.add_argument("--workload", default="qwen3_480b_fp8", choices=sorted(WORKLOADS))
     ap.add_argument("--tokens", type=int, default=None, help="batch size (default per workload)")
     ap.add_argument("--experts", type=int, default=None,
                     help="expert count (default per workload); a smaller count keeps the "
@@ -86,6 +91,8 @@ def parse(argv=None):
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-energy", action="store_true")
+    ap.add_argument("--no-sweep", action="store_true",
+                    help="skip the batch sweep of the default run")
     return ap.parse_args(argv)
 
 
@@ -163,6 +170,13 @@ class ClockSampler:
             self.proc.wait(timeout=5)
         except subprocess.TimeoutExpired:
             self.proc.kill()
+        return self.summary(t0, t1)
+
+    def summary(self, t0=None, t1=None):
+        """Median SM clock, max clock, throttle reasons and median power of the
+        samples that arrived between host times t0 and t1."""
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
         sm, smax, reasons, watts = [], None, set(), []
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         for ts, ln in list(self.lines):
@@ -222,12 +236,26 @@ def zipf_bias(wl, seed, device):
 
 
 # ---------------------------------------------------------------- CPU oracle
-def _oracle_weights(w):
+def _oracle_weights(w, experts=None):
+    """The oracle's copy of w; with `experts`, only those experts are copied
+    (the others stay zero; numpy's zeros are not touched until written)."""
+    import numpy as np
+
     from oracle import oracle
-    return oracle.ExpertWeights(w.fmt, w.E, w.H, w.I, *[
-        None if t is None else t.detach().cpu().numpy()
-        for t in (w.w_gate, w.w_up, w.w_down, w.s_gate, w.s_up, w.s_down, w.ts_gate, w.ts_up,
-                  w.ts_down)])
+    ts = (w.w_gate, w.w_up, w.w_down, w.s_gate, w.s_up, w.s_down, w.ts_gate, w.ts_up, w.ts_down)
+    if experts is None:
+        return oracle.ExpertWeights(w.fmt, w.E, w.H, w.I, *[
+            None if t is None else t.detach().cpu().numpy() for t in ts])
+    out = []
+    for t in ts:
+        if t is None:
+            out.append(None)
+            continue
+        a = np.zeros(tuple(t.shape), dtype=t.cpu()[:0].numpy().dtype)
+        for e in experts:
+            a[int(e)] = t[int(e)].detach().cpu().numpy()
+        out.append(a)
+    return oracle.ExpertWeights(w.fmt, w.E, w.H, w.I, *out)
 
 
 class OracleSample:
@@ -255,22 +283,21 @@ class OracleSample:
         self.bias = None if b is None else b.numpy()
         xr = oracle.rmsnorm_bf16(self.xb) if self.prenorm else self.xb
         ids, _ = oracle.topk(oracle.router_logits(xr, self.wr, self.bias), k)
-        # calibrate on one token
-        if w is None:
-            w = synth.make_weights(fmt, E, H, I, seed=s0, experts=np.unique(ids[:1]))
-        self.ow = _oracle_weights(w)
+        # calibrate on one token; weights given (the device's): copy only the
+        # experts the sample routes to; else generate only those on the host
+        def weights_for(n_tok):
+            ex = np.unique(ids[:n_tok])
+            if w is not None:
+                return _oracle_weights(w, ex)
+            return _oracle_weights(synth.make_weights(fmt, E, H, I, seed=s0, experts=ex))
+        self.ow = weights_for(1)
         self.n = 1
         dt = self.run()
         n = max(1, min(T, int(budget_s / max(dt, 1e-3))))
         self.n = n
-        if n > 1 and not self._full(w, E):
-            w = synth.make_weights(fmt, E, H, I, seed=s0, experts=np.unique(ids[:n]))
-            self.ow = _oracle_weights(w)
+        if n > 1:
+            self.ow = weights_for(n)
         self.experts = int(np.unique(ids[:n]).size)
-
-    @staticmethod
-    def _full(w, E):
-        return bool((w.w_gate.reshape(E, -1)[:, :64] != 0).any(dim=1).all())
 
     def run(self):
         from oracle import oracle
@@ -391,6 +418,226 @@ def gateup_roofline(wl, fmt, T, k, H, I, gu_ms, gu_gbs, peaks, traffic):
             "hbm": {"achieved": gu_gbs, "peak": hbm, "unit": "GB/s", "frac": gu_gbs / hbm}}
 
 
+class Runner:
+    """One workload at one batch size on this GPU: the layers' weights, the
+    resident input batches, a workspace, and the timings of this file.
+
+    Steps rotate over distinct input batches, all resident before timing, when
+    one step touches less than four times L2: consecutive steps then route to
+    different experts and a step does not find the weights of the previous ones
+    in L2.  Steps are replayed from CUDA graphs of G steps (one rotation cycle,
+    at least eight layer calls); within a graph the layer calls follow one
+    another as in a decode loop and the host takes no decision between them."""
+
+    def __init__(self, wl, layers, bias, seed, rank, dev="cuda"):
+        import torch
+
+        from paper_2609_11133_gb300 import binding, synth
+        self.torch, self.binding = torch, binding
+        self.wl, self.layers, self.bias = wl, layers, bias
+        self.T, self.H, self.k, self.E, self.L = wl["T"], wl["H"], wl["k"], wl["E"], wl["layers"]
+        self.flags = MOE_FLAG_PRENORM_RMS if wl["prenorm"] else 0
+        T, H = self.T, self.H
+        self.dev = dev
+        x = synth.make_x(T, H, seed=seed + rank, device=dev)
+        # the residual stream of a stack: layer l reads cur and writes nxt
+        self.bufs = [torch.empty((T, H), dtype=torch.bfloat16, device=dev) for _ in range(2)]
+        self.ws = binding.alloc_workspace(binding.moe_workspace_size(layers[0][0], T, self.k))
+        self.stream = torch.cuda.current_stream()
+        w0 = layers[0][0]
+        self.gu_bytes, self.dn_bytes = expert_bytes(w0)
+        self.per_expert = w0.nbytes_expert()
+        self.router_bytes = self.E * H * 4
+        self.act_bytes = 2 * T * H * 2  # x in, out
+        n_active, self.ids, B = self.touched(x)
+        l2 = torch.cuda.get_device_properties(0).L2_cache_size
+        self.l2 = l2
+        self.n_rot = 1 if B >= 4 * l2 else min(16, math.ceil(4 * l2 / B))
+        self.xs = [x] + [synth.make_x(T, H, seed=seed + rank + 7919 * r, device=dev)
+                         for r in range(1, self.n_rot)]
+        if self.n_rot > 1:
+            rot = [self.touched(xr) for xr in self.xs]
+            n_active = [statistics.mean(r[0][l] for r in rot) for l in range(self.L)]
+            B = statistics.mean(r[2] for r in rot)
+        self.n_active, self.B = n_active, B
+        self.G = self.n_rot * max(1, math.ceil(8 / (self.n_rot * self.L)))
+
+    def io(self, l, x_in):
+        """(input, residual, output) of layer l."""
+        if self.L == 1:
+            return x_in, None, self.bufs[0]
+        cur = x_in if l == 0 else self.bufs[(l - 1) % 2]
+        return cur, cur, self.bufs[l % 2]
+
+    def run_layers(self, x_in, ev=None, ids=None):
+        b = self.binding
+        for l, (w, wr) in enumerate(self.layers):
+            xi, res, out = self.io(l, x_in)
+            if ev is None and ids is None:
+                b.moe_decode_layer(xi, wr, self.bias, w, self.k, out, self.ws, flags=self.flags,
+                                   residual=res)
+            else:
+                b.moe_decode_layer_ex(xi, wr, self.bias, w, self.k, out, self.ws,
+                                      flags=self.flags, residual=res,
+                                      events=None if ev is None else ev[l],
+                                      topk_ids_out=None if ids is None else ids[l])
+        return self.io(self.L - 1, x_in)[2]
+
+    def touched(self, x_in):
+        """Unique experts per layer of one batch, and the step's algorithmic bytes."""
+        torch = self.torch
+        ids = [torch.empty((self.T, self.k), dtype=torch.int32, device=self.dev)
+               for _ in range(self.L)]
+        self.run_layers(x_in, ids=ids)
+        torch.cuda.synchronize()
+        assert self.binding.moe_read_status(self.ws) == 0
+        n = [int(torch.unique(i).numel()) for i in ids]
+        return n, ids, sum(self.router_bytes + a * self.per_expert + self.act_bytes for a in n)
+
+    def capture(self, nsteps, body):
+        g = self.torch.cuda.CUDAGraph()
+        with self.torch.cuda.graph(g):
+            for s_ in range(nsteps):
+                body(s_ % self.n_rot)
+        return g
+
+    def graphs(self, steps, body=None):
+        body = body or (lambda r: self.run_layers(self.xs[r]))
+        g_full = self.capture(self.G, body)
+        g_rem = self.capture(steps % self.G, body) if steps % self.G else None
+        return g_full, g_rem
+
+    def timed(self, g_full, g_rem, steps, marks=None):
+        """Replays that run exactly `steps` steps; `marks` gets an event after
+        every full replay (the spread over repetitions)."""
+        for _ in range(steps // self.G):
+            g_full.replay()
+            if marks is not None:
+                marks.append(self.torch.cuda.Event(enable_timing=True))
+                marks[-1].record(self.stream)
+        if g_rem is not None:
+            g_rem.replay()
+
+    def warm(self, g_full, warmup):
+        for _ in range(max(3, warmup)):
+            self.run_layers(self.xs[0])
+        for _ in range(max(3, math.ceil(warmup / self.G))):
+            g_full.replay()
+        self.torch.cuda.synchronize()
+
+    def time_steps(self, g_full, g_rem, steps, world, marks=None):
+        """Device time of exactly `steps` steps (ms per step, max over ranks),
+        bracketed by a barrier and a synchronisation on both sides; host
+        times of the region."""
+        torch = self.torch
+        t_beg = torch.cuda.Event(enable_timing=True)
+        t_end = torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        barrier(world)
+        h_beg = time.perf_counter()
+        t_beg.record(self.stream)
+        self.timed(g_full, g_rem, steps, marks)
+        t_end.record(self.stream)
+        torch.cuda.synchronize()
+        h_end = time.perf_counter()
+        ms = t_beg.elapsed_time(t_end)
+        reps = None
+        if marks:
+            reps = [a.elapsed_time(b) / self.G for a, b in zip([t_beg] + marks[:-1], marks)]
+        return barrier_max(ms / steps, world), h_beg, h_end, reps
+
+    def energy(self, g_full, ms_step, local, seconds):
+        """J/token from the NVML energy counter over >= `seconds` of
+        back-to-back steps; (result, host end time)."""
+        torch = self.torch
+        nv = Nvml(local)
+        if not nv.ok:
+            return None, time.perf_counter()
+        n_rep = max(1, int(seconds / (ms_step * 1e-3 * self.G)))
+        torch.cuda.synchronize()
+        j0 = nv.energy_mj()
+        t0 = time.perf_counter()
+        for _ in range(n_rep):
+            g_full.replay()
+        torch.cuda.synchronize()
+        t1 = time.perf_counter()
+        j1 = nv.energy_mj()
+        return {"j_per_token": (j1 - j0) * 1e-3 / (n_rep * self.G * self.T),
+                "avg_w": (j1 - j0) * 1e-3 / (t1 - t0), "window_s": t1 - t0,
+                "source": "nvmlDeviceGetTotalEnergyConsumption"}, t1
+
+    def kernel_ms(self, n):
+        """Mean CUDA-event durations (ms per layer) of route (+ gather), gate/up
+        and SwiGLU + down + finalize, from eager calls with events between
+        the kernels on the launching stream."""
+        torch = self.torch
+        ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(self.L)]
+        kern = [[], [], []]
+        for i_ in range(n):
+            self.run_layers(self.xs[i_ % self.n_rot], ev=ev)
+            torch.cuda.synchronize()
+            for i in range(3):
+                kern[i].append(sum(ev[l][i].elapsed_time(ev[l][i + 1]) for l in range(self.L)))
+        return [statistics.mean(k_) / self.L for k_ in kern]
+
+    def hbm(self, ms_step, gu_ms, peaks):
+        hbm = float(peaks.get("hbm_gbs", 6800.0))
+        gu_alg = statistics.mean(self.n_active) * self.gu_bytes  # per launch
+        gu_gbs = gu_alg / (gu_ms * 1e-3) / 1e9
+        layer_gbs = self.B / (ms_step * 1e-3) / 1e9
+        return {"layer_gbs": layer_gbs, "layer_frac_of_measured": layer_gbs / hbm,
+                "layer_frac_of_8tbs": layer_gbs / 8000.0, "gateup_gbs": gu_gbs,
+                "gateup_frac_of_measured": gu_gbs / hbm, "gateup_frac_of_8tbs": gu_gbs / 8000.0}
+
+
+def load_peaks():
+    pp = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    return json.load(open(pp)) if os.path.exists(pp) else {}
+
+
+def make_layers(wl, seed, dev="cuda"):
+    from paper_2609_11133_gb300 import synth
+    out = []
+    for l in range(wl["layers"]):
+        sl = layer_seed(seed, l)
+        out.append((synth.make_weights(wl["fmt"], wl["E"], wl["H"], wl["I"], seed=sl, device=dev),
+                    synth.make_router(wl["E"], wl["H"], seed=sl, device=dev)))
+    return out
+
+
+# The sweep of the default run: (workload, batch sizes).  The 480B-shaped
+# layers reuse the headline's weights (same seed); only the router bias and
+# the batch differ.
+SWEEP = [("qwen3_235b_nvfp4", (1, 8, 32, 64)), ("qwen3_480b_fp8_zipf", (1, 8, 32, 128, 256))]
+SWEEP_TIMED_S = 0.25   # timed device work per sweep entry
+SWEEP_ENERGY_S = 1.0   # energy window per sweep entry
+
+
+def sweep_entry(run, peaks, clocks, local, no_energy):
+    """Time, HBM fractions, J/token and clocks of one sweep entry."""
+    g_full, _ = run.graphs(0)
+    run.warm(g_full, 3)
+    ms0, _, _, _ = run.time_steps(g_full, None, run.G, 1)
+    steps = max(50, run.G * math.ceil(SWEEP_TIMED_S / (ms0 * 1e-3) / run.G))
+    ms, h0, h1, _ = run.time_steps(g_full, None, steps, 1)
+    energy = None
+    if not no_energy:
+        energy, h1 = run.energy(g_full, ms, local, SWEEP_ENERGY_S)
+    rt, gu, dn = run.kernel_ms(20)
+    clk = clocks.summary(h0, h1)
+    e = {"tokens": run.T, "ms_per_step": ms, "tokens_per_s": run.T / (ms * 1e-3),
+         "steps": steps, "active_experts": statistics.mean(run.n_active),
+         "algorithmic_bytes_per_step": run.B,
+         "kernel_ms": {"route": rt, "gate_up": gu, "down": dn}}
+    e.update(run.hbm(ms, gu, peaks))
+    e["j_per_token"] = energy["j_per_token"] if energy else None
+    e["sm_mhz_median"] = clk.get("sm_mhz")
+    e["clock_reasons"] = clk.get("reasons")
+    if run.wl["zipf"]:
+        e["popularity"] = zipf_stats(run.ids[0].cpu().numpy(), run.E)
+    return e
+
+
 def run_ours(args):
     import numpy as np
     import torch
@@ -402,102 +649,17 @@ def run_ours(args):
         dist.init_process_group("nccl")
     else:
         torch.cuda.set_device(0)
-    from paper_2609_11133_gb300 import binding, synth
+    from paper_2609_11133_gb300 import binding
 
     wl = workload(args)
     fmt, H, E, k, I, T, L = (wl[n] for n in ("fmt", "H", "E", "k", "I", "T", "layers"))
-    flags = MOE_FLAG_PRENORM_RMS if wl["prenorm"] else 0
     dev = "cuda"
-    layers = []
-    for l in range(L):
-        sl = layer_seed(args.seed, l)
-        layers.append((synth.make_weights(fmt, E, H, I, seed=sl, device=dev),
-                       synth.make_router(E, H, seed=sl, device=dev)))
-    bias = zipf_bias(wl, args.seed, dev)
-    x = synth.make_x(T, H, seed=args.seed + rank, device=dev)
-    # the residual stream of a stack: layer l reads cur and writes nxt
-    bufs = [torch.empty((T, H), dtype=torch.bfloat16, device=dev) for _ in range(2)]
-    ws = binding.alloc_workspace(binding.moe_workspace_size(layers[0][0], T, k))
-    stream = torch.cuda.current_stream()
+    layers = make_layers(wl, args.seed, dev)
+    run = Runner(wl, layers, zipf_bias(wl, args.seed, dev), args.seed, rank, dev)
+    G, n_rot = run.G, run.n_rot
 
-    def io(l, x_in):
-        """(input, residual, output) of layer l."""
-        if L == 1:
-            return x_in, None, bufs[0]
-        cur = x_in if l == 0 else bufs[(l - 1) % 2]
-        return cur, cur, bufs[l % 2]
-
-    def run_layers(x_in, ev=None, ids=None):
-        for l, (w, wr) in enumerate(layers):
-            xi, res, out = io(l, x_in)
-            if ev is None and ids is None:
-                binding.moe_decode_layer(xi, wr, bias, w, k, out, ws, flags=flags, residual=res)
-            else:
-                binding.moe_decode_layer_ex(xi, wr, bias, w, k, out, ws, flags=flags,
-                                            residual=res, events=None if ev is None else ev[l],
-                                            topk_ids_out=None if ids is None else ids[l])
-        return io(L - 1, x_in)[2]
-
-    def touched(x_in):
-        """Unique experts per layer of one batch, and the step's algorithmic bytes."""
-        ids = [torch.empty((T, k), dtype=torch.int32, device=dev) for _ in range(L)]
-        run_layers(x_in, ids=ids)
-        torch.cuda.synchronize()
-        assert binding.moe_read_status(ws) == 0
-        n = [int(torch.unique(i).numel()) for i in ids]
-        return n, ids, sum(router_bytes + a * per_expert + act_bytes for a in n)
-
-    w0 = layers[0][0]
-    per_expert = w0.nbytes_expert()
-    gu_bytes, dn_bytes = expert_bytes(w0)
-    router_bytes = E * H * 4
-    act_bytes = 2 * T * H * 2  # x in, out
-    n_active, ids, B = touched(x)
-
-    # Steps rotate over distinct input batches, all resident before timing,
-    # when one step touches less than four times L2: consecutive steps then
-    # route to different experts and a step does not find the weights of the
-    # previous ones in L2.
-    l2 = torch.cuda.get_device_properties(0).L2_cache_size
-    n_rot = 1 if B >= 4 * l2 else min(16, math.ceil(4 * l2 / B))
-    xs = [x] + [synth.make_x(T, H, seed=args.seed + rank + 7919 * r, device=dev)
-                for r in range(1, n_rot)]
-    if n_rot > 1:
-        rot = [touched(xr) for xr in xs]
-        n_active = [statistics.mean(r[0][l] for r in rot) for l in range(L)]
-        B = statistics.mean(r[2] for r in rot)
-    # Steps per CUDA graph: one rotation cycle, at least eight layer calls.
-    # Within a graph the layer calls follow one another as in a decode loop;
-    # the host takes no decision between them.
-    G = n_rot * max(1, math.ceil(8 / (n_rot * L)))
-
-    def capture(nsteps, body):
-        g = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g):
-            for s_ in range(nsteps):
-                body(s_ % n_rot)
-        return g
-
-    def timed(g_full, g_rem, steps, marks=None):
-        """Replays that run exactly `steps` steps; `marks` gets an event after
-        every full replay (the spread over repetitions)."""
-        for _ in range(steps // G):
-            g_full.replay()
-            if marks is not None:
-                marks.append(torch.cuda.Event(enable_timing=True))
-                marks[-1].record(stream)
-        if g_rem is not None:
-            g_rem.replay()
-
-    for _ in range(max(3, args.warmup)):
-        run_layers(x)
-    torch.cuda.synchronize()
-
-    g_step = capture(G, lambda r: run_layers(xs[r]))
-    g_rem = capture(args.steps % G, lambda r: run_layers(xs[r])) if args.steps % G else None
-    for _ in range(max(3, math.ceil(args.warmup / G))):
-        g_step.replay()
-    torch.cuda.synchronize()
+    g_step, g_rem = run.graphs(args.steps)
+    run.warm(g_step, args.warmup)
     barrier(world)
 
     # clock sampler: started before the timed region; the replays below keep
@@ -511,118 +673,68 @@ def run_ours(args):
         torch.cuda.synchronize()
 
     # ---- timed region (device time, CUDA events on the launching stream)
-    t_beg = torch.cuda.Event(enable_timing=True)
-    t_end = torch.cuda.Event(enable_timing=True)
-    torch.cuda.synchronize()
-    barrier(world)
-    h_beg = time.perf_counter()
-    t_beg.record(stream)
     marks = []
-    timed(g_step, g_rem, args.steps, marks)
-    t_end.record(stream)
-    torch.cuda.synchronize()
-    h_end = time.perf_counter()
-    ms_total = t_beg.elapsed_time(t_end)
-    ms_step = barrier_max(ms_total / args.steps, world)
+    ms_step, h_beg, h_end, reps = run.time_steps(g_step, g_rem, args.steps, world, marks)
     tok_s = job_throughput(ms_step, T, world)
-    # per-step time of each repetition (one graph replay of G steps)
-    reps = [a.elapsed_time(b) / G for a, b in zip([t_beg] + marks[:-1], marks)]
     repeats = None
     if reps:
         repeats = {"n": len(reps), "steps_each": G, "median_ms": float(np.median(reps)),
                    "p10_ms": float(np.percentile(reps, 10)),
                    "p90_ms": float(np.percentile(reps, 90))}
 
+    # ---- energy per token (NVML counter over >= 2 s of back-to-back steps)
+    energy = None
+    if not args.no_energy:
+        energy, h_end = run.energy(g_step, ms_step, local, 2.0)
+    clk = clocks.summary(h_beg, h_end)
+    clk["window"] = "timed region" + (" + energy window (same steps replayed)" if energy else "")
+
     # single-call latency: one step, eager (host launches included) and as a
     # one-step graph, each timed alone on an idle GPU
     lat_eager, lat_graph = [], []
-    g_one = capture(1, lambda r: run_layers(xs[r]))
+    g_one = run.capture(1, lambda r: run.run_layers(run.xs[r]))
     for i_ in range(12):
         a_, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         torch.cuda.synchronize()
-        a_.record(stream)
+        a_.record(run.stream)
         if i_ % 2:
             g_one.replay()
         else:
-            run_layers(xs[0])
-        b_.record(stream)
+            run.run_layers(run.xs[0])
+        b_.record(run.stream)
         torch.cuda.synchronize()
         (lat_graph if i_ % 2 else lat_eager).append(a_.elapsed_time(b_) * 1e3)
     latency = {"eager_us": statistics.median(lat_eager[1:]),
                "graph_us": statistics.median(lat_graph[1:]),
                "per": "layer call" if L == 1 else f"{L}-layer step"}
 
-    # ---- energy per token (NVML counter over >= 2 s of back-to-back steps)
-    energy = None
-    if not args.no_energy:
-        nv = Nvml(local)
-        if nv.ok:
-            n_rep = max(1, int(2.0 / (ms_step * 1e-3 * G)))
-            torch.cuda.synchronize()
-            j0 = nv.energy_mj()
-            t0 = time.perf_counter()
-            for _ in range(n_rep):
-                g_step.replay()
-            torch.cuda.synchronize()
-            h_end = time.perf_counter()
-            dt = h_end - t0
-            j1 = nv.energy_mj()
-            energy = {"j_per_token": (j1 - j0) * 1e-3 / (n_rep * G * T),
-                      "avg_w": (j1 - j0) * 1e-3 / dt,
-                      "window_s": dt, "source": "nvmlDeviceGetTotalEnergyConsumption"}
-    clk = clocks.stop(h_beg, h_end)
-    clk["window"] = "timed region" + (" + energy window (same steps replayed)" if energy else "")
-
     # per-kernel durations: eager calls with events between the kernels
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(L)]
-    kern = [[], [], []]
-    for i_ in range(max(1, min(args.steps, 20 if L == 1 else 2))):
-        run_layers(xs[i_ % n_rot], ev=ev)
-        torch.cuda.synchronize()
-        for i in range(3):
-            kern[i].append(sum(ev[l][i].elapsed_time(ev[l][i + 1]) for l in range(L)))
+    rt_ms, gu_ms, dn_ms = run.kernel_ms(max(1, min(args.steps, 20 if L == 1 else 2)))
 
     # ---- end to end through the public API with host buffers: every step
     # copies its input from pinned host memory, runs, and copies its output
     # back (the same steps per graph and the same input rotation)
     x_host = [torch.empty((T, H), dtype=torch.bfloat16, pin_memory=True) for _ in range(n_rot)]
-    for xh, xr in zip(x_host, xs):
+    for xh, xr in zip(x_host, run.xs):
         xh.copy_(xr.cpu())
     out_host = torch.empty((T, H), dtype=torch.bfloat16, pin_memory=True)
-    x_dev = torch.empty_like(x)
+    x_dev = torch.empty_like(run.xs[0])
 
     def e2e_step(r):
         x_dev.copy_(x_host[r], non_blocking=True)
-        o = run_layers(x_dev)
+        o = run.run_layers(x_dev)
         out_host.copy_(o, non_blocking=True)
 
-    g_e2e = capture(G, e2e_step)
-    g_e2e_rem = capture(args.steps % G, e2e_step) if args.steps % G else None
+    g_e2e, g_e2e_rem = run.graphs(args.steps, e2e_step)
     for _ in range(3):
         g_e2e.replay()
     torch.cuda.synchronize()
-    barrier(world)
-    e0 = torch.cuda.Event(enable_timing=True)
-    e1 = torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    timed(g_e2e, g_e2e_rem, args.steps)
-    e1.record(stream)
-    torch.cuda.synchronize()
-    ms_e2e = barrier_max(e0.elapsed_time(e1) / args.steps, world)
+    ms_e2e, _, _, _ = run.time_steps(g_e2e, g_e2e_rem, args.steps, world)
     assert torch.isfinite(out_host.float()).all()
 
     # ---- roofline of the dominant kernel (gate/up) and of the whole step
-    peaks = {}
-    pp = os.path.join(ROOT, "MEASURED_PEAKS.json")
-    if os.path.exists(pp):
-        peaks = json.load(open(pp))
-    hbm = float(peaks.get("hbm_gbs", 6800.0))
-    gu_ms = statistics.mean(kern[1]) / L
-    dn_ms = statistics.mean(kern[2]) / L
-    rt_ms = statistics.mean(kern[0]) / L
-    gu_alg = statistics.mean(n_active) * gu_bytes  # per launch
-    gu_gbs = gu_alg / (gu_ms * 1e-3) / 1e9
-    layer_gbs = B / (ms_step * 1e-3) / 1e9
+    peaks = load_peaks()
+    hb = run.hbm(ms_step, gu_ms, peaks)
     # DRAM bytes of one gate/up launch from a committed ncu capture, valid only
     # while the kernel sources are the ones that capture was taken on
     traffic = None
@@ -632,13 +744,15 @@ def run_ours(args):
         if tj and kernel_sources_sha256() == tj.get("kernel_sources_sha256"):
             traffic = tj.get("gateup_dram_bytes")
 
+    B = run.B
     cfg = {"workload": wl["name"], "H": H, "E": E, "k": k, "I": I,
            "tokens": T, "format": "nvfp4" if fmt == 2 else "fp8_block128",
-           "active_experts": n_active[0] if L == 1 else statistics.mean(n_active),
+           "active_experts": run.n_active[0] if L == 1 else statistics.mean(run.n_active),
            "l2": (f"inputs larger than L2: {B / 1e9:.2f} GB of weights touched per step"
                   if n_rot == 1 else
                   f"{n_rot} resident input batches rotated step by step: {B / 1e9:.3f} GB "
-                  f"touched per step, {n_rot * B / 1e9:.2f} GB per rotation (L2 {l2 / 1e6:.0f} MB)"),
+                  f"touched per step, {n_rot * B / 1e9:.2f} GB per rotation "
+                  f"(L2 {run.l2 / 1e6:.0f} MB)"),
            "steps_per_graph": G,
            "arithmetic": ("e2m1 x e2m1 block-scaled MMA (ue4m3 per 16), activations as 4 nvfp4 "
                           "terms, fp32 accumulate" if fmt == 2 else
@@ -650,8 +764,8 @@ def run_ours(args):
                    weights_gb=round(sum(w.nbytes_expert() * E for w, _ in layers) / 1e9, 1))
     if wl["zipf"]:
         cfg["router_bias"] = f"zipf s={wl['zipf']}"
-        cfg["popularity"] = zipf_stats(ids[0].cpu().numpy(), E)
-    roofline = gateup_roofline(wl, fmt, T, k, H, I, gu_ms, gu_gbs, peaks, traffic)
+        cfg["popularity"] = zipf_stats(run.ids[0].cpu().numpy(), E)
+    roofline = gateup_roofline(wl, fmt, T, k, H, I, gu_ms, hb["gateup_gbs"], peaks, traffic)
     res = {
         "metric": metric_name(wl),
         "value": tok_s,
@@ -666,9 +780,10 @@ def run_ours(args):
         "dtype": "nvfp4" if fmt == 2 else "fp8_e4m3",
         "data": "synthetic (seeded N(0,1) activations, N(0,0.02) weights quantised)",
         "config": cfg,
-        "hbm_gbs": layer_gbs,
-        "hbm_frac_of_measured": layer_gbs / hbm,
-        "hbm_frac_of_8tbs": layer_gbs / 8000.0,
+        "hbm_gbs": hb["layer_gbs"],
+        "hbm_frac_of_measured": hb["layer_frac_of_measured"],
+        "hbm_frac_of_8tbs": hb["layer_frac_of_8tbs"],
+        "gateup_frac_of_8tbs": hb["gateup_frac_of_8tbs"],
         "algorithmic_bytes_per_step": B,
         "kernel_ms": {"route": rt_ms, "gate_up": gu_ms, "down": dn_ms,
                       "per": "layer" if L == 1 else f"layer, mean of {L}"},
@@ -684,8 +799,31 @@ def run_ours(args):
     }
     if energy:
         res["j_per_token"] = energy["j_per_token"]
+
+    # ---- the batch sweep (default run, one GPU): other batch sizes and the
+    # other served model's layer, each measured over its own window
+    if world == 1 and not args.no_sweep and args.workload == "qwen3_480b_fp8" \
+            and args.tokens is None and args.experts is None:
+        sweep = {}
+        for name, batches in SWEEP:
+            base = dict(layers=1, zipf=None, prenorm=False, prefill=False)
+            base.update(WORKLOADS[name])
+            lay = layers if base["fmt"] == fmt and base["E"] == E and base["H"] == H \
+                and base["I"] == I else make_layers(base, args.seed, dev)
+            bias = zipf_bias(base, args.seed, dev)
+            for t_ in batches:
+                wl_t = dict(base, T=t_, name=f"{name}_T{t_}")
+                r_t = Runner(wl_t, lay, bias, args.seed, rank, dev)
+                sweep[wl_t["name"]] = sweep_entry(r_t, peaks, clocks, local, args.no_energy)
+                del r_t
+            if lay is not layers:
+                del lay
+                torch.cuda.empty_cache()
+        res["sweep"] = sweep
+    clocks.stop()
+
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        res["cpu_baseline"] = cpu_oracle_sample(wl, args.seed, w=w0)  # layer 0's weights
+        res["cpu_baseline"] = cpu_oracle_sample(wl, args.seed, w=layers[0][0])  # layer 0
     if rank == 0:
         print(json.dumps(res))
     if world > 1:
@@ -709,11 +847,14 @@ def run_reference(args):
     v = s.n / (dt * L)
     res = {"metric": metric_name(wl),
            "value": v, "unit": "tokens/s", "n_gpus": world,
-           "steps": steps, "warmup": warm, "ms_per_step": dt * L * 1e3 * T / s.n,
+           "steps": steps, "warmup": warm, "ms_per_step": dt * L * 1e3,
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
            "data": "synthetic", "impl": "reference",
            "config": {"workload": wl["name"], "H": wl["H"], "E": wl["E"],
-                      "k": wl["k"], "I": wl["I"], "tokens": T},
+                      "k": wl["k"], "I": wl["I"], "tokens": T,
+                      "step": f"the first {s.n} of the batch's {T} tokens (a bounded sample); "
+                              f"ms_per_step is the time of that sample"
+                              + (f", layer 0 timed and counted {L} times" if L > 1 else "")},
            "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": s.cores, "kind": "oracle",
                             "sample": f"first {s.n} of {T} tokens per step ({s.experts} experts)"
                                       + (f", layer 0 of {L}" if L > 1 else "")},

@@ -230,18 +230,31 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
  *   Arguments as moe_decode_layer, minus ws / ws_bytes.
  *   Scratch: a 16 MiB device array inside libmoe.so; every GPU that loads the
  *     library holds it until the process exits.  Shapes whose
- *     moe_workspace_size() exceeds 16 MiB return MOE_ERR_WORKSPACE_TOO_SMALL
- *     (e.g. the 235B-shaped NVFP4 layer fits up to T = 110 tokens).
- *   The first call on a device looks up the array's device address; make
- *     that first call before capturing the stream into a CUDA graph.
- *   Every call shares the one array and clears its control words itself;
- *     calls that overlap on the GPU (two streams, or two host threads) race
- *     and must be serialised by the caller.  Device-side error status is not
- *     reported by this call.
+ *     moe_workspace_size() exceeds 16 MiB return MOE_ERR_WORKSPACE_TOO_SMALL:
+ *     the 235B-shaped NVFP4 layer (H=4096, E=128, k=8, I=1536) fits up to
+ *     T = 74 tokens, the 480B-shaped FP8 layer (H=6144, E=160, k=8, I=2560)
+ *     up to T = 64.
+ *   The first call on a device looks up the array's device address and
+ *     clears the array's status word; make that first call before capturing
+ *     the stream into a CUDA graph.  A lookup that fails returns MOE_ERR_CUDA
+ *     and is tried again by the next call.
+ *   Every call shares the one array and clears its counters itself; calls
+ *     that overlap on the GPU (two streams, or two host threads) race and must
+ *     be serialised by the caller.
+ *   Device-side errors (an expired bounded wait) are recorded in the array's
+ *     status word; read them with moe_noalloc_read_status().
  *   Allocates nothing: no cudaMalloc, no cudaFree. */
 int moe_decode_layer_noalloc(const void* x, const float* router_w, const float* router_bias,
                              const moe_expert_weights_t* w, int T, int k, int flags,
                              const void* residual, void* out, void* stream);
+
+/* The device status word of moe_decode_layer_noalloc's array on the current
+ * device, as moe_read_status does for a workspace: *status (host pointer)
+ * gets MOE_OK or the code of the first device-side error of any
+ * moe_decode_layer_noalloc call since the last read, and the word is
+ * cleared.  Synchronises `stream`.  Allocates nothing.  The paper has no
+ * counterpart of this call. */
+int moe_noalloc_read_status(int* status, void* stream);
 
 #ifdef __cplusplus
 }

@@ -69,6 +69,7 @@ _SIGS = {
                          _SZ, _P],
     "moe_decode_layer_noalloc": [_P, _P, _P, ctypes.POINTER(ExpertWeightsC), _I, _I, _I, _P, _P,
                                  _P],
+    "moe_noalloc_read_status": [ctypes.POINTER(_I), _P],
     "moe_decode_layer_ex": [_P, _P, _P, ctypes.POINTER(ExpertWeightsC), _I, _I, _I, _P, _P, _P,
                             _SZ, _P, _P, _P, ctypes.POINTER(_P), _P],
 }
@@ -251,3 +252,11 @@ def moe_decode_layer_noalloc(x, router_w, router_bias, w, k: int, out, flags: in
                                            ctypes.byref(c), T, k, flags, _ptr(residual),
                                            _ptr(out), _stream(stream)),
            "moe_decode_layer_noalloc")
+
+
+def moe_noalloc_read_status(stream=None) -> int:
+    """Read and clear the device status word of moe_decode_layer_noalloc's array."""
+    st = _I(0)
+    _check(load().moe_noalloc_read_status(ctypes.byref(st), _stream(stream)),
+           "moe_noalloc_read_status")
+    return st.value

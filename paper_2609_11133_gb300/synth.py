@@ -130,6 +130,13 @@ class LayerWeights:
         return [t for t in (self.w_gate, self.w_up, self.w_down, self.s_gate, self.s_up,
                             self.s_down, self.ts_gate, self.ts_up, self.ts_down) if t is not None]
 
+    def to(self, device) -> "LayerWeights":
+        """A copy with every tensor on `device` (one copy per tensor)."""
+        mv = lambda t: None if t is None else t.to(device)
+        return LayerWeights(self.fmt, self.E, self.H, self.I, mv(self.w_gate), mv(self.w_up),
+                            mv(self.w_down), mv(self.s_gate), mv(self.s_up), mv(self.s_down),
+                            mv(self.ts_gate), mv(self.ts_up), mv(self.ts_down))
+
 
 def make_weights(fmt: int, E: int, H: int, I: int, seed: int = 0, device="cpu",
                  std: float = 0.02, experts=None) -> LayerWeights:

@@ -8,10 +8,21 @@ PEAKS = {"hbm_gbs": 6790.3, "bf16_tflops": 1904.5, "bf16_tflops_sustained": 1717
 
 
 def test_default_workload_is_the_headline():
+    """The 480B-shaped FP8 layer at 64 tokens: the largest single-GPU decode
+    layer of the two served models."""
     wl = bench.workload(bench.parse([]))
     assert (wl["name"], wl["fmt"], wl["H"], wl["E"], wl["k"], wl["I"], wl["T"]) == \
-        ("qwen3_235b_nvfp4_T64", 2, 4096, 128, 8, 1536, 64)
+        ("qwen3_480b_fp8_T64", 1, 6144, 160, 8, 2560, 64)
     assert not wl["prefill"] and wl["layers"] == 1
+
+
+def test_sweep_covers_both_served_models_at_small_batches():
+    names = {n for n, _ in bench.SWEEP}
+    assert names == {"qwen3_235b_nvfp4", "qwen3_480b_fp8_zipf"}
+    batches = dict(bench.SWEEP)
+    assert set(batches["qwen3_235b_nvfp4"]) == {1, 8, 32, 64}
+    assert {1, 8, 32}.issubset(batches["qwen3_480b_fp8_zipf"])
+    assert not bench.parse([]).no_sweep and bench.parse(["--no-sweep"]).no_sweep
 
 
 def test_decode_roofline_is_hbm():

@@ -23,14 +23,17 @@ def test_qwen3_235b_nvfp4_layer(T):
     c.check_output()
 
 
-def test_qwen3_235b_nvfp4_t64_sampled_tokens():
+def test_qwen3_235b_nvfp4_t64_full_batch():
+    """Every token of the 235B-shaped NVFP4 layer at T=64, each row also
+    within 2e-2 of its own maximum."""
     c = Case(FP4, T=64, H=4096, E=128, k=8, I=1536, seed=1).run()
-    c.check_output(tokens=[0, 17, 33, 63])
+    c.check_output(row_tol=2e-2)
 
 
-def test_qwen3_480b_fp8_t64_sampled_tokens():
+def test_qwen3_480b_fp8_t64_full_batch():
+    """Every token of the 480B-shaped FP8 layer at T=64 (the bench's layer)."""
     c = Case(FP8, T=64, H=6144, E=160, k=8, I=2560, seed=0).run()
-    c.check_output(tokens=[0, 31, 63])
+    c.check_output(row_tol=2e-2)
 
 
 @pytest.mark.parametrize("fmt,T,E,k", [(FP8, 13, 16, 4), (FP4, 37, 12, 3), (FP8, 3, 5, 5),
