@@ -26,10 +26,12 @@ on synthetic seeded inputs.  Workloads:
 The metric is decode tokens/s; achieved HBM GB/s, the roofline fraction of
 the dominant kernel (gate/up) and J/token (NVML energy counter) are reported
 beside it.  The default run (N=1) adds a "sweep" key: the 235B-shaped NVFP4
-layer at T = 1, 8, 32, 64 and the 480B-shaped FP8 layer with Zipf-skewed
-routing at T = 1, 8, 32, 128, 256, each with its time per step, layer and
-gate/up HBM fractions against the measured copy rate and 8 TB/s, J/token and
-the SM clock over its own window (--no-sweep skips it).  Under torchrun each rank runs an independent replica on its own
+layer at T = 1, 8, 32, 64, the 480B-shaped FP8 layer with Zipf-skewed
+routing at T = 1, 8, 32, 128, 256 and the 235B-shaped layer on a
+prefill-shaped batch of 2048 tokens (with its gate/up tensor-core fraction),
+each with its time per step, layer and gate/up HBM fractions against the
+measured copy rate and 8 TB/s, J/token and the SM clock over its own window
+(--no-sweep skips it).  Under torchrun each rank runs an independent replica on its own
 GPU (the layer does not shard across GPUs); the timed region is bracketed by
 a barrier and the slowest rank's time is reported.
 
@@ -608,7 +610,8 @@ def make_layers(wl, seed, dev="cuda"):
 # The sweep of the default run: (workload, batch sizes).  The 480B-shaped
 # layers reuse the headline's weights (same seed); only the router bias and
 # the batch differ.
-SWEEP = [("qwen3_235b_nvfp4", (1, 8, 32, 64)), ("qwen3_480b_fp8_zipf", (1, 8, 32, 128, 256))]
+SWEEP = [("qwen3_235b_nvfp4", (1, 8, 32, 64)), ("qwen3_480b_fp8_zipf", (1, 8, 32, 128, 256)),
+         ("qwen3_235b_nvfp4_prefill", (2048,))]
 SWEEP_TIMED_S = 0.25   # timed device work per sweep entry
 SWEEP_ENERGY_S = 1.0   # energy window per sweep entry
 
@@ -630,6 +633,12 @@ def sweep_entry(run, peaks, clocks, local, no_energy):
          "algorithmic_bytes_per_step": run.B,
          "kernel_ms": {"route": rt, "gate_up": gu, "down": dn}}
     e.update(run.hbm(ms, gu, peaks))
+    if run.wl["prefill"]:  # the tensor-core roofline of the gate/up kernel
+        wl = run.wl
+        rf = gateup_roofline(wl, wl["fmt"], run.T, run.k, run.H, wl["I"], gu,
+                             e["gateup_gbs"], peaks, None)
+        e["gateup_tensor"] = {k_: rf[k_] for k_ in ("achieved", "peak", "unit", "frac",
+                                                    "peak_source")}
     e["j_per_token"] = energy["j_per_token"] if energy else None
     e["sm_mhz_median"] = clk.get("sm_mhz")
     e["clock_reasons"] = clk.get("reasons")

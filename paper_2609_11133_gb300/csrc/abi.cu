@@ -100,6 +100,24 @@ bool map_sf(CUtensorMap* m, const void* sf, int E, int N, int K) {
                 (uint64_t)(K / 16), 16, kRowsHalf, CU_TENSOR_MAP_SWIZZLE_NONE);
 }
 
+// Activation-term arrays [rows, 4 terms, row_bytes] as a 3-D map whose box is
+// the first kPfTerms terms of kPfTok rows: the prefill engine's B operand
+// (codes, 128 bytes of K per row, 128B swizzle) and its scales (16 bytes per
+// row, no swizzle); B row 3j + t = term t of row j.
+bool map_terms3(CUtensorMap* m, const void* base, int row_bytes, int rows, bool codes) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[3] = {(cuuint64_t)row_bytes, (cuuint64_t)kTerms, (cuuint64_t)rows};
+  cuuint64_t strides[2] = {(cuuint64_t)row_bytes, (cuuint64_t)row_bytes * kTerms};
+  cuuint32_t box[3] = {codes ? (cuuint32_t)kRowBytes : 16u, (cuuint32_t)kPfTerms,
+                       (cuuint32_t)kPfTok};
+  cuuint32_t es[3] = {1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, const_cast<void*>(base), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE,
+            codes ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
 // Expert engines: the block-scaled tcgen05 engine (ffn_bs.cuh) for NVFP4 and
@@ -150,6 +168,17 @@ int route_epb(int T, int E, int sms) {
   if (T <= 16) return 1;
   const int chunks = (T + kRouteTok - 1) / kRouteTok;
   return (long long)((E + 3) / 4) * chunks > 2LL * sms ? 8 : 4;
+}
+
+// Prefill-shaped NVFP4 batches run on the prefill engine (ffn_pf.cuh);
+// MOE_PF=0 keeps them on the decode engine (for comparisons).
+bool use_prefill(int T, int k, int E, int eng) {
+  static int off = -1;
+  if (off < 0) {
+    const char* s = std::getenv("MOE_PF");
+    off = (s && std::strcmp(s, "0") == 0) ? 1 : 0;
+  }
+  return !off && eng == kEngBs && prefill_shape(T, k, E, act_for(MOE_FMT_NVFP4, eng));
 }
 
 // ------------------------------------------------------------------ validation
@@ -322,6 +351,67 @@ int run_experts(const ExpertRun& r, cudaStream_t st, cudaEvent_t ev_mid) {
   if (err != cudaSuccess) return MOE_ERR_CUDA;
   if (r.fused) err = launch_finalize(r.sms, p2, st);
   return err == cudaSuccess ? MOE_OK : MOE_ERR_CUDA;
+}
+
+// The expert steps of a prefill-shaped NVFP4 batch: gate/up on the prefill
+// engine into the fp32 gate|up rows, SwiGLU into activation terms, down on
+// the prefill engine into each assignment's row of y_perm, and the combine
+// (gates, residual, bf16), which also zeroes the per-expert counters.
+int run_prefill(const moe_expert_weights_t* w, int T, int k, int sms, void* ws,
+                const WsLayout& L, const float* gates, const void* residual, void* out,
+                int test_stall, cudaEvent_t ev_mid, cudaStream_t st) {
+  const int E = w->E, H = w->H, I = w->I;
+  FfnMaps m1{}, m2{};
+  bool ok = map_codes(&m1.a0, w->w_gate, E, I, H / 2) && map_codes(&m1.a1, w->w_up, E, I, H / 2) &&
+            map_sf(&m1.s0, w->s_gate, E, I, H) && map_sf(&m1.s1, w->s_up, E, I, H) &&
+            map_terms3(&m1.b, ws_ptr<uint8_t>(ws, L.xg), H / 2, T * k, true) &&
+            map_terms3(&m1.sb, ws_ptr<uint8_t>(ws, L.xgsf), H / 16, T * k, false) &&
+            map_codes(&m2.a0, w->w_down, E, H, I / 2) && map_sf(&m2.s0, w->s_down, E, H, I) &&
+            map_terms3(&m2.b, ws_ptr<uint8_t>(ws, L.hq), I / 2, T * k, true) &&
+            map_terms3(&m2.sb, ws_ptr<uint8_t>(ws, L.hsf), I / 16, T * k, false);
+  if (!ok) return MOE_ERR_CUDA;
+  m2.a1 = m2.a0;
+  m2.s1 = m2.s0;
+  FfnParams p{};
+  p.T = T;
+  p.k = k;
+  p.E = E;
+  p.H = H;
+  p.I = I;
+  p.counts = ws_ptr<int>(ws, L.acnt);
+  p.sorted = ws_ptr<int>(ws, L.alist);
+  p.list_T = 1;
+  p.b_compact = 1;
+  p.gates = gates;
+  p.status = ws_ptr<uint32_t>(ws, L.status);
+  p.units = ws_ptr<uint32_t>(ws, L.units);
+  p.wait_ns = wait_limit_ns();
+  FfnParams p1 = p;
+  p1.phase = 1;
+  p1.ts0 = w->ts_gate;
+  p1.ts1 = w->ts_up;
+  p1.xinv = ws_ptr<float>(ws, L.xinv);
+  p1.gu = ws_ptr<float>(ws, L.gu);
+  p1.bsf = ws_ptr<uint8_t>(ws, L.xgsf);
+  p1.hq = ws_ptr<uint8_t>(ws, L.hq);
+  p1.hsf = ws_ptr<uint8_t>(ws, L.hsf);
+  p1.hinv = ws_ptr<float>(ws, L.hinv);
+  p1.test_stall = test_stall;
+  FfnParams p2 = p;
+  p2.phase = 2;
+  p2.ts0 = w->ts_down;
+  p2.ts1 = w->ts_down;
+  p2.xinv = ws_ptr<float>(ws, L.hinv);
+  p2.y_perm = ws_ptr<float>(ws, L.yperm);
+  p2.bsf = ws_ptr<uint8_t>(ws, L.hsf);
+  if (launch_ffn_pf(sms, m1, p1, st) != cudaSuccess) return MOE_ERR_CUDA;
+  if (ev_mid && cudaEventRecord(ev_mid, st) != cudaSuccess) return MOE_ERR_CUDA;
+  if (launch_swiglu_terms(T * k, sms, p1, st) != cudaSuccess) return MOE_ERR_CUDA;
+  if (launch_ffn_pf(sms, m2, p2, st) != cudaSuccess) return MOE_ERR_CUDA;
+  CombineParams c{p2.y_perm, gates, ws_ptr<int>(ws, L.inv), T, k, H,
+                  static_cast<const __nv_bfloat16*>(residual), static_cast<__nv_bfloat16*>(out),
+                  ws_ptr<unsigned>(ws, L.acnt), E};
+  return launch_combine(c, st) == cudaSuccess ? MOE_OK : MOE_ERR_CUDA;
 }
 
 }  // namespace
@@ -583,6 +673,7 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
     for (int i = 0; i < 4; ++i) ev[i] = static_cast<cudaEvent_t>(events[i]);
   const int eng = engine_for(w->fmt);
   const int nt = nt_for(T, eng);
+  const bool pf = use_prefill(T, k, E, eng);
 
   RouteParams p{};
   p.x = static_cast<const __nv_bfloat16*>(x);
@@ -608,10 +699,12 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
   p.xq = ws_ptr<uint8_t>(ws, L.xq);
   p.xsf = ws_ptr<uint8_t>(ws, L.xsf);
   p.xinv = ws_ptr<float>(ws, L.xinv);
+  // the decode engine adds its partial sums into zeroed accumulators; the
+  // prefill engine stores complete sums and needs none
   p.zero_a = ws_ptr<float4>(ws, L.gu);
-  p.zero_a_n4 = (size_t)T * k * 2 * I / 4;
+  p.zero_a_n4 = pf ? 0 : (size_t)T * k * 2 * I / 4;
   p.zero_b = ws_ptr<float4>(ws, L.oacc);
-  p.zero_b_n4 = (size_t)T * H / 4;
+  p.zero_b_n4 = pf ? 0 : (size_t)T * H / 4;
   p.acnt = ws_ptr<unsigned>(ws, L.acnt);
   p.alist = ws_ptr<int>(ws, L.alist);
   if (ev[0] && cudaEventRecord(ev[0], st) != cudaSuccess) return MOE_ERR_CUDA;
@@ -632,9 +725,17 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
     g.terms = fp4 ? kTerms : kF8Terms;
     g.qrow = fp4 ? H / 2 : H;
     g.sfrow = H / 16;
+    g.inv = pf ? ws_ptr<int>(ws, L.inv) : nullptr;
     if (launch_gather(g, st) != cudaSuccess) return MOE_ERR_CUDA;
   }
   if (ev[1] && cudaEventRecord(ev[1], st) != cudaSuccess) return MOE_ERR_CUDA;
+  if (pf) {
+    rc = run_prefill(w, T, k, sms, ws, L, p.gates, residual, out,
+                     (flags & kFlagTestStall) ? 1 : 0, ev[2], st);
+    if (rc) return rc;
+    if (ev[3] && cudaEventRecord(ev[3], st) != cudaSuccess) return MOE_ERR_CUDA;
+    return MOE_OK;
+  }
 
   ExpertRun r{};
   r.w = w;

@@ -69,6 +69,10 @@ struct WsLayout {
   // (rows as h: terms per assignment), and their NVFP4 scales
   size_t xg;
   size_t xgsf;
+  // prefill-shaped NVFP4 batches: each assignment's down row and the compact
+  // row of each assignment (zero-sized otherwise)
+  size_t yperm;    // f32 [T*k, H]
+  size_t inv;      // i32 [T*k]
   size_t total;
   int nChunks;
 };
@@ -87,6 +91,13 @@ inline size_t hq_rows(int T, int k, int terms) {
 // per token.
 inline bool gather_terms(int T, int act) {
   return T > 64 && (act == kActTerms || act == kActE4M3);
+}
+
+// Prefill-shaped NVFP4 batches, at least 32 tokens per expert on average, run
+// on the prefill engine (ffn_pf.cuh): items of 64 tokens, each assignment's
+// down row in y_perm, summed by the combine kernel.
+inline bool prefill_shape(int T, int k, int E, int act) {
+  return act == kActTerms && T > 64 && (long long)T * k >= 32LL * E;
 }
 
 inline WsLayout ws_layout(int T, int k, int E, int H, int I, int act = kActF16) {
@@ -123,6 +134,9 @@ inline WsLayout ws_layout(int T, int k, int E, int H, int I, int act = kActF16) 
   const size_t ng = gather_terms(T, act) ? 1 : 0;
   L.xg = take(ng * (n4 * hq_rows(T, k, 4) * (size_t)H / 2 + n8 * hq_rows(T, k, 2) * (size_t)H));
   L.xgsf = take(ng * n4 * hq_rows(T, k, 4) * (size_t)H / 16);
+  const size_t npf = prefill_shape(T, k, E, act) ? 1 : 0;
+  L.yperm = take(npf * 4 * TK * (size_t)H);
+  L.inv = take(npf * 4 * TK);
   L.total = o;
   return L;
 }

@@ -50,6 +50,9 @@ template <int KS>
 constexpr int ffn_threads() { return (kFfnMTiles * KS + 1) * 32; }
 constexpr int kRowsHalf = 128;  // rows of each of the two weight boxes of a stage
 constexpr int kRowBytes = 128;  // weight bytes per row per stage
+// Prefill engine (ffn_pf.cuh): tokens per item and activation terms used.
+constexpr int kPfTok = 64;
+constexpr int kPfTerms = 3;
 
 template <int FMT>
 struct FmtTraits;

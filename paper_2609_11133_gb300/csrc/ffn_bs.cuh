@@ -491,7 +491,7 @@ __global__ void __launch_bounds__(kBsThreads, 1)
 // power of two, then the terms of each 16-column block by a quad of lanes
 // (four columns each).  One CTA per row, one pass over the row when I <= 1536
 // (96 blocks); every load of the row is issued before the first is used.
-__global__ void __launch_bounds__(kSwigluThreads, 2) swiglu_terms_kernel(const FfnParams p, int rows) {
+static __global__ void __launch_bounds__(kSwigluThreads, 2) swiglu_terms_kernel(const FfnParams p, int rows) {
   constexpr int BPP = kSwigluThreads / 4;          // blocks per pass
   constexpr int PMAX = (8192 / 16 + BPP - 1) / BPP;  // passes for I <= 8192
   __shared__ float s_max[kSwigluThreads / 32];
@@ -557,7 +557,7 @@ __global__ void __launch_bounds__(kSwigluThreads, 2) swiglu_terms_kernel(const F
 // serially by that thread) in 128-thread CTAs: more rows in flight per SM
 // (five CTAs), which pays when there are many rows.  Same codes as the quad
 // kernel.
-__global__ void __launch_bounds__(128) swiglu_terms_rows_kernel(const FfnParams p, int rows) {
+static __global__ void __launch_bounds__(128) swiglu_terms_rows_kernel(const FfnParams p, int rows) {
   constexpr int G = 4;  // blocks per thread (I <= 8192)
   __shared__ float s_max[4];
   // the down step may launch now: what it does before its own wait (plan,

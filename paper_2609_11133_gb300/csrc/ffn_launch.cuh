@@ -27,6 +27,7 @@ cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t sme
 
 struct FfnMaps {
   CUtensorMap a0, a1, s0, s1, b;
+  CUtensorMap sb;  // prefill engine: the activation terms' scales
 };
 
 // Instantiated in ffn_fp8.cu (FMT = 1) and ffn_nvfp4.cu (FMT = 2).
@@ -53,6 +54,11 @@ cudaError_t launch_swiglu_terms(int rows, int sms, const FfnParams& p, cudaStrea
 cudaError_t launch_ffn_f8(int nt, int grid, const FfnMaps& maps, const FfnParams& p,
                           cudaStream_t st);
 cudaError_t launch_swiglu_e4m3(int rows, int sms, const FfnParams& p, cudaStream_t st);
+
+// The NVFP4 prefill engine (ffn_pf.cuh, instantiated in ffn_pf.cu): maps as
+// for the decode engine, with b and sb 3-D maps of the term arrays [rows, 4,
+// K/2] and their scales [rows, 4, K/16], boxes of 3 terms x 64 rows.
+cudaError_t launch_ffn_pf(int grid, const FfnMaps& maps, const FfnParams& p, cudaStream_t st);
 
 
 #define MOE_DEFINE_FFN_LAUNCH(FMTV)                                                            \

@@ -628,8 +628,15 @@ __global__ void __launch_bounds__(256) gather_kernel(const GatherParams p) {
     if (lane == 0) s_off = sum;
   }
   const int nj = min(8, n_e - g0);
-  if (threadIdx.x < nj) s_tok[threadIdx.x] = __ldcg(p.alist + (size_t)e * p.T + g0 + threadIdx.x) / p.k;
+  int a_own = -1;  // thread j < nj: the assignment at list position g0 + j
+  if (threadIdx.x < nj) {
+    a_own = __ldcg(p.alist + (size_t)e * p.T + g0 + threadIdx.x);
+    s_tok[threadIdx.x] = a_own / p.k;
+  }
   __syncthreads();
+  // its compact row (prefill engine: the combine kernel reads each
+  // assignment's down row there)
+  if (p.inv && a_own >= 0) p.inv[a_own] = s_off + g0 + threadIdx.x;
   const int q16 = p.terms * p.qrow / 16;  // 16-byte units of one token's term rows
   for (int i = threadIdx.x; i < nj * q16; i += blockDim.x) {
     const int j = i / q16, u = i - j * q16;
@@ -648,6 +655,10 @@ __global__ void __launch_bounds__(256) gather_kernel(const GatherParams p) {
 }
 
 __global__ void __launch_bounds__(256) combine_kernel(const CombineParams p) {
+  pdl_wait();
+  // the per-expert assignment counters start the next layer call from zero
+  if (p.acnt_reset && blockIdx.x == 0)
+    for (int e = threadIdx.x; e < p.E; e += blockDim.x) p.acnt_reset[e] = 0u;
   const size_t n4 = (size_t)p.T * p.H / 4;
   for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4;
        i += (size_t)gridDim.x * blockDim.x) {
@@ -656,9 +667,9 @@ __global__ void __launch_bounds__(256) combine_kernel(const CombineParams p) {
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
     for (int j = 0; j < p.k; ++j) {
       const size_t a = t * p.k + j;
-      const float w = __ldg(p.topk_w + a);
-      const int row = __ldg(p.inv + a);
-      const float4 y = __ldg(reinterpret_cast<const float4*>(p.y_perm + (size_t)row * p.H + h));
+      const float w = __ldcg(p.topk_w + a);
+      const int row = __ldcg(p.inv + a);
+      const float4 y = __ldcg(reinterpret_cast<const float4*>(p.y_perm + (size_t)row * p.H + h));
       acc.x = fmaf(w, y.x, acc.x);
       acc.y = fmaf(w, y.y, acc.y);
       acc.z = fmaf(w, y.z, acc.z);
@@ -735,8 +746,16 @@ cudaError_t launch_combine(const CombineParams& p, cudaStream_t st) {
   size_t blocks = (n4 + 255) / 256;
   if (blocks > 4096) blocks = 4096;
   if (blocks == 0) blocks = 1;
-  combine_kernel<<<(unsigned)blocks, 256, 0, st>>>(p);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)blocks);
+  cfg.blockDim = dim3(256);
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, combine_kernel, p);
 }
 
 }  // namespace moe

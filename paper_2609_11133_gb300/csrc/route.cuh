@@ -72,6 +72,7 @@ struct GatherParams {
   uint8_t* gsf;       // [T*k*terms, sfrow] (when sf)
   const unsigned* acnt;
   const int* alist;   // [E, T]
+  int* inv;           // [T*k] compact row of each assignment, or null
   int T, k, E, terms, qrow, sfrow;
 };
 
@@ -82,6 +83,8 @@ struct CombineParams {
   int T, k, H;
   const __nv_bfloat16* residual;
   __nv_bfloat16* out;
+  unsigned* acnt_reset;  // the fused layer's per-expert counters, zeroed here (or null)
+  int E;
 };
 
 cudaError_t launch_route(const RouteParams& p, cudaStream_t st);

@@ -18,10 +18,11 @@ def test_default_workload_is_the_headline():
 
 def test_sweep_covers_both_served_models_at_small_batches():
     names = {n for n, _ in bench.SWEEP}
-    assert names == {"qwen3_235b_nvfp4", "qwen3_480b_fp8_zipf"}
+    assert names == {"qwen3_235b_nvfp4", "qwen3_480b_fp8_zipf", "qwen3_235b_nvfp4_prefill"}
     batches = dict(bench.SWEEP)
     assert set(batches["qwen3_235b_nvfp4"]) == {1, 8, 32, 64}
     assert {1, 8, 32}.issubset(batches["qwen3_480b_fp8_zipf"])
+    assert batches["qwen3_235b_nvfp4_prefill"] == (2048,)
     assert not bench.parse([]).no_sweep and bench.parse(["--no-sweep"]).no_sweep
 
 
