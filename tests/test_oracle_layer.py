@@ -147,6 +147,26 @@ def test_exact_rational_reference_tiny_nvfp4():
             assert abs(float(y) - out[t, r]) <= 1e-12 * max(1.0, abs(float(y)))
 
 
+def test_rmsnorm_eps_and_mean_pinned_by_worked_values():
+    """The pre-norm reading bf16(x / sqrt(mean(x^2) + eps)), eps = 1e-6 inside
+    the root, pinned by values worked out by hand where the other readings
+    differ: a constant row at 2^-10, whose mean square (2^-20) is comparable
+    to eps, gives 2^-10 / sqrt(2^-20 + 1e-6) = 0.698677..., bf16 0.69921875
+    (eps outside the root would give 0.99898 -> 1.0, no eps 1.0); a row with
+    one element 1 and 63 zeros gives 1 / sqrt(1/64 + 1e-6) = 7.99974..., bf16
+    8.0 (a sum instead of a mean would give 1.0)."""
+    H = 64
+    const = np.full((1, H), 2.0 ** -10)
+    one = np.zeros((1, H))
+    one[0, 0] = 1.0
+    # both rows hold values exact in bf16: their bits are the top half of the fp32 bits
+    rows = np.concatenate([const, one]).astype(np.float32)
+    bits = (rows.view(np.uint32) >> 16).astype(np.uint16)
+    out = indep.bf16_to_f64(oracle.rmsnorm_bf16(bits, 1e-6))
+    assert (out[0] == 0.69921875).all()
+    assert out[1, 0] == 8.0 and (out[1, 1:] == 0.0).all()
+
+
 def test_rmsnorm_rounds_to_nearest_bf16():
     x = np_(synth.make_x(4, 64, seed=90, std=3.0))
     xn = oracle.rmsnorm_bf16(x, 1e-6)
