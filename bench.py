@@ -65,6 +65,7 @@ WORKLOADS = {
     "tiny_fp8": dict(fmt=1, H=512, E=8, k=2, I=256, T=4),
 }
 MOE_FLAG_PRENORM_RMS = 0x2
+MOE_FLAG_DETERMINISTIC = 0x4
 
 
 def workload(args):
@@ -74,8 +75,9 @@ def workload(args):
         wl["T"] = args.tokens
     if args.experts is not None:
         wl["E"] = args.experts
+    wl["det"] = bool(getattr(args, "deterministic", False))
     wl["name"] = args.workload + (f"_E{wl['E']}" if args.experts is not None else "") \
-        + f"_T{wl['T']}"
+        + f"_T{wl['T']}" + ("_det" if wl["det"] else "")
     return wl
 
 
@@ -95,6 +97,9 @@ def parse(argv=None):
     ap.add_argument("--no-energy", action="store_true")
     ap.add_argument("--no-sweep", action="store_true",
                     help="skip the batch sweep of the default run")
+    ap.add_argument("--deterministic", action="store_true",
+                    help="run the layer with MOE_FLAG_DETERMINISTIC (the same output bits "
+                         "on every run)")
     return ap.parse_args(argv)
 
 
@@ -438,13 +443,15 @@ class Runner:
         self.torch, self.binding = torch, binding
         self.wl, self.layers, self.bias = wl, layers, bias
         self.T, self.H, self.k, self.E, self.L = wl["T"], wl["H"], wl["k"], wl["E"], wl["layers"]
-        self.flags = MOE_FLAG_PRENORM_RMS if wl["prenorm"] else 0
+        self.flags = (MOE_FLAG_PRENORM_RMS if wl["prenorm"] else 0) | \
+            (MOE_FLAG_DETERMINISTIC if wl.get("det") else 0)
         T, H = self.T, self.H
         self.dev = dev
         x = synth.make_x(T, H, seed=seed + rank, device=dev)
         # the residual stream of a stack: layer l reads cur and writes nxt
         self.bufs = [torch.empty((T, H), dtype=torch.bfloat16, device=dev) for _ in range(2)]
-        self.ws = binding.alloc_workspace(binding.moe_workspace_size(layers[0][0], T, self.k))
+        self.ws = binding.alloc_workspace(
+            binding.moe_workspace_size(layers[0][0], T, self.k, self.flags))
         self.stream = torch.cuda.current_stream()
         w0 = layers[0][0]
         self.gu_bytes, self.dn_bytes = expert_bytes(w0)
@@ -768,6 +775,8 @@ def run_ours(args):
                           "e4m3 x e4m3 MMA, 128x128 fp32 block scales applied per stage, "
                           "activations as 2 e4m3 terms, fp32 accumulate"),
            "parallelism": f"replicas x{world}"}
+    if wl["det"]:
+        cfg["deterministic"] = "MOE_FLAG_DETERMINISTIC (down step timed with its combine)"
     if L > 1:
         cfg.update(layers=L, prenorm="rms, eps 1e-6, unit weight", residual="threaded",
                    weights_gb=round(sum(w.nbytes_expert() * E for w, _ in layers) / 1e9, 1))

@@ -96,6 +96,8 @@ typedef enum { MOE_FMT_FP8_B128 = 1, MOE_FMT_NVFP4 = 2 } moe_format_t;
 #define MOE_FLAG_NO_RENORM 0x1   /* gates = full-softmax probabilities at the top-k */
 #define MOE_FLAG_PRENORM_RMS 0x2 /* route and run the experts on bf16(RMSNorm(x)),
                                     unit weight, eps 1e-6; residual is still added */
+#define MOE_FLAG_DETERMINISTIC 0x4 /* the same output bits on every run: see
+                                      moe_decode_layer */
 
 /* The expert weights of one layer.  All pointers are device pointers to the
  * caller's buffers; the struct itself is read on the host during the call. */
@@ -117,6 +119,13 @@ int moe_version(void);
  * these weights and T tokens with k experts each (*bytes, host pointer).
  * Pure host computation. */
 int moe_workspace_size(const moe_expert_weights_t* w, int T, int k, size_t* bytes);
+
+/* As moe_workspace_size, for a moe_decode_layer call with these flags
+ * (MOE_FLAG_*): MOE_FLAG_DETERMINISTIC adds T*k*H*4 bytes (one fp32 down row
+ * per assignment) unless the batch already keeps them; the other flags add
+ * nothing.  MOE_ERR_INVALID_ARG for an unknown flag bit. */
+int moe_workspace_size_flags(const moe_expert_weights_t* w, int T, int k, int flags,
+                             size_t* bytes);
 
 /* Kernels one moe_decode_layer call launches for these weights and T tokens
  * with k experts each (*count, host pointer): the router, the gather of the
@@ -204,8 +213,20 @@ int moe_combine(const float* y_perm, const float* topk_w, const int32_t* inv_per
  *   flags: MOE_FLAG_*; residual [T, H] bf16 or NULL (may alias out);
  *   out [T, H] bf16, must not alias x;
  *   alignment: x and router_w 16 bytes, out and residual 8 bytes, ws 256 bytes;
- *   ws: at least moe_workspace_size(w, T, k) bytes, zeroed once before
- *   first use (moe_workspace_init). */
+ *   ws: at least moe_workspace_size_flags(w, T, k, flags) bytes, zeroed
+ *   once before first use (moe_workspace_init).
+ * Reproducibility.  The expert kernels split the work of an expert's row tile
+ * over K between CTAs, and the partial sums meet in fp32 atomic adds, as do
+ * the k expert rows of a token; the order of those adds varies from run to
+ * run, and so may the last bits of `out`.  MOE_FLAG_DETERMINISTIC removes
+ * every such order: each (expert, 128-row tile, token chunk) is summed over
+ * its whole K range by one CTA (CTA shares end on those boundaries), each
+ * assignment's down row is written to its own fp32 row, and a combine kernel
+ * adds a token's k rows in the order j = 0..k-1.  The same call then gives
+ * the same bits on every run, whatever the stream, the concurrent work or the
+ * order in which the routing lists an expert's tokens.  It costs the larger
+ * workspace and a less even division of the stages between the SMs (most at
+ * T = 1, where few items meet many SMs). */
 int moe_decode_layer(const void* x, const float* router_w, const float* router_bias,
                      const moe_expert_weights_t* w, int T, int k, int flags, const void* residual,
                      void* out, void* ws, size_t ws_bytes, void* stream);
@@ -230,10 +251,10 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
  *   Arguments as moe_decode_layer, minus ws / ws_bytes.
  *   Scratch: a 16 MiB device array inside libmoe.so; every GPU that loads the
  *     library holds it until the process exits.  Shapes whose
- *     moe_workspace_size() exceeds 16 MiB return MOE_ERR_WORKSPACE_TOO_SMALL:
+ *     moe_workspace_size_flags() exceeds 16 MiB return MOE_ERR_WORKSPACE_TOO_SMALL:
  *     the 235B-shaped NVFP4 layer (H=4096, E=128, k=8, I=1536) fits up to
  *     T = 74 tokens, the 480B-shaped FP8 layer (H=6144, E=160, k=8, I=2560)
- *     up to T = 64.
+ *     up to T = 64 (without MOE_FLAG_DETERMINISTIC).
  *   The first call on a device looks up the array's device address and
  *     clears the array's status word; make that first call before capturing
  *     the stream into a CUDA graph.  A lookup that fails returns MOE_ERR_CUDA

@@ -22,6 +22,7 @@ MOE_FMT_FP8_B128 = 1
 MOE_FMT_NVFP4 = 2
 MOE_FLAG_NO_RENORM = 0x1
 MOE_FLAG_PRENORM_RMS = 0x2
+MOE_FLAG_DETERMINISTIC = 0x4
 _FLAG_TEST_STALL = 0x100  # test hook of moe_decode_layer (see moe.h)
 
 _STATUS = {
@@ -55,6 +56,8 @@ _SZ = ctypes.c_size_t
 _SIGS = {
     "moe_version": [],
     "moe_workspace_size": [ctypes.POINTER(ExpertWeightsC), _I, _I, ctypes.POINTER(_SZ)],
+    "moe_workspace_size_flags": [ctypes.POINTER(ExpertWeightsC), _I, _I, _I,
+                                 ctypes.POINTER(_SZ)],
     "moe_route_workspace_size": [_I, _I, ctypes.POINTER(_SZ)],
     "moe_layer_kernel_count": [ctypes.POINTER(ExpertWeightsC), _I, _I, ctypes.POINTER(_I)],
     "moe_cost_split_stage": [_P, _I, _I, _I, _I, _I, _I, ctypes.c_longlong, ctypes.c_longlong,
@@ -133,11 +136,17 @@ def moe_version() -> int:
     return load().moe_version()
 
 
-def moe_workspace_size(w, T: int, k: int) -> int:
+def moe_workspace_size(w, T: int, k: int, flags: int = 0) -> int:
+    """Workspace bytes of a moe_decode_layer call with these flags (flags = 0:
+    moe_workspace_size, which also covers moe_expert_ffn)."""
     n = _SZ(0)
     ws = weights_struct(w)
-    _check(load().moe_workspace_size(ctypes.byref(ws), T, k, ctypes.byref(n)),
-           "moe_workspace_size")
+    if flags:
+        _check(load().moe_workspace_size_flags(ctypes.byref(ws), T, k, flags, ctypes.byref(n)),
+               "moe_workspace_size_flags")
+    else:
+        _check(load().moe_workspace_size(ctypes.byref(ws), T, k, ctypes.byref(n)),
+               "moe_workspace_size")
     return n.value
 
 

@@ -208,6 +208,16 @@ int check_tk(int T, int k, int E) {
   return MOE_OK;
 }
 
+constexpr int kLayerFlags =
+    MOE_FLAG_NO_RENORM | MOE_FLAG_PRENORM_RMS | MOE_FLAG_DETERMINISTIC | kFlagTestStall;
+
+// Workspace of a moe_decode_layer call: the deterministic mode keeps one fp32
+// down row per assignment (the prefill engine keeps them anyway).
+WsLayout layer_layout(const moe_expert_weights_t* w, int T, int k, int flags) {
+  return ws_layout(T, k, w->E, w->H, w->I, act_for(w->fmt, engine_for(w->fmt)),
+                   (flags & MOE_FLAG_DETERMINISTIC) != 0);
+}
+
 // ------------------------------------------------------------------ the expert steps
 struct ExpertRun {
   const moe_expert_weights_t* w;
@@ -224,6 +234,7 @@ struct ExpertRun {
   __nv_bfloat16* out;
   const __nv_bfloat16* residual;
   int test_stall;
+  int det;  // deterministic mode (FfnParams::det)
 };
 
 int run_experts(const ExpertRun& r, cudaStream_t st, cudaEvent_t ev_mid) {
@@ -297,6 +308,7 @@ int run_experts(const ExpertRun& r, cudaStream_t st, cudaEvent_t ev_mid) {
   p.status = ws_ptr<uint32_t>(r.ws, r.L.status);
   p.units = ws_ptr<uint32_t>(r.ws, r.L.units);
   p.wait_ns = wait_limit_ns();
+  p.det = r.det;
 
   FfnParams p1 = p;
   p1.phase = 1;
@@ -435,14 +447,19 @@ const char* moe_status_string(int s) {
 
 int moe_version(void) { return kAbiVersion; }
 
-int moe_workspace_size(const moe_expert_weights_t* w, int T, int k, size_t* bytes) {
-  if (!bytes) return MOE_ERR_INVALID_ARG;
+int moe_workspace_size_flags(const moe_expert_weights_t* w, int T, int k, int flags,
+                             size_t* bytes) {
+  if (!bytes || (flags & ~kLayerFlags)) return MOE_ERR_INVALID_ARG;
   int rc = check_weights(w);
   if (rc) return rc;
   rc = check_tk(T, k, w->E);
   if (rc) return rc;
-  *bytes = ws_layout(T, k, w->E, w->H, w->I, act_for(w->fmt, engine_for(w->fmt))).total;
+  *bytes = layer_layout(w, T, k, flags).total;
   return MOE_OK;
+}
+
+int moe_workspace_size(const moe_expert_weights_t* w, int T, int k, size_t* bytes) {
+  return moe_workspace_size_flags(w, T, k, 0, bytes);
 }
 
 int moe_layer_kernel_count(const moe_expert_weights_t* w, int T, int k, int* count) {
@@ -648,8 +665,7 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
                         const void* residual, void* out, void* ws, size_t ws_bytes,
                         float* logits_out, int32_t* topk_ids_out, float* topk_w_out,
                         void* const* events, void* stream) {
-  if (flags & ~(MOE_FLAG_NO_RENORM | MOE_FLAG_PRENORM_RMS | kFlagTestStall))
-    return MOE_ERR_INVALID_ARG;
+  if (flags & ~kLayerFlags) return MOE_ERR_INVALID_ARG;
   int rc = check_weights(w);
   if (rc) return rc;
   rc = check_tk(T, k, w->E);
@@ -661,7 +677,7 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
     return MOE_ERR_INVALID_ARG;
   if (out == x) return MOE_ERR_INVALID_ARG;
   const int E = w->E, H = w->H, I = w->I;
-  const WsLayout L = ws_layout(T, k, E, H, I, act_for(w->fmt, engine_for(w->fmt)));
+  const WsLayout L = layer_layout(w, T, k, flags);
   if (ws_bytes < L.total) return MOE_ERR_WORKSPACE_TOO_SMALL;
   if (T == 0) return MOE_OK;
   int sms = 0;
@@ -674,6 +690,9 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
   const int eng = engine_for(w->fmt);
   const int nt = nt_for(T, eng);
   const bool pf = use_prefill(T, k, E, eng);
+  // deterministic mode of the decode engines (the prefill engine sums every
+  // item in one CTA and each token's rows in the combine kernel anyway)
+  const bool det = (flags & MOE_FLAG_DETERMINISTIC) && !pf;
 
   RouteParams p{};
   p.x = static_cast<const __nv_bfloat16*>(x);
@@ -699,12 +718,15 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
   p.xq = ws_ptr<uint8_t>(ws, L.xq);
   p.xsf = ws_ptr<uint8_t>(ws, L.xsf);
   p.xinv = ws_ptr<float>(ws, L.xinv);
-  // the decode engine adds its partial sums into zeroed accumulators; the
-  // prefill engine stores complete sums and needs none
+  // the decode engines add their partial sums into zeroed accumulators (the
+  // token rows, or in the deterministic mode each assignment's row); the
+  // prefill engine, and the tensor-core engines in the deterministic mode,
+  // store complete sums and need none
+  const bool stores = pf || (det && eng != kEngMma);
   p.zero_a = ws_ptr<float4>(ws, L.gu);
-  p.zero_a_n4 = pf ? 0 : (size_t)T * k * 2 * I / 4;
-  p.zero_b = ws_ptr<float4>(ws, L.oacc);
-  p.zero_b_n4 = pf ? 0 : (size_t)T * H / 4;
+  p.zero_a_n4 = stores ? 0 : (size_t)T * k * 2 * I / 4;
+  p.zero_b = ws_ptr<float4>(ws, det ? L.yperm : L.oacc);
+  p.zero_b_n4 = stores ? 0 : (size_t)T * (det ? k : 1) * H / 4;
   p.acnt = ws_ptr<unsigned>(ws, L.acnt);
   p.alist = ws_ptr<int>(ws, L.alist);
   if (ev[0] && cudaEventRecord(ev[0], st) != cudaSuccess) return MOE_ERR_CUDA;
@@ -750,12 +772,21 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
   r.gathered = gathered ? 1 : 0;
   r.counts = reinterpret_cast<const int*>(p.acnt);
   r.gates = p.gates;
-  r.fused = 1;
+  r.fused = det ? 0 : 1;  // deterministic: down rows by assignment, then the combine
+  r.y_perm = det ? ws_ptr<float>(ws, L.yperm) : nullptr;
+  r.det = det ? 1 : 0;
   r.out = static_cast<__nv_bfloat16*>(out);
   r.residual = static_cast<const __nv_bfloat16*>(residual);
   r.test_stall = (flags & kFlagTestStall) ? 1 : 0;
   rc = run_experts(r, st, ev[2]);
   if (rc) return rc;
+  if (det) {
+    // a token's k rows in the order j = 0..k-1; also zeroes the counters
+    CombineParams c{r.y_perm, p.gates, nullptr, T, k, H,
+                    static_cast<const __nv_bfloat16*>(residual), static_cast<__nv_bfloat16*>(out),
+                    p.acnt, E};
+    if (launch_combine(c, st) != cudaSuccess) return MOE_ERR_CUDA;
+  }
   if (ev[3] && cudaEventRecord(ev[3], st) != cudaSuccess) return MOE_ERR_CUDA;
   return MOE_OK;
 }

@@ -70,7 +70,8 @@ struct WsLayout {
   size_t xg;
   size_t xgsf;
   // prefill-shaped NVFP4 batches: each assignment's down row and the compact
-  // row of each assignment (zero-sized otherwise)
+  // row of each assignment (zero-sized otherwise); the deterministic mode of
+  // the decode engines keeps the down rows too (by assignment)
   size_t yperm;    // f32 [T*k, H]
   size_t inv;      // i32 [T*k]
   size_t total;
@@ -100,7 +101,8 @@ inline bool prefill_shape(int T, int k, int E, int act) {
   return act == kActTerms && T > 64 && (long long)T * k >= 32LL * E;
 }
 
-inline WsLayout ws_layout(int T, int k, int E, int H, int I, int act = kActF16) {
+inline WsLayout ws_layout(int T, int k, int E, int H, int I, int act = kActF16,
+                          bool det = false) {
   WsLayout L{};
   size_t o = 0;
   auto take = [&](size_t bytes) {
@@ -135,7 +137,7 @@ inline WsLayout ws_layout(int T, int k, int E, int H, int I, int act = kActF16) 
   L.xg = take(ng * (n4 * hq_rows(T, k, 4) * (size_t)H / 2 + n8 * hq_rows(T, k, 2) * (size_t)H));
   L.xgsf = take(ng * n4 * hq_rows(T, k, 4) * (size_t)H / 16);
   const size_t npf = prefill_shape(T, k, E, act) ? 1 : 0;
-  L.yperm = take(npf * 4 * TK * (size_t)H);
+  L.yperm = take((npf || det ? 1 : 0) * 4 * TK * (size_t)H);
   L.inv = take(npf * 4 * TK);
   L.total = o;
   return L;
@@ -302,6 +304,16 @@ __device__ __forceinline__ uint32_t hmul2_u32(uint32_t a, uint32_t b) {
 
 __device__ __forceinline__ void red_add_f32(float* p, float v) {
   asm volatile("red.global.add.f32 [%0], %1;" ::"l"(p), "f"(v) : "memory");
+}
+
+// A sum into an output element: added to the zeroed accumulator, or stored
+// where it is the element's only sum (the deterministic mode of the
+// tensor-core engines, whose CTAs each sum whole items).
+__device__ __forceinline__ void put_f32(float* p, float v, bool store) {
+  if (store)
+    asm volatile("st.global.f32 [%0], %1;" ::"l"(p), "f"(v) : "memory");
+  else
+    red_add_f32(p, v);
 }
 
 // Power-of-two factor that maps max|v| into [2^14, 2^15): f16 holds the

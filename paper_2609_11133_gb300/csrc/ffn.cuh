@@ -105,6 +105,14 @@ struct StageGeom {
 struct FfnParams {
   int T, k, E, H, I, phase;  // phase 1 = gate/up, 2 = down
   int fused;                 // phase 2: 1 = scatter into oacc + bf16 out, 0 = y_perm
+  // 1 = deterministic mode: every CTA's share of the stages starts and ends
+  // on an item boundary (the units of the FP8 engine's shared tail are whole
+  // items), and the unfused phase 2 writes row
+  // a (the assignment t*k + j) of y_perm instead of the compact row.  The
+  // tensor-core engines then store each output element once (gu and y_perm
+  // need no zeroing); the warp-MMA engine still adds the partial sums of its
+  // two K-halves (two adds onto zero give the same bits in either order).
+  int det;
   // routing: tokens per expert, and each expert's assignments (t*k + j).
   // list_T = 1: expert e's list starts at sorted[e*T] (the fused layer's
   // per-expert lists); 0: at sorted[offsets[e]] (one array sorted by expert).
@@ -260,6 +268,13 @@ __host__ __device__ __forceinline__ int cost_split_stage(const PlanSmem& pl, int
   return ((pl.cpre[lo] * rtiles) + rt * ch + chunk) * KB + kb;
 }
 
+// Deterministic mode: a share boundary moved to the nearest item boundary
+// (items are KB stages long), so that every item is summed by one CTA over
+// its whole K range.  Both CTAs beside a boundary round it alike.
+__host__ __device__ __forceinline__ long long item_boundary(long long s, int KB) {
+  return (s + KB / 2) / KB * KB;
+}
+
 // Position of a CTA's current stage without divisions: item `it`, K-block
 // `kb` inside it, ring slot and that slot's phase parity ((i / S) & 1).
 template <int S>
@@ -292,6 +307,8 @@ struct StageCursor {
 // kUnitStages stages of the rest, taken one at a time from a global counter
 // by the lead producer and handed to the CTA's other roles through a ring in
 // shared memory.  A CTA whose copies land faster takes more of the tail.
+// In the deterministic mode a unit is one whole item (KB stages) and the tail
+// starts on an item boundary, so that every item is still summed by one CTA.
 constexpr int kUnitStages = 8;
 constexpr int kStaticNum = 4, kStaticDen = 5;
 constexpr int kTailMinStages = 200;  // per CTA
@@ -319,9 +336,9 @@ __device__ __forceinline__ bool unit_push(UnitRing& r, int j, int a, uint64_t wa
 // when the wait expired (*ok = false).  A warp-wide reader calls this on all
 // lanes and lane 0 reports the entry read; a one-thread reader reports it
 // itself (warp_wide false).
-__device__ __forceinline__ bool unit_next(UnitRing& r, int& j, int total, int& a, int& b,
-                                          bool warp_wide, uint64_t wait_ns, volatile int* abort,
-                                          bool* ok) {
+__device__ __forceinline__ bool unit_next(UnitRing& r, int& j, int total, int us, int& a,
+                                          int& b, bool warp_wide, uint64_t wait_ns,
+                                          volatile int* abort, bool* ok) {
   const int q = j % kUnitRing;
   if (!mbar_wait_bounded(&r.full[q], (uint32_t)(j / kUnitRing) & 1u, wait_ns, abort)) {
     *ok = false;
@@ -337,7 +354,7 @@ __device__ __forceinline__ bool unit_next(UnitRing& r, int& j, int total, int& a
   ++j;
   if (first < 0) return false;
   a = first;
-  b = min(first + kUnitStages, total);
+  b = min(first + us, total);
   return true;
 }
 
@@ -354,8 +371,8 @@ __device__ __forceinline__ void unit_done(uint32_t* units) {
 }
 
 // The unit that follows a CTA's last one: first stage, or -1 past the end.
-__device__ __forceinline__ int unit_take(uint32_t* units, int s_dyn, int total) {
-  const long long a = (long long)s_dyn + (long long)atomicAdd(units, 1u) * kUnitStages;
+__device__ __forceinline__ int unit_take(uint32_t* units, int s_dyn, int total, int us) {
+  const long long a = (long long)s_dyn + (long long)atomicAdd(units, 1u) * us;
   return a < total ? (int)a : -1;
 }
 
@@ -524,8 +541,12 @@ __global__ void __launch_bounds__(ffn_threads<KS>(), 1)
   const int KB = K / KEL;
   const long long items = (long long)pl.cpre[pl.nA] * rtiles;
   const long long total = items * KB;
-  const long long s_begin = total * blockIdx.x / gridDim.x;
-  const long long s_end = total * (blockIdx.x + 1) / gridDim.x;
+  long long s_begin = total * blockIdx.x / gridDim.x;
+  long long s_end = total * (blockIdx.x + 1) / gridDim.x;
+  if (p.det) {
+    s_begin = item_boundary(s_begin, KB);
+    s_end = item_boundary(s_end, KB);
+  }
   const uint32_t timeout_bit = (p.phase == 1) ? kStatusTimeoutGateUp : kStatusTimeoutDown;
 
   if (is_producer) {
@@ -643,7 +664,7 @@ __global__ void __launch_bounds__(ffn_threads<KS>(), 1)
               colrow[n][c] = a / p.k;
               colgate[n][c] = __ldg(p.gates + a);
             } else {
-              colrow[n][c] = arow;
+              colrow[n][c] = p.det ? a : arow;
               colgate[n][c] = 1.f;
             }
           }

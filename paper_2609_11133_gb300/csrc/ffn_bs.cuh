@@ -165,9 +165,12 @@ __global__ void __launch_bounds__(kBsThreads, 1)
   // shape), divided by cost (items of many tokens cost more per stage when
   // their rows come token by token)
   const int cost_a = stage_cost_base((PHASE == 1) && !p.b_compact);
-  const int s_begin = cost_split_stage(pl, rtiles, KB, NT, cost_a, kTokenCost, blockIdx.x, gridDim.x);
-  const int s_end = cost_split_stage(pl, rtiles, KB, NT, cost_a, kTokenCost, blockIdx.x + 1,
-                                     gridDim.x);
+  int s_begin = cost_split_stage(pl, rtiles, KB, NT, cost_a, kTokenCost, blockIdx.x, gridDim.x);
+  int s_end = cost_split_stage(pl, rtiles, KB, NT, cost_a, kTokenCost, blockIdx.x + 1, gridDim.x);
+  if (p.det) {
+    s_begin = (int)item_boundary(s_begin, KB);
+    s_end = (int)item_boundary(s_end, KB);
+  }
   const int nst = s_end - s_begin;
   const uint32_t timeout_bit = (PHASE == 1) ? kStatusTimeoutGateUp : kStatusTimeoutDown;
   // B rows: per token (phase 1, tokens scattered) or one box per chunk
@@ -462,8 +465,8 @@ __global__ void __launch_bounds__(kBsThreads, 1)
             const float sc = __ldg(p.xinv + a / p.k);
             const int f = inf.rt * kRowsHalf + row;
             float* gr = p.gu + (size_t)arow * 2 * p.I + f;
-            red_add_f32(gr, acc[0][j] * sc * ts0);
-            red_add_f32(gr + p.I, acc[1][j] * sc * ts1);
+            put_f32(gr, acc[0][j] * sc * ts0, p.det);
+            put_f32(gr + p.I, acc[1][j] * sc * ts1, p.det);
           } else {
             const float sc = __ldcg(p.xinv + arow);  // hinv, written by the previous kernel
             const int hrow = inf.rt * 2 * kRowsHalf + row;
@@ -473,9 +476,9 @@ __global__ void __launch_bounds__(kBsThreads, 1)
               red_add_f32(orow, gw * acc[0][j] * ts0);
               red_add_f32(orow + kRowsHalf, gw * acc[1][j] * ts1);
             } else {
-              float* yrow = p.y_perm + (size_t)arow * p.H + hrow;
-              red_add_f32(yrow, acc[0][j] * sc * ts0);
-              red_add_f32(yrow + kRowsHalf, acc[1][j] * sc * ts1);
+              float* yrow = p.y_perm + (size_t)(p.det ? a : arow) * p.H + hrow;
+              put_f32(yrow, acc[0][j] * sc * ts0, p.det);
+              put_f32(yrow + kRowsHalf, acc[1][j] * sc * ts1, p.det);
             }
           }
         }

@@ -141,12 +141,18 @@ __global__ void __launch_bounds__(kF8Threads, 1)
   const int snum = tail ? kStaticNum : 1, sden = tail ? kStaticDen : 1;
   const int cost_a = stage_cost_base((PHASE == 1) && !p.b_compact);
   const long long den = (long long)gridDim.x * sden;
-  const int s_begin = cost_split_stage(pl, rtiles, KB, NT, cost_a, kTokenCost,
-                                       (long long)blockIdx.x * snum, den);
-  const int s_end = cost_split_stage(pl, rtiles, KB, NT, cost_a, kTokenCost,
-                                     (long long)(blockIdx.x + 1) * snum, den);
-  const int s_dyn = tail ? cost_split_stage(pl, rtiles, KB, NT, cost_a, kTokenCost, snum, sden)
-                         : total;
+  int s_begin = cost_split_stage(pl, rtiles, KB, NT, cost_a, kTokenCost,
+                                 (long long)blockIdx.x * snum, den);
+  int s_end = cost_split_stage(pl, rtiles, KB, NT, cost_a, kTokenCost,
+                               (long long)(blockIdx.x + 1) * snum, den);
+  if (p.det) {
+    s_begin = (int)item_boundary(s_begin, KB);
+    s_end = (int)item_boundary(s_end, KB);
+  }
+  int s_dyn = tail ? cost_split_stage(pl, rtiles, KB, NT, cost_a, kTokenCost, snum, sden)
+                   : total;
+  if (p.det) s_dyn = (int)item_boundary(s_dyn, KB);  // the last CTA's share ends here too
+  const int us = p.det ? KB : kUnitStages;  // stages per unit of the tail
   uint32_t* units = p.units + 2 * (PHASE - 1);
   const uint32_t timeout_bit = (PHASE == 1) ? kStatusTimeoutGateUp : kStatusTimeoutDown;
   // B rows: per token (phase 1, tokens scattered) or one box per chunk
@@ -230,15 +236,15 @@ __global__ void __launch_bounds__(kF8Threads, 1)
         }
         if (!ok || !tail) break;
         if (lead) {
-          const int next = unit_take(units, s_dyn, total);
+          const int next = unit_take(units, s_dyn, total, us);
           if (!unit_push(s_units, uj++, next, p.wait_ns, &s_abort)) {
             ok = false;
             break;
           }
           if (next < 0) break;
           a = next;
-          b = min(next + kUnitStages, total);
-        } else if (!unit_next(s_units, uj, total, a, b, false, p.wait_ns, &s_abort, &ok)) {
+          b = min(next + us, total);
+        } else if (!unit_next(s_units, uj, total, us, a, b, false, p.wait_ns, &s_abort, &ok)) {
           break;
         }
         c.seek(a);
@@ -294,7 +300,7 @@ __global__ void __launch_bounds__(kF8Threads, 1)
           tc_commit(&empty_bar[slot]);
           tc_commit(&dfull_bar[db]);
         }
-        if (!ok || !tail || !unit_next(s_units, uj, total, a, b, false, p.wait_ns, &s_abort, &ok))
+        if (!ok || !tail || !unit_next(s_units, uj, total, us, a, b, false, p.wait_ns, &s_abort, &ok))
           break;
       }
       if (!ok) {
@@ -345,7 +351,7 @@ __global__ void __launch_bounds__(kF8Threads, 1)
     int cs = s_begin, cend = s_end, uj = 0;
     bool ok = true;
     bool have = cs < cend;
-    if (!have && tail && unit_next(s_units, uj, total, cs, cend, true, p.wait_ns, &s_abort, &ok)) {
+    if (!have && tail && unit_next(s_units, uj, total, us, cs, cend, true, p.wait_ns, &s_abort, &ok)) {
       c.seek(cs);
       have = true;
     }
@@ -361,7 +367,7 @@ __global__ void __launch_bounds__(kF8Threads, 1)
       nc.next();
       bool have_next = ns < nend, jump = false;
       if (!have_next && tail) {
-        have_next = unit_next(s_units, uj, total, ns, nend, true, p.wait_ns, &s_abort, &ok);
+        have_next = unit_next(s_units, uj, total, us, ns, nend, true, p.wait_ns, &s_abort, &ok);
         jump = true;
         if (have_next) nc.seek(ns);
       }
@@ -412,8 +418,8 @@ __global__ void __launch_bounds__(kF8Threads, 1)
               const float sc = __ldg(p.xinv + a / p.k);
               const int f = inf.rt * kRowsHalf + row;
               float* gr = p.gu + (size_t)arow * 2 * p.I + f;
-              red_add_f32(gr, acc0[j] * sc);
-              red_add_f32(gr + p.I, acc1[j] * sc);
+              put_f32(gr, acc0[j] * sc, p.det);
+              put_f32(gr + p.I, acc1[j] * sc, p.det);
             } else {
               const float sc = __ldcg(p.xinv + arow);  // hinv, written by the previous kernel
               const int hrow = inf.rt * 2 * kRowsHalf + row;
@@ -423,9 +429,9 @@ __global__ void __launch_bounds__(kF8Threads, 1)
                 red_add_f32(orow, gw * acc0[j]);
                 red_add_f32(orow + kRowsHalf, gw * acc1[j]);
               } else {
-                float* yrow = p.y_perm + (size_t)arow * p.H + hrow;
-                red_add_f32(yrow, acc0[j] * sc);
-                red_add_f32(yrow + kRowsHalf, acc1[j] * sc);
+                float* yrow = p.y_perm + (size_t)(p.det ? a : arow) * p.H + hrow;
+                put_f32(yrow, acc0[j] * sc, p.det);
+                put_f32(yrow + kRowsHalf, acc1[j] * sc, p.det);
               }
             }
           }

@@ -57,7 +57,7 @@ extern "C" int moe_decode_layer_noalloc(const void* x, const float* router_w,
                                         int T, int k, int flags, const void* residual, void* out,
                                         void* stream) {
   size_t need = 0;
-  int rc = moe_workspace_size(w, T, k, &need);
+  int rc = moe_workspace_size_flags(w, T, k, flags, &need);
   if (rc != MOE_OK) return rc;
   if (need > kNoAllocBytes) return MOE_ERR_WORKSPACE_TOO_SMALL;
   if (T == 0) return MOE_OK;

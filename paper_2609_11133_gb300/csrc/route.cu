@@ -668,7 +668,7 @@ __global__ void __launch_bounds__(256) combine_kernel(const CombineParams p) {
     for (int j = 0; j < p.k; ++j) {
       const size_t a = t * p.k + j;
       const float w = __ldcg(p.topk_w + a);
-      const int row = __ldcg(p.inv + a);
+      const int row = p.inv ? __ldcg(p.inv + a) : (int)a;  // no inv: rows by assignment
       const float4 y = __ldcg(reinterpret_cast<const float4*>(p.y_perm + (size_t)row * p.H + h));
       acc.x = fmaf(w, y.x, acc.x);
       acc.y = fmaf(w, y.y, acc.y);

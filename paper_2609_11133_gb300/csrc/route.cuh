@@ -79,7 +79,7 @@ struct GatherParams {
 struct CombineParams {
   const float* y_perm;
   const float* topk_w;
-  const int* inv;
+  const int* inv;  // row of y_perm of each assignment, or null: row a = assignment a
   int T, k, H;
   const __nv_bfloat16* residual;
   __nv_bfloat16* out;

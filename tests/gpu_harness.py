@@ -36,7 +36,7 @@ class Case:
         """One moe_decode_layer_ex call (on `ws` if given, else a new zeroed
         workspace); the device status must be clean afterwards."""
         T, H, E, k = self.T, self.H, self.E, self.k
-        n = binding.moe_workspace_size(self.w, T, k)
+        n = binding.moe_workspace_size(self.w, T, k, self.flags)
         self.ws = binding.alloc_workspace(n) if ws is None else ws
         self.out = torch.empty((T, H), dtype=torch.bfloat16, device="cuda") if out is None else out
         self.logits = torch.empty((T, E), dtype=torch.float32, device="cuda")

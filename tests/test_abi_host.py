@@ -122,3 +122,34 @@ def test_layer_kernel_count(lib):
     assert count(fake_weights(fmt=3), 4, 2)[0] == -1
     assert count(fake_weights(E=600), 4, 2)[0] == -2
     assert lib.moe_layer_kernel_count(ctypes.byref(fake_weights()), 4, 2, None) == -1
+
+
+def test_deterministic_flag_sizes_the_workspace(lib):
+    """MOE_FLAG_DETERMINISTIC keeps one fp32 down row per assignment: T*k*H*4
+    more bytes (256-byte aligned) unless the batch is prefill-shaped NVFP4,
+    whose engine keeps them anyway; the other flags add nothing."""
+    DET = binding.MOE_FLAG_DETERMINISTIC
+
+    def size(c, T, k, flags):
+        n = ctypes.c_size_t(0)
+        rc = lib.moe_workspace_size_flags(ctypes.byref(c), T, k, flags, ctypes.byref(n))
+        return rc, n.value
+
+    for fmt, E, H, I, T, k in ((1, 8, 512, 256, 4, 2), (2, 8, 512, 256, 1, 1),
+                               (1, 160, 6144, 2560, 64, 8), (2, 128, 4096, 1536, 64, 8)):
+        c = fake_weights(fmt=fmt, E=E, H=H, I=I)
+        rc0, n0 = ws_size(lib, c, T, k)
+        assert rc0 == 0 and size(c, T, k, 0) == (0, n0)
+        assert size(c, T, k, binding.MOE_FLAG_NO_RENORM | binding.MOE_FLAG_PRENORM_RMS) == (0, n0)
+        rc1, n1 = size(c, T, k, DET)
+        assert rc1 == 0 and n1 - n0 == (T * k * H * 4 + 255) // 256 * 256
+    c = fake_weights(fmt=2, E=8)
+    assert size(c, 100, 8, DET) == size(c, 100, 8, 0)  # prefill-shaped: rows kept anyway
+    assert size(c, 4, 2, 0x40)[0] == -1
+    assert lib.moe_workspace_size_flags(ctypes.byref(c), 4, 2, DET, None) == -1
+    # the decode layer asks for the larger size when it gets the flag
+    c = fake_weights()
+    _, n0 = ws_size(lib, c, 4, 2)
+    P = ctypes.c_void_p
+    assert lib.moe_decode_layer(P(0x100000), P(0x200000), None, ctypes.byref(c), 4, 2, DET,
+                                None, P(0x300000), P(0x400000), n0, None) == -3
