@@ -254,7 +254,7 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
  *     moe_workspace_size_flags() exceeds 16 MiB return MOE_ERR_WORKSPACE_TOO_SMALL:
  *     the 235B-shaped NVFP4 layer (H=4096, E=128, k=8, I=1536) fits up to
  *     T = 74 tokens, the 480B-shaped FP8 layer (H=6144, E=160, k=8, I=2560)
- *     up to T = 64 (without MOE_FLAG_DETERMINISTIC).
+ *     up to T = 64; with MOE_FLAG_DETERMINISTIC up to T = 59 and T = 38.
  *   The first call on a device looks up the array's device address and
  *     clears the array's status word; make that first call before capturing
  *     the stream into a CUDA graph.  A lookup that fails returns MOE_ERR_CUDA
