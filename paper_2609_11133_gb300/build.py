@@ -17,8 +17,8 @@ ROOT = os.path.dirname(HERE)
 SRC_DIR = os.path.join(HERE, "csrc")
 OUT_DIR = os.path.join(HERE, "_build")
 LIB_PATH = os.path.join(OUT_DIR, "libmoe.so")
-SOURCES = ["abi.cu", "route.cu", "ffn_fp8.cu", "ffn_nvfp4.cu", "ffn_bs.cu", "ffn_f8tc.cu",
-           "ffn_pf.cu", "noalloc.cu"]
+SOURCES = ["abi.cu", "route.cu", "route_tc.cu", "ffn_fp8.cu", "ffn_nvfp4.cu", "ffn_bs.cu",
+           "ffn_f8tc.cu", "ffn_pf.cu", "noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 CFLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
           "-I", os.path.join(ROOT, "include")]

@@ -170,6 +170,24 @@ int route_epb(int T, int E, int sms) {
   return (long long)((E + 3) / 4) * chunks > 2LL * sms ? 8 : 4;
 }
 
+// Batches with T * H >= kRouteTcMinTH (E <= 256) compute the router logits on
+// the tensor cores (route_tc.cu).  Measured (route and gather, us, GEMV ->
+// tensor cores): H=4096 T=256 51.7 -> 60.4, T=512 76.5 -> 68.1, T=1024 125.8
+// -> 81.0, T=2048 238.2 -> 134.6; H=6144 T=256 71.8 -> 70.5, T=512 114.2 ->
+// 87.4.  MOE_ROUTE_TC=0 keeps every batch on the CUDA-core GEMV of
+// route_kernel, MOE_ROUTE_TC=1 sends every batch with E <= 256 to the tensor
+// cores (for comparisons).
+constexpr long long kRouteTcMinTH = 1LL << 21;
+bool use_route_tc(int T, int H, int E) {
+  static int mode = -2;  // -1 default, 0 off, 1 on
+  if (mode == -2) {
+    const char* s = std::getenv("MOE_ROUTE_TC");
+    mode = !s ? -1 : (std::strcmp(s, "0") == 0 ? 0 : (std::strcmp(s, "1") == 0 ? 1 : -1));
+  }
+  if (E > kRouteTcMaxE || mode == 0) return false;
+  return mode == 1 || (long long)T * H >= kRouteTcMinTH;
+}
+
 // Prefill-shaped NVFP4 batches run on the prefill engine (ffn_pf.cuh);
 // MOE_PF=0 keeps them on the decode engine (for comparisons).
 bool use_prefill(int T, int k, int E, int eng) {
@@ -215,7 +233,7 @@ constexpr int kLayerFlags =
 // down row per assignment (the prefill engine keeps them anyway).
 WsLayout layer_layout(const moe_expert_weights_t* w, int T, int k, int flags) {
   return ws_layout(T, k, w->E, w->H, w->I, act_for(w->fmt, engine_for(w->fmt)),
-                   (flags & MOE_FLAG_DETERMINISTIC) != 0);
+                   (flags & MOE_FLAG_DETERMINISTIC) != 0, use_route_tc(T, w->H, w->E));
 }
 
 // ------------------------------------------------------------------ the expert steps
@@ -418,7 +436,7 @@ int run_prefill(const moe_expert_weights_t* w, int T, int k, int sms, void* ws,
   p2.bsf = ws_ptr<uint8_t>(ws, L.hsf);
   if (launch_ffn_pf(sms, m1, p1, st) != cudaSuccess) return MOE_ERR_CUDA;
   if (ev_mid && cudaEventRecord(ev_mid, st) != cudaSuccess) return MOE_ERR_CUDA;
-  if (launch_swiglu_terms(T * k, sms, p1, st) != cudaSuccess) return MOE_ERR_CUDA;
+  if (launch_swiglu_terms(T * k, sms, p1, st, kPfTerms) != cudaSuccess) return MOE_ERR_CUDA;
   if (launch_ffn_pf(sms, m2, p2, st) != cudaSuccess) return MOE_ERR_CUDA;
   CombineParams c{p2.y_perm, gates, ws_ptr<int>(ws, L.inv), T, k, H,
                   static_cast<const __nv_bfloat16*>(residual), static_cast<__nv_bfloat16*>(out),
@@ -468,8 +486,10 @@ int moe_layer_kernel_count(const moe_expert_weights_t* w, int T, int k, int* cou
   if (rc) return rc;
   rc = check_tk(T, k, w->E);
   if (rc) return rc;
-  // route, (gather), gate/up, SwiGLU, down, finalize
-  *count = (T == 0) ? 0 : 5 + (gather_terms(T, act_for(w->fmt, engine_for(w->fmt))) ? 1 : 0);
+  // (router prep and GEMM), route, (gather), gate/up, SwiGLU, down, finalize
+  *count = (T == 0) ? 0
+                    : 5 + (gather_terms(T, act_for(w->fmt, engine_for(w->fmt))) ? 1 : 0) +
+                          (use_route_tc(T, w->H, w->E) ? 2 : 0);
   return MOE_OK;
 }
 
@@ -532,7 +552,7 @@ int moe_read_status(void* ws, size_t ws_bytes, int* status, void* stream) {
     if (cudaMemsetAsync(ws, 0, 4, st) != cudaSuccess || cudaStreamSynchronize(st) != cudaSuccess)
       return MOE_ERR_CUDA;
   }
-  if (word & (kStatusTimeoutGateUp | kStatusTimeoutDown))
+  if (word & (kStatusTimeoutGateUp | kStatusTimeoutDown | kStatusTimeoutRoute))
     *status = MOE_ERR_DEVICE_TIMEOUT;
   else if (word & kStatusBadExpertId)
     *status = MOE_ERR_BAD_EXPERT_ID;
@@ -730,6 +750,44 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
   p.acnt = ws_ptr<unsigned>(ws, L.acnt);
   p.alist = ws_ptr<int>(ws, L.alist);
   if (ev[0] && cudaEventRecord(ev[0], st) != cudaSuccess) return MOE_ERR_CUDA;
+  if (use_route_tc(T, H, E)) {
+    // logits on the tensor cores; route_kernel adds the slices and routes
+    RouteTcParams q{};
+    q.wr = router_w;
+    q.x = p.x;
+    q.xn = ws_ptr<__nv_bfloat16>(ws, L.xn);
+    q.w3 = ws_ptr<__nv_bfloat16>(ws, L.w3);
+    q.plog = ws_ptr<float>(ws, L.plog);
+    q.T = T;
+    q.H = H;
+    q.E = E;
+    q.Ep = route_tc_ep(E);
+    q.prenorm = p.prenorm;
+    q.status = ws_ptr<uint32_t>(ws, L.status);
+    q.wait_ns = wait_limit_ns();
+    CUtensorMap ta, tb;
+    if (!map_2d(&ta, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, q.prenorm ? (const void*)q.xn : x,
+                (uint64_t)H, (uint64_t)T, (uint64_t)H * 2, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !map_2d(&tb, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, q.w3, (uint64_t)H, 3 * (uint64_t)q.Ep,
+                (uint64_t)H * 2, 64, (uint32_t)q.Ep, CU_TENSOR_MAP_SWIZZLE_128B))
+      return MOE_ERR_CUDA;
+    if (launch_router_prep(q, st) != cudaSuccess || launch_route_tc(ta, tb, q, st) != cudaSuccess)
+      return MOE_ERR_CUDA;
+    p.plog = q.plog;
+    p.nsplit = kRouteTcSplit;
+    p.ep = q.Ep;
+    // without the GEMV a CTA's work is the chunk's staging, its share of the
+    // activation terms and of the zeroing, and the partial sums of its
+    // experts: about one wave of CTAs, each chunk's experts split between them
+    const int chunks = (T + kRouteTok - 1) / kRouteTok;
+    int per = (sms + chunks - 1) / chunks;
+    per = per < 1 ? 1 : (per > (E + 3) / 4 ? (E + 3) / 4 : per);
+    p.epb = (E + per - 1) / per;
+    if (p.prenorm) {  // the router kernel stages the normalised rows
+      p.x = q.xn;
+      p.prenorm = 0;
+    }
+  }
   if (launch_route(p, st) != cudaSuccess) return MOE_ERR_CUDA;
   const bool gathered = gather_terms(T, p.act);
   if (gathered) {

@@ -67,12 +67,13 @@ __device__ __forceinline__ uint32_t e2m1x8_from_f32(const float* q) {
 }
 
 // Encode one 16-element block r (already scaled by the row's power of two)
-// into kTerms terms: codes[t] (16 E2M1 codes, 8 bytes) and sf[t] (UE4M3).
-// r is consumed (it ends as the final residual).
+// into its first NTERM terms (of kTerms): codes[t] (16 E2M1 codes, 8 bytes)
+// and sf[t] (UE4M3).  r is consumed (it ends as the residual).
+template <int NTERM = kTerms>
 __device__ __forceinline__ void encode_terms16(float (&r)[16], uint2 (&codes)[kTerms],
                                                uint32_t (&sf)[kTerms]) {
 #pragma unroll
-  for (int t = 0; t < kTerms; ++t) {
+  for (int t = 0; t < NTERM; ++t) {
     float m = 0.f;
 #pragma unroll
     for (int i = 0; i < 16; ++i) m = fmaxf(m, fabsf(r[i]));
@@ -163,11 +164,12 @@ __device__ __forceinline__ void store_terms16_quad(const uint32_t (&part)[kTerms
 
 // Write block b of a row's terms: row r of the term arrays is token/assignment
 // `row4 / kTerms`, term `row4 % kTerms`; q rows are K/2 bytes, sf rows K/16.
+template <int NTERM = kTerms>
 __device__ __forceinline__ void store_terms16(const uint2 (&codes)[kTerms],
                                               const uint32_t (&sf)[kTerms], uint8_t* q,
                                               uint8_t* sfp, size_t row4, int K, int b) {
 #pragma unroll
-  for (int t = 0; t < kTerms; ++t) {
+  for (int t = 0; t < NTERM; ++t) {
     *reinterpret_cast<uint2*>(q + (row4 + t) * (size_t)(K / 2) + 8 * b) = codes[t];
     sfp[(row4 + t) * (size_t)(K / 16) + b] = (uint8_t)sf[t];
   }

@@ -25,6 +25,16 @@ constexpr int kRouteWarps = 8;      // warps per router CTA
 constexpr uint32_t kStatusTimeoutGateUp = 1u;
 constexpr uint32_t kStatusTimeoutDown = 2u;
 constexpr uint32_t kStatusBadExpertId = 4u;
+constexpr uint32_t kStatusTimeoutRoute = 8u;
+
+// Tensor-core router (route_tc.cu), used for large batches: the logits as a
+// bf16 GEMM against the fp32 router split exactly into three bf16 parts, its
+// K range cut into kRouteTcSplit slices whose fp32 partial sums the router
+// kernel adds in slice order.  The slice count does not depend on T, so a
+// token's logits are the same in every batch that takes this router.
+constexpr int kRouteTcSplit = 8;
+constexpr int kRouteTcMaxE = 256;  // experts: one MMA N (a multiple of 16, <= 256)
+inline int route_tc_ep(int E) { return (E + 15) / 16 * 16; }
 
 // Bounded waits give up after this many nanoseconds of %globaltimer.
 constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s
@@ -74,6 +84,11 @@ struct WsLayout {
   // the decode engines keeps the down rows too (by assignment)
   size_t yperm;    // f32 [T*k, H]
   size_t inv;      // i32 [T*k]
+  // tensor-core router (zero-sized otherwise): the router's three bf16 parts,
+  // the partial logits of the K slices, and the pre-normalised rows of x
+  size_t w3;       // bf16 [3, Ep, H]
+  size_t plog;     // f32 [kRouteTcSplit, T, Ep]
+  size_t xn;       // bf16 [T, H]
   size_t total;
   int nChunks;
 };
@@ -102,7 +117,7 @@ inline bool prefill_shape(int T, int k, int E, int act) {
 }
 
 inline WsLayout ws_layout(int T, int k, int E, int H, int I, int act = kActF16,
-                          bool det = false) {
+                          bool det = false, bool tcr = false) {
   WsLayout L{};
   size_t o = 0;
   auto take = [&](size_t bytes) {
@@ -139,6 +154,10 @@ inline WsLayout ws_layout(int T, int k, int E, int H, int I, int act = kActF16,
   const size_t npf = prefill_shape(T, k, E, act) ? 1 : 0;
   L.yperm = take((npf || det ? 1 : 0) * 4 * TK * (size_t)H);
   L.inv = take(npf * 4 * TK);
+  const size_t nr = tcr ? 1 : 0, Ep = (size_t)route_tc_ep(E);
+  L.w3 = take(nr * 3 * Ep * H * 2);
+  L.plog = take(nr * kRouteTcSplit * (size_t)T * Ep * 4);
+  L.xn = take(nr * (size_t)T * H * 2);
   L.total = o;
   return L;
 }

@@ -36,12 +36,44 @@ cudaError_t launch_ffn_bs(int nt, int grid, const FfnMaps& m, const FfnParams& p
   }
 }
 
-cudaError_t launch_swiglu_terms(int rows, int sms, const FfnParams& p, cudaStream_t st) {
+// One wave of the rows kernel: every resident CTA takes the same number of
+// rows (within one), so none of them is left running alone at the end.
+template <typename K>
+static int resident_blocks(K kern, int sms, std::atomic<int>& cache) {
+  int per = cache.load();
+  if (per <= 0) {
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, kern, 128, 0) != cudaSuccess ||
+        per < 1)
+      per = 4;
+    cache.store(per);
+  }
+  return per * sms;
+}
+
+template <int G, int NTERM>
+static cudaError_t launch_rows_g(int sms, int rows, const FfnParams& p, cudaStream_t st) {
+  static std::atomic<int> per{0};
+  auto kern = swiglu_terms_rows_kernel<G, NTERM>;
+  int blocks = resident_blocks(kern, sms, per);
+  if (blocks > rows) blocks = rows;
+  return launch_pdl(kern, dim3(blocks), dim3(128), 0, st, p, rows);
+}
+
+template <int NTERM>
+static cudaError_t launch_rows(int sms, int rows, const FfnParams& p, cudaStream_t st) {
+  if (p.I <= 2048) return launch_rows_g<1, NTERM>(sms, rows, p, st);
+  if (p.I <= 4096) return launch_rows_g<2, NTERM>(sms, rows, p, st);
+  return launch_rows_g<4, NTERM>(sms, rows, p, st);
+}
+
+cudaError_t launch_swiglu_terms(int rows, int sms, const FfnParams& p, cudaStream_t st,
+                                int nterms) {
   int blocks = rows;
   if (blocks > 8 * sms) blocks = 8 * sms;
   if (blocks < 1) blocks = 1;
   if (rows > kSwigluQuadMaxRows)
-    return launch_pdl(swiglu_terms_rows_kernel, dim3(blocks), dim3(128), 0, st, p, rows);
+    return nterms == kPfTerms ? launch_rows<kPfTerms>(sms, rows, p, st)
+                              : launch_rows<kTerms>(sms, rows, p, st);
   return launch_pdl(swiglu_terms_kernel, dim3(blocks), dim3(kSwigluThreads), 0, st, p, rows);
 }
 

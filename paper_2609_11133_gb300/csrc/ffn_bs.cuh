@@ -557,21 +557,44 @@ static __global__ void __launch_bounds__(kSwigluThreads, 2) swiglu_terms_kernel(
 }
 
 // The same SwiGLU with one thread per 16-column block (encode_terms16 run
-// serially by that thread) in 128-thread CTAs: more rows in flight per SM
-// (five CTAs), which pays when there are many rows.  Same codes as the quad
-// kernel.
+// serially by that thread) in 128-thread CTAs, G blocks per thread (I <= 2048
+// G), for batches with many rows.  With one block per thread the next row's
+// gate|up values load while this row is encoded (with more, the registers
+// that would take cost more CTAs per SM than the overlap gains).  The row
+// maximum meets in a double-buffered shared array, one barrier per row.  The
+// first NTERM terms are written (the prefill engine reads three); the codes
+// are the quad kernel's.
+template <int G, int NTERM>
 static __global__ void __launch_bounds__(128) swiglu_terms_rows_kernel(const FfnParams p, int rows) {
-  constexpr int G = 4;  // blocks per thread (I <= 8192)
-  __shared__ float s_max[4];
+  __shared__ float s_max[2][4];
   // the down step may launch now: what it does before its own wait (plan,
   // weight copies) does not read this kernel's output
   pdl_launch_dependents();
   pdl_wait();
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int nb = p.I / 16;
-  for (int row = blockIdx.x; row < rows; row += gridDim.x) {
+  constexpr bool kAhead = (G == 1);
+  float4 ng[4], nu[4];  // kAhead: the next row's gate and up values of this thread's block
+  auto load_ahead = [&](int row) {
+    const float* g = p.gu + (size_t)row * 2 * p.I + 16 * threadIdx.x;
+    if (row < rows && (int)threadIdx.x < nb) {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        ng[i] = __ldcg(reinterpret_cast<const float4*>(g + 4 * i));
+        nu[i] = __ldcg(reinterpret_cast<const float4*>(g + p.I + 4 * i));
+      }
+    }
+  };
+  auto silu4 = [](float4 gv, float4 uv, float* h) {
+    h[0] = gv.x / (1.f + expf(-gv.x)) * uv.x;
+    h[1] = gv.y / (1.f + expf(-gv.y)) * uv.y;
+    h[2] = gv.z / (1.f + expf(-gv.z)) * uv.z;
+    h[3] = gv.w / (1.f + expf(-gv.w)) * uv.w;
+  };
+  if (kAhead) load_ahead(blockIdx.x);
+  int par = 0;
+  for (int row = blockIdx.x; row < rows; row += gridDim.x, par ^= 1) {
     const float* g = p.gu + (size_t)row * 2 * p.I;
-    const float* u = g + p.I;
     float h[G][16];
     float amax = 0.f;
 #pragma unroll
@@ -579,22 +602,23 @@ static __global__ void __launch_bounds__(128) swiglu_terms_rows_kernel(const Ffn
       const int b = threadIdx.x + 128 * q;
       if (b < nb) {
 #pragma unroll
-        for (int i = 0; i < 16; i += 4) {
-          const float4 gv = __ldcg(reinterpret_cast<const float4*>(g + 16 * b + i));
-          const float4 uv = __ldcg(reinterpret_cast<const float4*>(u + 16 * b + i));
-          h[q][i + 0] = gv.x / (1.f + expf(-gv.x)) * uv.x;
-          h[q][i + 1] = gv.y / (1.f + expf(-gv.y)) * uv.y;
-          h[q][i + 2] = gv.z / (1.f + expf(-gv.z)) * uv.z;
-          h[q][i + 3] = gv.w / (1.f + expf(-gv.w)) * uv.w;
+        for (int i = 0; i < 4; ++i) {
+          if (kAhead) {
+            silu4(ng[i], nu[i], &h[q][4 * i]);
+          } else {
+            silu4(__ldcg(reinterpret_cast<const float4*>(g + 16 * b + 4 * i)),
+                  __ldcg(reinterpret_cast<const float4*>(g + p.I + 16 * b + 4 * i)), &h[q][4 * i]);
+          }
         }
 #pragma unroll
         for (int i = 0; i < 16; ++i) amax = fmaxf(amax, fabsf(h[q][i]));
       }
     }
+    if (kAhead) load_ahead(row + gridDim.x);
     amax = warp_max(amax);
-    if (lane == 0) s_max[warp] = amax;
-    __syncthreads();
-    amax = fmaxf(fmaxf(s_max[0], s_max[1]), fmaxf(s_max[2], s_max[3]));
+    if (lane == 0) s_max[par][warp] = amax;
+    __syncthreads();  // a warp reaches the next row's barrier only after this row's reads
+    amax = fmaxf(fmaxf(s_max[par][0], s_max[par][1]), fmaxf(s_max[par][2], s_max[par][3]));
     const float sc = pow2_scale_terms(amax);
 #pragma unroll
     for (int q = 0; q < G; ++q) {
@@ -604,12 +628,11 @@ static __global__ void __launch_bounds__(128) swiglu_terms_rows_kernel(const Ffn
         for (int i = 0; i < 16; ++i) h[q][i] *= sc;
         uint2 codes[kTerms];
         uint32_t sf[kTerms];
-        encode_terms16(h[q], codes, sf);
-        store_terms16(codes, sf, p.hq, p.hsf, (size_t)row * kTerms, p.I, b);
+        encode_terms16<NTERM>(h[q], codes, sf);
+        store_terms16<NTERM>(codes, sf, p.hq, p.hsf, (size_t)row * kTerms, p.I, b);
       }
     }
     if (threadIdx.x == 0) p.hinv[row] = 1.f / sc;
-    __syncthreads();  // s_max is reused by the next row
   }
 }
 

@@ -47,7 +47,11 @@ cudaError_t launch_finalize(int sms, const FfnParams& p, cudaStream_t st);
 // ffn_bs.cu); nt in {8, 16}.  SwiGLU into NVFP4 terms for its down step.
 cudaError_t launch_ffn_bs(int nt, int grid, const FfnMaps& maps, const FfnParams& p,
                           cudaStream_t st);
-cudaError_t launch_swiglu_terms(int rows, int sms, const FfnParams& p, cudaStream_t st);
+// SwiGLU into NVFP4 terms; batches of more than kSwigluQuadMaxRows rows may
+// write only the first `nterms` of the four terms (the prefill engine reads
+// kPfTerms).
+cudaError_t launch_swiglu_terms(int rows, int sms, const FfnParams& p, cudaStream_t st,
+                                int nterms = 4);
 
 // The FP8 tcgen05 engine (ffn_f8.cuh, instantiated in ffn_f8tc.cu); nt in
 // {8, 16, 32}.  SwiGLU into E4M3 terms for its down step.

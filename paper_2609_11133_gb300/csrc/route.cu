@@ -399,6 +399,7 @@ __global__ void __launch_bounds__(256) route_kernel(const RouteParams p) {
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int chunk = blockIdx.y, eb = blockIdx.x;
+  if (p.plog) pdl_wait();  // the GEMM's partial logits (and xn) are complete
   pdl_launch_dependents();  // the expert kernel may start its prologue now
   const int t0 = chunk * kRouteTok;
   const int nt = min(kRouteTok, p.T - t0);
@@ -427,17 +428,8 @@ __global__ void __launch_bounds__(256) route_kernel(const RouteParams p) {
   }
   __syncthreads();
   if (p.prenorm && warp < nt) {
-    // bf16(x / sqrt(mean(x^2) + eps)), unit weight
     __nv_bfloat16* row = xs + (size_t)warp * H;
-    float ss = 0.f;
-    for (int h = lane; h < H; h += 32) {
-      const float v = __bfloat162float(row[h]);
-      ss = fmaf(v, v, ss);
-    }
-    ss = warp_sum(ss);
-    const float r = 1.f / sqrtf(ss / (float)H + 1e-6f);
-    __syncwarp();
-    for (int h = lane; h < H; h += 32) row[h] = __float2bfloat16_rn(__bfloat162float(row[h]) * r);
+    rms_norm_row_bf16(row, row, H, lane);
   }
   __syncthreads();
   if (p.fused) {
@@ -460,7 +452,20 @@ __global__ void __launch_bounds__(256) route_kernel(const RouteParams p) {
   // in warp order.
   __shared__ float s_part[kRouteWarps][32];
   const int nexp = min(p.epb, E - eb * p.epb);  // experts of this CTA
-  for (int q0 = 0; q0 < nexp; q0 += 4) {
+  if (p.plog) {
+    // the tensor-core router's partial logits of this chunk and these
+    // experts, added in slice order
+    const size_t slice = (size_t)p.T * p.ep;
+    for (int i = threadIdx.x; i < nt * nexp; i += blockDim.x) {
+      const int t = i / nexp, e = eb * p.epb + (i - t * nexp);
+      const float* q = p.plog + (size_t)(t0 + t) * p.ep + e;
+      float sum = __ldcg(q);
+      for (int j = 1; j < p.nsplit; ++j) sum += __ldcg(q + j * slice);
+      const float b = p.bias ? __ldg(p.bias + e) : 0.f;
+      p.logits[(size_t)(t0 + t) * E + e] = sum + b;
+    }
+  }
+  for (int q0 = 0; q0 < (p.plog ? 0 : nexp); q0 += 4) {
     constexpr int MAXEPB = 4;
     const int e0 = eb * p.epb + q0;
     const int nq = min(MAXEPB, nexp - q0);  // experts of this round
@@ -610,48 +615,85 @@ __global__ void __launch_bounds__(256) prep_kernel(const PrepParams p) {
       p.counts[e] = __ldg(p.offsets + e + 1) - __ldg(p.offsets + e);
 }
 
-// grid (E, ceil(T/8)): CTA (e, g) copies list positions 8g..8g+7 of expert e.
+// grid ceil(T*k / 8): CTA b copies compact rows 8b..8b+7.  Compact row r is
+// position r - pre[e] of expert e's list, pre the exclusive prefix of the
+// per-expert counts (every CTA scans the counts; E <= 512).
 __global__ void __launch_bounds__(256) gather_kernel(const GatherParams p) {
-  __shared__ int s_off;
-  __shared__ int s_tok[8];
+  __shared__ int s_pre[kMaxE + 1];
+  __shared__ int s_tok[8], s_row[8];
   pdl_wait();  // the routing that wrote the lists is complete
   pdl_launch_dependents();
-  const int e = blockIdx.x, g0 = blockIdx.y * 8;
-  const int n_e = (int)__ldcg(p.acnt + e);
-  if (g0 >= n_e) return;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (warp == 0) {  // first compact row of expert e: the counts of the experts before it
-    int sum = 0;
-    for (int i = lane; i < e; i += 32) sum += (int)__ldcg(p.acnt + i);
+  if (warp == 0) {
+    constexpr int PER = kMaxE / 32;  // counts per lane
+    int c[PER], run = 0;
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
-    if (lane == 0) s_off = sum;
-  }
-  const int nj = min(8, n_e - g0);
-  int a_own = -1;  // thread j < nj: the assignment at list position g0 + j
-  if (threadIdx.x < nj) {
-    a_own = __ldcg(p.alist + (size_t)e * p.T + g0 + threadIdx.x);
-    s_tok[threadIdx.x] = a_own / p.k;
+    for (int i = 0; i < PER; ++i) {
+      const int e = lane * PER + i;
+      c[i] = e < p.E ? (int)__ldcg(p.acnt + e) : 0;
+      run += c[i];
+    }
+    int inc = run;  // inclusive scan of the lanes' sums
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, inc, o);
+      if (lane >= o) inc += y;
+    }
+    int pre = inc - run;
+#pragma unroll
+    for (int i = 0; i < PER; ++i) {
+      s_pre[lane * PER + i] = pre;
+      pre += c[i];
+    }
+    if (lane == 31) s_pre[kMaxE] = pre;
   }
   __syncthreads();
-  // its compact row (prefill engine: the combine kernel reads each
-  // assignment's down row there)
-  if (p.inv && a_own >= 0) p.inv[a_own] = s_off + g0 + threadIdx.x;
-  const int q16 = p.terms * p.qrow / 16;  // 16-byte units of one token's term rows
-  for (int i = threadIdx.x; i < nj * q16; i += blockDim.x) {
-    const int j = i / q16, u = i - j * q16;
-    const uint4 v = __ldcg(reinterpret_cast<const uint4*>(p.q + (size_t)s_tok[j] * p.terms * p.qrow) + u);
-    reinterpret_cast<uint4*>(p.gq + (size_t)(s_off + g0 + j) * p.terms * p.qrow)[u] = v;
-  }
-  if (p.sf) {
-    const int s16 = p.terms * p.sfrow / 16;
-    for (int i = threadIdx.x; i < nj * s16; i += blockDim.x) {
-      const int j = i / s16, u = i - j * s16;
-      const uint4 v =
-          __ldcg(reinterpret_cast<const uint4*>(p.sf + (size_t)s_tok[j] * p.terms * p.sfrow) + u);
-      reinterpret_cast<uint4*>(p.gsf + (size_t)(s_off + g0 + j) * p.terms * p.sfrow)[u] = v;
+  const int total = s_pre[kMaxE];
+  const int r0 = blockIdx.x * 8;
+  const int nj = min(8, total - r0);
+  if (nj <= 0) return;
+  if (threadIdx.x < nj) {
+    const int r = r0 + threadIdx.x;
+    int lo = 0, hi = p.E - 1;  // the last expert whose list starts at or before r
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (s_pre[mid] <= r) lo = mid; else hi = mid - 1;
     }
+    const int a = __ldcg(p.alist + (size_t)lo * p.T + (r - s_pre[lo]));
+    s_tok[threadIdx.x] = a / p.k;
+    s_row[threadIdx.x] = r;
+    // its compact row (prefill engine: the combine kernel reads each
+    // assignment's down row there)
+    if (p.inv) p.inv[a] = r;
   }
+  __syncthreads();
+  // 16-byte units, eight loads in flight per thread before their stores
+  auto copy = [&](const uint8_t* src, uint8_t* dst, int row_bytes) {
+    const int u16 = row_bytes / 16;  // units of one token's term rows
+    const int n = nj * u16;
+    constexpr int B = 8;
+    for (int base = 0; base < n; base += B * 256) {
+      uint4 v[B];
+#pragma unroll
+      for (int q = 0; q < B; ++q) {
+        const int i = base + q * 256 + threadIdx.x;
+        if (i < n) {
+          const int j = i / u16, u = i - j * u16;
+          v[q] = __ldcg(reinterpret_cast<const uint4*>(src + (size_t)s_tok[j] * row_bytes) + u);
+        }
+      }
+#pragma unroll
+      for (int q = 0; q < B; ++q) {
+        const int i = base + q * 256 + threadIdx.x;
+        if (i < n) {
+          const int j = i / u16, u = i - j * u16;
+          reinterpret_cast<uint4*>(dst + (size_t)s_row[j] * row_bytes)[u] = v[q];
+        }
+      }
+    }
+  };
+  copy(p.q, p.gq, p.terms * p.qrow);
+  if (p.sf) copy(p.sf, p.gsf, p.terms * p.sfrow);
 }
 
 __global__ void __launch_bounds__(256) combine_kernel(const CombineParams p) {
@@ -705,6 +747,22 @@ cudaError_t launch_route(const RouteParams& p, cudaStream_t st) {
   const size_t smem = route_smem_bytes(p.H, p.E);
   cudaError_t err = set_smem_once(route_kernel, (int)route_smem_bytes(8192, kMaxE), done);
   if (err != cudaSuccess) return err;
+  if (p.plog) {
+    // after the tensor-core router's GEMM, launched as a programmatic
+    // dependent (it waits for the GEMM before it reads)
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)((p.E + p.epb - 1) / p.epb),
+                       (unsigned)((p.T + kRouteTok - 1) / kRouteTok));
+    cfg.blockDim = dim3(256);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, route_kernel, p);
+  }
   dim3 grid((p.E + p.epb - 1) / p.epb, (p.T + kRouteTok - 1) / kRouteTok);
   route_kernel<<<grid, 256, smem, st>>>(p);
   return cudaGetLastError();
@@ -712,7 +770,7 @@ cudaError_t launch_route(const RouteParams& p, cudaStream_t st) {
 
 cudaError_t launch_gather(const GatherParams& p, cudaStream_t st) {
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)p.E, (unsigned)((p.T + 7) / 8));
+  cfg.gridDim = dim3((unsigned)(((size_t)p.T * p.k + 7) / 8));
   cfg.blockDim = dim3(256);
   cfg.stream = st;
   cudaLaunchAttribute attr[1];

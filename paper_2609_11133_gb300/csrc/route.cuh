@@ -10,7 +10,9 @@
 //   fused layer it also appends each assignment to its expert's list (an
 //   atomic counter per expert), from which the expert kernels build their
 //   work plan.  Tickets and counters are reset by their last user; nothing
-//   waits on another CTA.
+//   waits on another CTA.  Batches routed on the tensor cores (route_tc.cu)
+//   run the same grid after the GEMM: each CTA adds the GEMM's partial logits
+//   of its experts in slice order instead of the GEMV.
 #pragma once
 
 #include "common.cuh"
@@ -20,12 +22,28 @@ namespace moe {
 constexpr int kMaxK = 32;
 
 
+// bf16(x / sqrt(mean(x^2) + eps)) of one row by one warp (unit weight, eps
+// 1e-6); `out` may be `in`.  The router kernel and the tensor-core router's
+// prep kernel both normalise with it, so their rows have the same bits.
+__device__ __forceinline__ void rms_norm_row_bf16(const __nv_bfloat16* in, __nv_bfloat16* out,
+                                                  int H, int lane) {
+  float ss = 0.f;
+  for (int h = lane; h < H; h += 32) {
+    const float v = __bfloat162float(in[h]);
+    ss = fmaf(v, v, ss);
+  }
+  ss = warp_sum(ss);
+  const float r = 1.f / sqrtf(ss / (float)H + 1e-6f);
+  __syncwarp();
+  for (int h = lane; h < H; h += 32) out[h] = __float2bfloat16_rn(__bfloat162float(in[h]) * r);
+}
+
 struct RouteParams {
   const __nv_bfloat16* x;
   const float* wr;
   const float* bias;
   int T, H, E, k, renorm, prenorm, fmt, fused;
-  int epb;  // experts per CTA (1 to 4)
+  int epb;  // experts per CTA (1, 4 or 8; any count with plog)
   int act;  // activation form for the expert kernels (kAct*)
   float* logits;  // [T, E]
   int* ids;       // [T, k]
@@ -44,6 +62,24 @@ struct RouteParams {
   size_t zero_b_n4;
   unsigned* acnt;  // [E] assignments per expert, zero on entry
   int* alist;      // [E, T] expert e's assignments t*k + j at alist[e*T + 0..]
+  // logits from the tensor-core router: partial sums [nsplit, T, ep] added in
+  // slice order (one CTA per token chunk, no GEMV here); null: the GEMV here
+  const float* plog;
+  int nsplit, ep;
+};
+
+// The tensor-core router's two kernels (route_tc.cu): router_prep_kernel
+// splits the fp32 router rows into three bf16 parts (and writes the
+// RMS-normalised rows of x when prenorm), route_tc_kernel multiplies.
+struct RouteTcParams {
+  const float* wr;          // [E, H]
+  const __nv_bfloat16* x;   // [T, H] (the prep kernel's input when prenorm)
+  __nv_bfloat16* xn;        // [T, H] normalised rows (prenorm), else unused
+  __nv_bfloat16* w3;        // [3, Ep, H]: wr = w3[0] + w3[1] + w3[2]; rows >= E zero
+  float* plog;              // [kRouteTcSplit, T, Ep]
+  int T, H, E, Ep, prenorm;
+  uint32_t* status;
+  uint64_t wait_ns;
 };
 
 struct PrepParams {
@@ -95,5 +131,9 @@ cudaError_t launch_prep(const PrepParams& p, cudaStream_t st);
 cudaError_t launch_combine(const CombineParams& p, cudaStream_t st);
 cudaError_t launch_gather(const GatherParams& p, cudaStream_t st);
 size_t route_smem_bytes(int H, int E);
+cudaError_t launch_router_prep(const RouteTcParams& p, cudaStream_t st);
+// tmA: rows of x (or xn), tmB: rows of w3; both bf16 boxes of 64 x rows, 128B swizzle
+cudaError_t launch_route_tc(const CUtensorMap& tmA, const CUtensorMap& tmB,
+                            const RouteTcParams& p, cudaStream_t st);
 
 }  // namespace moe

@@ -113,11 +113,16 @@ def test_layer_kernel_count(lib):
         return rc, n.value
 
     # route, gate/up, SwiGLU, down and finalize; the gather of the activation
-    # terms joins above 64 tokens
+    # terms joins above 64 tokens, the tensor-core router's prep and GEMM from
+    # T * H >= 2^21 when E <= 256
     for fmt in (1, 2):
         assert count(fake_weights(fmt=fmt), 0, 2) == (0, 0)
         assert count(fake_weights(fmt=fmt), 64, 2) == (0, 5)
         assert count(fake_weights(fmt=fmt), 65, 2) == (0, 6)
+        assert count(fake_weights(fmt=fmt, H=4096), 511, 2) == (0, 6)
+        assert count(fake_weights(fmt=fmt, H=4096), 512, 2) == (0, 8)
+        assert count(fake_weights(fmt=fmt, H=6144), 342, 2) == (0, 8)
+        assert count(fake_weights(fmt=fmt, H=4096, E=257), 512, 2) == (0, 6)
     assert count(fake_weights(), 4, 0)[0] == -1
     assert count(fake_weights(fmt=3), 4, 2)[0] == -1
     assert count(fake_weights(E=600), 4, 2)[0] == -2
