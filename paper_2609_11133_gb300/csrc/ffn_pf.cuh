@@ -4,44 +4,49 @@
 // The decode engine (ffn_bs.cuh) cuts an expert's tokens into chunks of 8-16
 // and reads each weight tile once per chunk; with ~128 tokens per expert that
 // re-stages every tile eight times and the kernel is bound by the traffic
-// between L2 and shared memory.  Here an item is one 128-row weight tile
-// against a group of up to kPfTok = 64 tokens, over the whole K range:
+// into each SM.  Here an item is two adjacent 128-row weight tiles against a
+// group of up to kPfTok = 64 tokens, over the whole K range:
 //
 //   * N = 3 x 64 = 192: the first kPfTerms = 3 of the four NVFP4 terms that
 //     encode each activation row (act_terms.cuh).  Three terms leave a block
 //     residual below ~1/216 of its maximum; the layer output stays within
-//     ~2e-3 of the exact result (four terms would need N = 256 for 64 tokens
-//     and leave no tensor memory for a second stage of scales).  One 3-D TMA
-//     box copies terms 0-2 of the group's 64 compact rows: B row 3j + t is
-//     term t of the group's token j.
-//   * Whole K per item: the partial sums are complete in the accumulator, so
+//     ~2e-3 of the exact result.  One 3-D TMA box copies terms 0-2 of the
+//     group's 64 compact rows: B row 3j + t is term t of the group's token j.
+//   * Two weight tiles per item, two MMAs per K step against the same
+//     activation box: a stage brings 63 KB (two 16 KB weight boxes and their
+//     scales, 24 KB of activation rows and theirs) for 256 x 192 outputs.
+//     The engine is bound by the bytes each SM can take in (about 70 GB/s
+//     with three or four stages in flight); one tile per item brought 45 KB
+//     for half the outputs.
+//   * Whole K per item: the partial sums are complete in the accumulators, so
 //     the epilogue stores them (no atomics, no zeroing): phase 1 the gate or
 //     up pre-activations, phase 2 each assignment's down row (y_perm, summed
 //     over a token's experts by the combine kernel).
-//   * Items (active expert, token group, matrix, row tile), dealt round-robin
-//     (CTA c takes items c, c + G, c + 2G, ...): at any moment the grid works
-//     on ~G consecutive items, two or three experts, so a group's activation
-//     rows (read by every tile of its expert) and a tile (read by both groups
-//     of its expert, evict-last until the last group) stay in L2.  Contiguous
-//     shares had the CTAs on ~90 experts at once, whose activation rows (134
-//     MB of terms at 2048 tokens) do not fit in L2.
+//   * Items (active expert, token group, matrix, tile pair), dealt
+//     round-robin (CTA c takes items c, c + G, c + 2G, ...): at any moment
+//     the grid works on ~G consecutive items, a few experts, so a group's
+//     activation rows (read by every tile of its expert) and a tile (read by
+//     both groups of its expert, evict-last until the last group) stay in L2.
 //
-// Roles (352 threads) as in ffn_bs.cuh: warps 0-3 write the stage's scales
-// into tensor memory (A: 128 rows of 16 B, B: 192 rows of 16 B, both from
-// shared memory), warps 4-7 are the epilogue (TMEM lane quadrant = warp % 4),
-// warp 8 the lead producer (weight box and its scales), warp 9 the MMA
-// issuer, warp 10 the second producer (the activation box and its scales:
-// 3-D boxes of three terms of 64 rows, one for codes and one for scales).
-// With 192 B rows per stage, B scales loaded by the scale writers from global
-// memory paced the whole ring at one L2 round trip per stage.
-// One accumulator (192 columns) is in flight: the MMA issuer waits for the
-// epilogue to read it out before an item starts; the epilogue loads its
-// per-token scales before that wait, so only the tensor-memory reads stall it.
+// Roles (480 threads): warps 0-3 write the stage's scales into tensor memory
+// (both weight tiles: 128 rows of 16 B each; the activation rows: 192 rows of
+// 16 B; all from shared memory), warps 4-7 and 11-14 are the epilogues of the
+// pair's two tiles (TMEM lane quadrant = warp % 4), warp 8 the lead producer
+// (the two weight boxes and their scales), warp 9 the MMA issuer, warp 10 the
+// second producer (the activation box and its scales: 3-D boxes of three
+// terms of 64 rows).  Each epilogue reads its tile, frees it, then stores
+// while the next item's MMAs run: with one epilogue for both tiles the MMAs
+// waited for its stores (measured on the 235B-shaped layer at 2048 tokens:
+// gate/up 406 us, 318 us with the stores left out).
 //
-// B scale factors in tensor memory (scale_vec::4X): B row n's four scales of
-// one MMA are the 32-bit cell at lane n % 32, column c + n / 32 (c a multiple
-// of 4), as for the decode engine's rows below 64; 192 rows take six columns
-// per MMA, eight reserved.
+// Tensor memory: the two accumulators (192 columns each, one item in flight:
+// the MMA issuer waits for the epilogue to read them before an item starts;
+// the epilogue loads its per-token scales before that wait), then two slots
+// of 64 columns of scales, fewer than the three shared-memory stages: a scale
+// slot has its own full and empty barriers.  B scale factors (scale_vec::4X):
+// B row n's four scales of one MMA are the 32-bit cell at lane n % 32,
+// column c + n / 32 (c a multiple of 4); 192 rows take six columns per MMA,
+// eight reserved.
 //
 // Every wait is bounded (p.wait_ns); an expired wait sets the status word and
 // the kernel winds down, freeing its tensor memory.
@@ -52,22 +57,29 @@
 namespace moe {
 
 constexpr int kPfN = kPfTok * kPfTerms;   // MMA N (kPfTok tokens x kPfTerms terms, ffn.cuh)
-constexpr int kPfThreads = 11 * 32;
+// warps 0-10 as in ffn_bs.cuh (warps 4-7: the epilogue of the pair's first
+// tile), warps 11-14 the epilogue of its second tile
+constexpr int kPfEpi1Warp0 = 11;
+constexpr int kPfThreads = 15 * 32;
 
 struct PfGeom {
-  static constexpr int A = 0;                                // 128 rows x 128 B of codes
-  static constexpr int SA = kRowsHalf * kRowBytes;           // 128 rows x 16 B of scales
-  static constexpr int B = SA + kRowsHalf * 16;              // 18 KB, 1024-aligned
+  static constexpr int A = 0;                                // 2 x 128 rows x 128 B of codes
+  static constexpr int SA = 2 * kRowsHalf * kRowBytes;       // 2 x 128 rows x 16 B of scales
+  static constexpr int B = SA + 2 * kRowsHalf * 16;          // 36 KB, 1024-aligned
   static constexpr int SB = B + kPfN * kRowBytes;            // + 24 KB of activation rows
   static constexpr int RAW = SB + kPfN * 16;                 // + their scales (16 B a row)
   static constexpr int BYTES = (RAW + 1023) / 1024 * 1024;
-  static constexpr int STAGES = 4;
+  static constexpr int STAGES = 3;
   static constexpr int SMEM = STAGES * BYTES + 1024;
   static constexpr int BYTES_USED = RAW;   // bytes the copies of one stage bring
-  static constexpr uint32_t D_COLS = 256;  // the accumulator: kPfN columns, padded
+  static constexpr uint32_t D1 = kPfN;     // tile 1's accumulator (tile 0's at column 0)
+  static constexpr uint32_t D_COLS = 2 * kPfN;
+  static constexpr int SF_SLOTS = 2;       // scale slots: A0 16, A1 16, B 32 columns
+  static constexpr uint32_t SF_COLS = 64;
   static_assert(B % 1024 == 0, "B tile must start a swizzle atom");
-  static_assert(D_COLS + STAGES * kBsSfCols <= kBsTmemCols, "tensor memory budget");
+  static_assert(D_COLS + SF_SLOTS * SF_COLS <= kBsTmemCols, "tensor memory budget");
   static_assert(kPfN % 16 == 0 && kPfN <= 256, "MMA N");
+  static_assert(SMEM <= 227 * 1024 - 10 * 1024, "shared memory");
 };
 
 // 3-D tiled TMA load: x the innermost (contiguous) coordinate in elements.
@@ -82,13 +94,13 @@ __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, u
 }
 
 struct PfItem {
-  int slot, e, mat, rt, arow0, lrow0, nvalid, last_group;
+  int slot, e, mat, rt, arow0, lrow0, nvalid, last_group;  // rt: the pair's first tile
 };
 
-// Item `it` of a phase: per active slot, (group, matrix, row tile) with the
-// row tile fastest; phase 1 has two matrices (gate, up) of rt1 = I/128 tiles,
-// phase 2 one matrix of H/128 tiles.  The plan's chunk prefix counts groups
-// of kPfTok tokens.
+// Item `it` of a phase: per active slot, (group, matrix, tile pair) with the
+// pair fastest; phase 1 has two matrices (gate, up) of I/256 pairs of 128-row
+// tiles, phase 2 one matrix of H/256 pairs.  `rtiles` counts pairs.  The
+// plan's chunk prefix counts groups of kPfTok tokens.
 __device__ __forceinline__ PfItem pf_item(int it, int per, int rtiles, const PlanSmem& pl,
                                           const FfnParams& p) {
   PfItem r;
@@ -101,7 +113,7 @@ __device__ __forceinline__ PfItem pf_item(int it, int per, int rtiles, const Pla
   const int ng = pl.cpre[lo + 1] - pl.cpre[lo];
   const int local = it - per * pl.cpre[lo];
   const int g = local / per, q = local - g * per;
-  r.rt = q % rtiles;
+  r.rt = 2 * (q % rtiles);
   r.mat = q / rtiles;
   r.e = pl.act[lo];
   r.arow0 = pl.aoff[lo] + g * kPfTok;
@@ -123,13 +135,15 @@ __global__ void __launch_bounds__(kPfThreads, 1)
                   const FfnParams p) {
   using G = PfGeom;
   constexpr int S = G::STAGES;
+  constexpr int SFS = G::SF_SLOTS;
 
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
 
   __shared__ __align__(8) uint64_t full_bar[S];
   __shared__ __align__(8) uint64_t empty_bar[S];
-  __shared__ __align__(8) uint64_t sf_bar[S];
+  __shared__ __align__(8) uint64_t sf_full[SFS];
+  __shared__ __align__(8) uint64_t sf_empty[SFS];
   __shared__ __align__(8) uint64_t dfull_bar;
   __shared__ __align__(8) uint64_t dempty_bar;
   __shared__ __align__(8) uint64_t final_bar;
@@ -146,10 +160,13 @@ __global__ void __launch_bounds__(kPfThreads, 1)
     for (int i = 0; i < S; ++i) {
       mbar_init(&full_bar[i], 1);
       mbar_init(&empty_bar[i], 1);
-      mbar_init(&sf_bar[i], 4);
+    }
+    for (int i = 0; i < SFS; ++i) {
+      mbar_init(&sf_full[i], 4);
+      mbar_init(&sf_empty[i], 1);
     }
     mbar_init(&dfull_bar, 1);
-    mbar_init(&dempty_bar, 4);
+    mbar_init(&dempty_bar, 8);  // the eight epilogue warps
     mbar_init(&final_bar, 1);
     fence_mbar_init();
   }
@@ -172,8 +189,8 @@ __global__ void __launch_bounds__(kPfThreads, 1)
 
   const int N = (PHASE == 1) ? p.I : p.H;  // rows of one expert matrix
   const int K = (PHASE == 1) ? p.H : p.I;  // contraction length
-  const int rtiles = N / kRowsHalf;
-  const int per = (PHASE == 1) ? 2 * rtiles : rtiles;  // items per token group
+  const int rpairs = N / (2 * kRowsHalf);  // pairs of 128-row tiles
+  const int per = (PHASE == 1) ? 2 * rpairs : rpairs;  // items per token group
   const int KB = K / 256;
   const int items = per * pl.cpre[pl.nA];
   // this CTA's items: blockIdx.x, + gridDim.x, ...
@@ -182,7 +199,7 @@ __global__ void __launch_bounds__(kPfThreads, 1)
   const int i_begin = blockIdx.x;
   const int nst = my_items * KB;
   const uint32_t timeout_bit = (PHASE == 1) ? kStatusTimeoutGateUp : kStatusTimeoutDown;
-  constexpr int kTeardown = 9 * 32;  // scale writers, epilogue and MMA warps
+  constexpr int kTeardown = 13 * 32;  // scale writers, epilogues and MMA warps
 
   // ================================================================ producers
   if (warp == kBsProducerWarp || warp == kBsProducerWarp2) {
@@ -200,7 +217,7 @@ __global__ void __launch_bounds__(kPfThreads, 1)
       const uint64_t pol_last = policy_evict_last();
       int it = i_begin, kb = 0, slot = 0, issued = 0;
       uint32_t par = 0u;
-      PfItem inf = pf_item(it, per, rtiles, pl, p);
+      PfItem inf = pf_item(it, per, rpairs, pl, p);
       for (; issued < nst; ++issued) {
         if (!mbar_wait_bounded(&empty_bar[slot], par ^ 1u, p.wait_ns, &s_abort)) {
           set_status(p.status, timeout_bit);
@@ -211,13 +228,18 @@ __global__ void __launch_bounds__(kPfThreads, 1)
           unsigned char* st = smem + (size_t)slot * G::BYTES;
           if (lead) {
             mbar_arrive_expect_tx(&full_bar[slot], (uint32_t)(G::BYTES_USED));
-            // the next group of the same expert reads this tile again
+            // the next group of the same expert reads these tiles again
             const uint64_t pol = inf.last_group ? pol_first : pol_last;
+            const CUtensorMap* ma = inf.mat ? &tmA1 : &tmA0;
+            const CUtensorMap* ms = inf.mat ? &tmS1 : &tmS0;
             const int row = inf.e * N + inf.rt * kRowsHalf;
-            tma_load_2d(st + G::A, inf.mat ? &tmA1 : &tmA0, &full_bar[slot], kb * kRowBytes,
-                        row, pol);
-            tma_load_2d(st + G::SA, inf.mat ? &tmS1 : &tmS0, &full_bar[slot], kb * 16, row,
-                        pol);
+#pragma unroll
+            for (int t = 0; t < 2; ++t) {
+              tma_load_2d(st + G::A + t * kRowsHalf * kRowBytes, ma, &full_bar[slot],
+                          kb * kRowBytes, row + t * kRowsHalf, pol);
+              tma_load_2d(st + G::SA + t * kRowsHalf * 16, ms, &full_bar[slot], kb * 16,
+                          row + t * kRowsHalf, pol);
+            }
           } else {
             tma_load_3d(st + G::B, &tmB, &full_bar[slot], kb * kRowBytes, 0, inf.arow0,
                         pol_last);
@@ -231,7 +253,7 @@ __global__ void __launch_bounds__(kPfThreads, 1)
         if (++kb == KB && issued + 1 < nst) {
           kb = 0;
           it += gridDim.x;
-          inf = pf_item(it, per, rtiles, pl, p);
+          inf = pf_item(it, per, rpairs, pl, p);
         }
       }
       // every copy this CTA issued lands before the CTA exits
@@ -251,23 +273,28 @@ __global__ void __launch_bounds__(kPfThreads, 1)
     if (lane == 0) {
       constexpr uint32_t idesc = tc_idesc_mxf4nvf4(128, kPfN);
       bool ok = true;
-      int slot = 0, kb = 0, nitem = 0;
-      uint32_t par = 0u;
+      int slot = 0, fs = 0, kb = 0, nitem = 0;
+      uint32_t par = 0u, fpar = 0u;
       for (int i = 0; i < nst && ok; ++i) {
         if (kb == 0)
           ok = mbar_wait_bounded(&dempty_bar, ((uint32_t)nitem & 1u) ^ 1u, p.wait_ns, &s_abort);
         ok = ok && mbar_wait_bounded(&full_bar[slot], par, p.wait_ns, &s_abort) &&
-             mbar_wait_bounded(&sf_bar[slot], par, p.wait_ns, &s_abort);
+             mbar_wait_bounded(&sf_full[fs], fpar, p.wait_ns, &s_abort);
         if (!ok) break;
         tc_fence_after();
         const uint32_t st = smem_u32(smem + (size_t)slot * G::BYTES);
-        const uint32_t sfc = tmem + G::D_COLS + (uint32_t)slot * kBsSfCols;
+        const uint32_t sfc = tmem + G::D_COLS + (uint32_t)fs * G::SF_COLS;
 #pragma unroll
-        for (int kk = 0; kk < 4; ++kk)
-          tc_mma_mxf4nvf4(tmem, tc_desc_sw128(st + G::A + 32 * kk),
-                          tc_desc_sw128(st + G::B + 32 * kk), idesc, sfc + 4 * kk,
-                          sfc + 16 + 8 * kk, (kb == 0 && kk == 0) ? 0u : 1u);
+        for (int kk = 0; kk < 4; ++kk) {
+          const uint64_t bdesc = tc_desc_sw128(st + G::B + 32 * kk);
+          const uint32_t acc = (kb == 0 && kk == 0) ? 0u : 1u;
+          tc_mma_mxf4nvf4(tmem, tc_desc_sw128(st + G::A + 32 * kk), bdesc, idesc, sfc + 4 * kk,
+                          sfc + 32 + 8 * kk, acc);
+          tc_mma_mxf4nvf4(tmem + G::D1, tc_desc_sw128(st + G::A + kRowsHalf * kRowBytes + 32 * kk),
+                          bdesc, idesc, sfc + 16 + 4 * kk, sfc + 32 + 8 * kk, acc);
+        }
         tc_commit(&empty_bar[slot]);
+        tc_commit(&sf_empty[fs]);
         if (++kb == KB) {
           kb = 0;
           tc_commit(&dfull_bar);
@@ -276,6 +303,10 @@ __global__ void __launch_bounds__(kPfThreads, 1)
         if (++slot == S) {
           slot = 0;
           par ^= 1u;
+        }
+        if (++fs == SFS) {
+          fs = 0;
+          fpar ^= 1u;
         }
       }
       if (!ok) {
@@ -299,22 +330,25 @@ __global__ void __launch_bounds__(kPfThreads, 1)
     const int quad = warp - kBsSfWarp0;
     const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
     constexpr int NH = kPfN / 32;  // B rows per lane: lane + 32 h
-    int slot = 0;
-    uint32_t par = 0u;
+    int slot = 0, fs = 0;
+    uint32_t par = 0u, fpar = 0u;
     for (int i = 0; i < nst; ++i) {
-      if (!mbar_wait_bounded(&empty_bar[slot], par ^ 1u, p.wait_ns, &s_abort) ||
-          !mbar_wait_bounded(&full_bar[slot], par, p.wait_ns, &s_abort)) {
+      // the stage's copies have landed, and the scale slot's previous MMAs are done
+      if (!mbar_wait_bounded(&full_bar[slot], par, p.wait_ns, &s_abort) ||
+          !mbar_wait_bounded(&sf_empty[fs], fpar ^ 1u, p.wait_ns, &s_abort)) {
         set_status(p.status, timeout_bit);
         s_abort = 1;
         break;
       }
       tc_fence_after();
       const uint32_t st = smem_u32(smem + (size_t)slot * G::BYTES);
-      const uint32_t sfc = tmem + lane_addr + G::D_COLS + (uint32_t)slot * kBsSfCols;
-      {
+      const uint32_t sfc = tmem + lane_addr + G::D_COLS + (uint32_t)fs * G::SF_COLS;
+#pragma unroll
+      for (int t = 0; t < 2; ++t) {  // the weight tiles' scales: columns 16t + 4kk + r
         uint4 v[4];
 #pragma unroll
-        for (int r1 = 0; r1 < 4; ++r1) v[r1] = lds128(st + G::SA + (lane + 32 * r1) * 16);
+        for (int r1 = 0; r1 < 4; ++r1)
+          v[r1] = lds128(st + G::SA + t * kRowsHalf * 16 + (lane + 32 * r1) * 16);
         uint32_t c[16];
 #pragma unroll
         for (int r1 = 0; r1 < 4; ++r1) {
@@ -323,11 +357,12 @@ __global__ void __launch_bounds__(kPfThreads, 1)
           c[8 + r1] = v[r1].z;
           c[12 + r1] = v[r1].w;
         }
-        tmem_st16(sfc, c);
+        tmem_st16(sfc + 16 * t, c);
       }
       {
         // B row n = 3j + t: term t of the group's token j (rows past the
-        // group's tokens were filled with zeros by the copy)
+        // group's tokens hold other rows or the copy's zeros; their columns
+        // are not stored)
         uint4 bsf[NH];
 #pragma unroll
         for (int h = 0; h < NH; ++h) bsf[h] = lds128(st + G::SB + (lane + 32 * h) * 16);
@@ -347,16 +382,20 @@ __global__ void __launch_bounds__(kPfThreads, 1)
               c[8 * m2 + h] = wv;
             }
           }
-          tmem_st16(sfc + 16 + 16 * half, c);
+          tmem_st16(sfc + 32 + 16 * half, c);
         }
       }
       tmem_st_wait();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&sf_bar[slot]);
+      if (lane == 0) mbar_arrive(&sf_full[fs]);
       if (++slot == S) {
         slot = 0;
         par ^= 1u;
+      }
+      if (++fs == SFS) {
+        fs = 0;
+        fpar ^= 1u;
       }
     }
     tc_fence_before();
@@ -364,21 +403,24 @@ __global__ void __launch_bounds__(kPfThreads, 1)
     return;
   }
 
-  // ================================================================ epilogue
-  // Warp 4+q reads TMEM lanes 32q..32q+31: row 32q+lane of the item's tile.
+  // ================================================================ epilogues
+  // Warp w reads TMEM lanes 32(w%4)..+31 of its tile's accumulator: row
+  // 32(w%4) + lane of the tile.
   {
     if (early) pdl_wait();  // the row scales of h are the SwiGLU output
-    const int quad = warp - kBsEpiWarp0;
-    const int tid = threadIdx.x - kBsEpiWarp0 * 32;  // 0..127
+    const int tile = warp >= kPfEpi1Warp0 ? 1 : 0;
+    const int quad = warp & 3;
+    const int tid = tile ? 128 + (warp - kPfEpi1Warp0) * 32 + lane
+                         : (warp - kBsEpiWarp0) * 32 + lane;  // 0..255
     const int row = quad * 32 + lane;
     const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
     // true in every epilogue thread when it is true in any (the waits are per
-    // thread; the named barrier of the next item needs all 128 threads)
+    // thread; the named barrier of the next item needs all 256 threads)
     auto any_dead = [&](bool v) -> bool {
       uint32_t rr;
       asm volatile(
           "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n"
-          " bar.red.or.pred q, 3, 128, p;\n selp.u32 %0, 1, 0, q;\n}\n"
+          " bar.red.or.pred q, 3, 256, p;\n selp.u32 %0, 1, 0, q;\n}\n"
           : "=r"(rr)
           : "r"((uint32_t)v)
           : "memory");
@@ -387,7 +429,7 @@ __global__ void __launch_bounds__(kPfThreads, 1)
     // per-token scales of item `it` (x's row scale in phase 1, h's in phase
     // 2) and its tensor scale, read by threads 0..kPfTok
     auto load_scales = [&](int it, float& v) {
-      const PfItem inf = pf_item(it, per, rtiles, pl, p);
+      const PfItem inf = pf_item(it, per, rpairs, pl, p);
       v = 0.f;
       if (tid < inf.nvalid) {
         if (PHASE == 1)
@@ -405,13 +447,13 @@ __global__ void __launch_bounds__(kPfThreads, 1)
       if (tid == kPfTok) s_ts[0] = v_next;
     }
     for (int n = 0, it = i_begin; n < my_items; ++n, it += gridDim.x) {
-      const PfItem inf = pf_item(it, per, rtiles, pl, p);
+      const PfItem inf = pf_item(it, per, rpairs, pl, p);
       const int b = n & 1;
       // the next item's scales are requested now and stored after this
       // item's accumulator is read: their latency overlaps the MMAs
       const bool has_next = n + 1 < my_items;
       if (has_next) load_scales(it + gridDim.x, v_next);
-      asm volatile("bar.sync 3, 128;" ::: "memory");
+      asm volatile("bar.sync 3, 256;" ::: "memory");
       const bool ok = mbar_wait_bounded(&dfull_bar, (uint32_t)n & 1u, p.wait_ns, &s_abort);
       if (any_dead(!ok)) {
         set_status(p.status, timeout_bit);
@@ -419,14 +461,15 @@ __global__ void __launch_bounds__(kPfThreads, 1)
         break;
       }
       tc_fence_after();
-      // the three terms of token j are accumulator columns 3j..3j+2
+      // the three terms of token j are the tile's accumulator columns 3j..3j+2
       float acc[kPfTok];
 #pragma unroll
       for (int c0 = 0; c0 < kPfN; c0 += 48) {
         uint32_t v[48];
-        tmem_ld16(tmem + lane_addr + c0, *reinterpret_cast<uint32_t(*)[16]>(v));
-        tmem_ld16(tmem + lane_addr + c0 + 16, *reinterpret_cast<uint32_t(*)[16]>(v + 16));
-        tmem_ld16(tmem + lane_addr + c0 + 32, *reinterpret_cast<uint32_t(*)[16]>(v + 32));
+        const uint32_t ta = tmem + lane_addr + (uint32_t)tile * G::D1 + (uint32_t)c0;
+        tmem_ld16(ta, *reinterpret_cast<uint32_t(*)[16]>(v));
+        tmem_ld16(ta + 16, *reinterpret_cast<uint32_t(*)[16]>(v + 16));
+        tmem_ld16(ta + 32, *reinterpret_cast<uint32_t(*)[16]>(v + 32));
         tmem_ld_wait();
 #pragma unroll
         for (int j = 0; j < 16; ++j)
@@ -435,13 +478,13 @@ __global__ void __launch_bounds__(kPfThreads, 1)
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&dempty_bar);
+      if (lane == 0) mbar_arrive(&dempty_bar);  // this warp's part of the accumulators is read
       if (has_next) {  // every thread is past the previous item: its buffer is free
         if (tid < kPfTok) s_sc[b ^ 1][tid] = v_next;
         if (tid == kPfTok) s_ts[b ^ 1] = v_next;
       }
       const float ts = s_ts[b];
-      const int col = inf.rt * kRowsHalf + row;
+      const int col = (inf.rt + tile) * kRowsHalf + row;
 #pragma unroll
       for (int j = 0; j < kPfTok; ++j) {
         if (j >= inf.nvalid) break;
