@@ -763,6 +763,10 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
     q.E = E;
     q.Ep = route_tc_ep(E);
     q.prenorm = p.prenorm;
+    q.act = p.act;
+    q.xq = p.xq;
+    q.xsf = p.xsf;
+    q.xinv = p.xinv;
     q.status = ws_ptr<uint32_t>(ws, L.status);
     q.wait_ns = wait_limit_ns();
     CUtensorMap ta, tb;
@@ -783,10 +787,12 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
     int per = (sms + chunks - 1) / chunks;
     per = per < 1 ? 1 : (per > (E + 3) / 4 ? (E + 3) / 4 : per);
     p.epb = (E + per - 1) / per;
-    if (p.prenorm) {  // the router kernel stages the normalised rows
+    if (p.act == kActTerms || p.act == kActE4M3) {
+      p.terms_done = 1;  // the prep kernel wrote the activation terms
+    } else if (p.prenorm) {  // the router kernel stages the normalised rows
       p.x = q.xn;
-      p.prenorm = 0;
     }
+    p.prenorm = 0;
   }
   if (launch_route(p, st) != cudaSuccess) return MOE_ERR_CUDA;
   const bool gathered = gather_terms(T, p.act);

@@ -237,4 +237,63 @@ __device__ __forceinline__ void store_e4m3x2_8(const uint2& hi, const uint2& lo,
   *reinterpret_cast<uint2*>(q + (row2 + 1) * (size_t)K + 8 * c8) = lo;
 }
 
+// The two E4M3 terms of one token row in global memory, by one warp.
+__device__ __forceinline__ void convert_row_e4m3(const __nv_bfloat16* row, int H, int t,
+                                                 uint8_t* xq, float* inv, int lane) {
+  float amax = 0.f;
+  for (int h = lane * 8; h < H; h += 256) {
+    const uint4 v = *reinterpret_cast<const uint4*>(row + h);
+    const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 f = __bfloat1622float2(b[i]);
+      amax = fmaxf(amax, fmaxf(fabsf(f.x), fabsf(f.y)));
+    }
+  }
+  amax = warp_max(amax);
+  const float sc = pow2_scale_e4m3(amax);
+  for (int c = lane; c < H / 8; c += 32) {
+    const uint4 v = *reinterpret_cast<const uint4*>(row + 8 * c);
+    const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&v);
+    float f[8];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 tt = __bfloat1622float2(b[i]);
+      f[2 * i] = tt.x * sc;
+      f[2 * i + 1] = tt.y * sc;
+    }
+    uint2 hi, lo;
+    encode_e4m3x2_8(f, hi, lo);
+    store_e4m3x2_8(hi, lo, xq, (size_t)t * kF8Terms, H, c);
+  }
+  if (lane == 0) *inv = 1.f / sc;
+}
+
+// The NVFP4 terms of one token row in global memory, by one warp.
+__device__ __forceinline__ void convert_row_terms(const __nv_bfloat16* row, int H, int t,
+                                                  uint8_t* xq, uint8_t* xsf, float* inv,
+                                                  int lane) {
+  float amax = 0.f;
+  for (int h = lane * 8; h < H; h += 256) {
+    const uint4 v = *reinterpret_cast<const uint4*>(row + h);
+    const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 f = __bfloat1622float2(b[i]);
+      amax = fmaxf(amax, fmaxf(fabsf(f.x), fabsf(f.y)));
+    }
+  }
+  amax = warp_max(amax);
+  const float sc = pow2_scale_terms(amax);
+  for (int b = lane; b < H / 16; b += 32) {
+    float r[16];
+    load_bf16x16_scaled(row + 16 * b, sc, r);
+    uint2 codes[kTerms];
+    uint32_t sf[kTerms];
+    encode_terms16(r, codes, sf);
+    store_terms16(codes, sf, xq, xsf, (size_t)t * kTerms, H, b);
+  }
+  if (lane == 0) *inv = 1.f / sc;
+}
+
 }  // namespace moe

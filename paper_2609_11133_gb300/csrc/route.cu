@@ -147,64 +147,6 @@ __device__ void convert_chunk_e4m3(const __nv_bfloat16* xs, int nt, int H, int t
   }
 }
 
-// The two E4M3 terms of one token row in global memory, by one warp.
-__device__ void convert_row_e4m3(const __nv_bfloat16* row, int H, int t, uint8_t* xq, float* inv,
-                                 int lane) {
-  float amax = 0.f;
-  for (int h = lane * 8; h < H; h += 256) {
-    const uint4 v = *reinterpret_cast<const uint4*>(row + h);
-    const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&v);
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const float2 f = __bfloat1622float2(b[i]);
-      amax = fmaxf(amax, fmaxf(fabsf(f.x), fabsf(f.y)));
-    }
-  }
-  amax = warp_max(amax);
-  const float sc = pow2_scale_e4m3(amax);
-  for (int c = lane; c < H / 8; c += 32) {
-    const uint4 v = *reinterpret_cast<const uint4*>(row + 8 * c);
-    const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&v);
-    float f[8];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const float2 tt = __bfloat1622float2(b[i]);
-      f[2 * i] = tt.x * sc;
-      f[2 * i + 1] = tt.y * sc;
-    }
-    uint2 hi, lo;
-    encode_e4m3x2_8(f, hi, lo);
-    store_e4m3x2_8(hi, lo, xq, (size_t)t * kF8Terms, H, c);
-  }
-  if (lane == 0) *inv = 1.f / sc;
-}
-
-// The NVFP4 terms of one token row in global memory, by one warp.
-__device__ void convert_row_terms(const __nv_bfloat16* row, int H, int t, uint8_t* xq,
-                                  uint8_t* xsf, float* inv, int lane) {
-  float amax = 0.f;
-  for (int h = lane * 8; h < H; h += 256) {
-    const uint4 v = *reinterpret_cast<const uint4*>(row + h);
-    const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&v);
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const float2 f = __bfloat1622float2(b[i]);
-      amax = fmaxf(amax, fmaxf(fabsf(f.x), fabsf(f.y)));
-    }
-  }
-  amax = warp_max(amax);
-  const float sc = pow2_scale_terms(amax);
-  for (int b = lane; b < H / 16; b += 32) {
-    float r[16];
-    load_bf16x16_scaled(row + 16 * b, sc, r);
-    uint2 codes[kTerms];
-    uint32_t sf[kTerms];
-    encode_terms16(r, codes, sf);
-    store_terms16(codes, sf, xq, xsf, (size_t)t * kTerms, H, b);
-  }
-  if (lane == 0) *inv = 1.f / sc;
-}
-
 // Order-preserving unsigned key of a finite float (larger value, larger key;
 // -0 maps like +0), and its inverse.  Keys of finite values are never 0.
 __device__ __forceinline__ unsigned logit_key(float v) {
@@ -407,7 +349,7 @@ __global__ void __launch_bounds__(256) route_kernel(const RouteParams p) {
 
   // stage this chunk's token rows: every thread issues all of its 16-byte
   // loads before storing any of them (one memory latency, not one per load)
-  {
+  if (!p.terms_done) {
     const uint4* src = reinterpret_cast<const uint4*>(p.x + (size_t)t0 * H);
     uint4* dst = reinterpret_cast<uint4*>(xs);
     const int n16 = nt * H / 8;
@@ -432,7 +374,7 @@ __global__ void __launch_bounds__(256) route_kernel(const RouteParams p) {
     rms_norm_row_bf16(row, row, H, lane);
   }
   __syncthreads();
-  if (p.fused) {
+  if (p.fused && !p.terms_done) {
     if (p.act == kActTerms) {
       convert_chunk_terms(xs, nt, H, t0, eb, gridDim.x, p.xq, p.xsf, p.xinv);
     } else if (p.act == kActE4M3) {
@@ -754,7 +696,7 @@ cudaError_t launch_route(const RouteParams& p, cudaStream_t st) {
     cfg.gridDim = dim3((unsigned)((p.E + p.epb - 1) / p.epb),
                        (unsigned)((p.T + kRouteTok - 1) / kRouteTok));
     cfg.blockDim = dim3(256);
-    cfg.dynamicSmemBytes = smem;
+    cfg.dynamicSmemBytes = p.terms_done ? 0 : smem;  // no rows staged
     cfg.stream = st;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;

@@ -63,18 +63,28 @@ struct RouteParams {
   unsigned* acnt;  // [E] assignments per expert, zero on entry
   int* alist;      // [E, T] expert e's assignments t*k + j at alist[e*T + 0..]
   // logits from the tensor-core router: partial sums [nsplit, T, ep] added in
-  // slice order (one CTA per token chunk, no GEMV here); null: the GEMV here
+  // slice order (no GEMV here); null: the GEMV here
   const float* plog;
   int nsplit, ep;
+  // 1: the activation terms of x were written by router_prep_kernel (no rows
+  // are staged here)
+  int terms_done;
 };
 
 // The tensor-core router's two kernels (route_tc.cu): router_prep_kernel
-// splits the fp32 router rows into three bf16 parts (and writes the
-// RMS-normalised rows of x when prenorm), route_tc_kernel multiplies.
+// splits the fp32 router rows into three bf16 parts and, a warp per token,
+// writes the RMS-normalised row (prenorm) and the row's activation terms;
+// route_tc_kernel multiplies.
 struct RouteTcParams {
   const float* wr;          // [E, H]
-  const __nv_bfloat16* x;   // [T, H] (the prep kernel's input when prenorm)
+  const __nv_bfloat16* x;   // [T, H]
   __nv_bfloat16* xn;        // [T, H] normalised rows (prenorm), else unused
+  // activation terms of the (normalised) rows for the expert kernels, when
+  // act is kActTerms or kActE4M3 (as route_kernel writes them otherwise)
+  int act;
+  uint8_t* xq;
+  uint8_t* xsf;
+  float* xinv;
   __nv_bfloat16* w3;        // [3, Ep, H]: wr = w3[0] + w3[1] + w3[2]; rows >= E zero
   float* plog;              // [kRouteTcSplit, T, Ep]
   int T, H, E, Ep, prenorm;

@@ -17,6 +17,7 @@
 // into one tensor-memory accumulator.  The epilogue writes the slice's fp32
 // partial logits; the router kernel adds the slices in order, then does the
 // softmax, top-k and the rest of the routing.
+#include "act_terms.cuh"
 #include "route.cuh"
 
 namespace moe {
@@ -63,7 +64,8 @@ __device__ __forceinline__ void split3(float w, __nv_bfloat16& a, __nv_bfloat16&
 }
 
 // Blocks [0, nsplit): the router rows as three bf16 parts (rows E..Ep-1 zero).
-// Blocks after them (prenorm only): the RMS-normalised rows of x, a warp per row.
+// Blocks after them, a warp per token row: the RMS-normalised row (prenorm)
+// and the row's activation terms (the same codes route_kernel writes).
 __global__ void __launch_bounds__(256) router_prep_kernel(const RouteTcParams p, int nsplit) {
   pdl_launch_dependents();
   if ((int)blockIdx.x < nsplit) {
@@ -89,8 +91,17 @@ __global__ void __launch_bounds__(256) router_prep_kernel(const RouteTcParams p,
   }
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int t = ((int)blockIdx.x - nsplit) * 8 + warp;
-  if (t < p.T)
-    rms_norm_row_bf16(p.x + (size_t)t * p.H, p.xn + (size_t)t * p.H, p.H, lane);
+  if (t >= p.T) return;
+  const __nv_bfloat16* row = p.x + (size_t)t * p.H;
+  if (p.prenorm) {
+    rms_norm_row_bf16(row, p.xn + (size_t)t * p.H, p.H, lane);
+    row = p.xn + (size_t)t * p.H;
+    __syncwarp();  // the warp's own stores of the row are read back below
+  }
+  if (p.act == kActTerms)
+    convert_row_terms(row, p.H, t, p.xq, p.xsf, p.xinv + t, lane);
+  else if (p.act == kActE4M3)
+    convert_row_e4m3(row, p.H, t, p.xq, p.xinv + t, lane);
 }
 
 __global__ void __launch_bounds__(kTcThreads, 1)
@@ -234,7 +245,8 @@ cudaError_t launch_router_prep(const RouteTcParams& p, cudaStream_t st) {
   const size_t n4 = (size_t)p.Ep * p.H / 4;
   int nsplit = (int)((n4 + 4 * 256 - 1) / (4 * 256));  // four float4 per thread
   if (nsplit < 1) nsplit = 1;
-  const int nnorm = p.prenorm ? (p.T + 7) / 8 : 0;
+  const bool rows = p.prenorm || p.act == kActTerms || p.act == kActE4M3;
+  const int nnorm = rows ? (p.T + 7) / 8 : 0;
   router_prep_kernel<<<nsplit + nnorm, 256, 0, st>>>(p, nsplit);
   return cudaGetLastError();
 }
