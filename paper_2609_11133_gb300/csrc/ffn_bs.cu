@@ -37,7 +37,11 @@ cudaError_t launch_ffn_bs(int nt, int grid, const FfnMaps& m, const FfnParams& p
 }
 
 // One wave of the rows kernel: every resident CTA takes the same number of
-// rows (within one), so none of them is left running alone at the end.
+// rows (within one), so none of them is left running alone at the end.  It
+// is launched after the gate/up kernel, not as its programmatic dependent:
+// launched early, the wave's CTAs pile up on the SMs whose gate/up CTAs end
+// first, and the rest of the SMs get none (measured on the 235B-shaped layer
+// at 2048 tokens: 818 us a layer with the early launch, 750 us without).
 template <typename K>
 static int resident_blocks(K kern, int sms, std::atomic<int>& cache) {
   int per = cache.load();
@@ -56,7 +60,7 @@ static cudaError_t launch_rows_g(int sms, int rows, const FfnParams& p, cudaStre
   auto kern = swiglu_terms_rows_kernel<G, NTERM>;
   int blocks = resident_blocks(kern, sms, per);
   if (blocks > rows) blocks = rows;
-  return launch_pdl(kern, dim3(blocks), dim3(128), 0, st, p, rows);
+  return launch_k(kern, dim3(blocks), dim3(128), 0, st, false, p, rows);
 }
 
 template <int NTERM>
