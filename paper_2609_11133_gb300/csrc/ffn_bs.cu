@@ -13,8 +13,8 @@ static cudaError_t launch_ffn_bs_ph(int grid, const FfnMaps& m, const FfnParams&
   static std::atomic<unsigned long long> done{0};
   cudaError_t err = set_smem_once(kern, smem, done);
   if (err != cudaSuccess) return err;
-  return launch_pdl(kern, dim3(grid), dim3(kBsThreads), smem, st, m.a0, m.a1, m.s0, m.s1, m.b,
-                    p);
+  return launch_k(kern, dim3(grid), dim3(kBsThreads), smem, st, expert_pdl(p, true), m.a0, m.a1,
+                  m.s0, m.s1, m.b, p);
 }
 
 template <int NT>

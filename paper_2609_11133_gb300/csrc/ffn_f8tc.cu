@@ -13,7 +13,8 @@ static cudaError_t launch_ffn_f8_ph(int grid, const FfnMaps& m, const FfnParams&
   static std::atomic<unsigned long long> done{0};
   cudaError_t err = set_smem_once(kern, smem, done);
   if (err != cudaSuccess) return err;
-  return launch_pdl(kern, dim3(grid), dim3(kF8Threads), smem, st, m.a0, m.a1, m.b, p);
+  return launch_k(kern, dim3(grid), dim3(kF8Threads), smem, st, expert_pdl(p, false), m.a0,
+                  m.a1, m.b, p);
 }
 
 template <int NT>

@@ -32,6 +32,21 @@ cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t sme
   return launch_k(kern, grid, block, smem, st, true, args...);
 }
 
+// Whether an expert kernel of the tensor-core engines starts as a programmatic
+// dependent of the kernel before it.  The persistent grid divides its stages
+// by CTA index and assumes every CTA starts at once; launched early behind a
+// short kernel of many CTAs (the gather before gate/up, the SwiGLU rows kernel
+// before NVFP4 down), its CTAs start as those SMs free up, and the last ones
+// finish late.  Measured in a graph of layer calls, early launch off: FP8
+// 480B-shaped T=512 gate/up 1600 -> 1572 us a layer; NVFP4 235B-shaped T=128
+// gate/up 278.7 -> 273.8, down 278.7 -> 274.2; prefill-shaped T=2048 gate/up
+// 750 -> 742.  Up to 64 tokens (no gather, the quad SwiGLU) the early start
+// pays: NVFP4 T=64 243 us with it, 254 without.
+inline bool expert_pdl(const FfnParams& p, bool nvfp4) {
+  if (p.phase == 1) return !p.b_compact;
+  return !nvfp4 || p.T * p.k <= 512;
+}
+
 struct FfnMaps {
   CUtensorMap a0, a1, s0, s1, b;
   CUtensorMap sb;  // prefill engine: the activation terms' scales

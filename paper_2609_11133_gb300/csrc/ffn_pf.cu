@@ -12,8 +12,8 @@ static cudaError_t launch_ffn_pf_ph(int grid, const FfnMaps& m, const FfnParams&
   static std::atomic<unsigned long long> done{0};
   cudaError_t err = set_smem_once(kern, smem, done);
   if (err != cudaSuccess) return err;
-  return launch_pdl(kern, dim3(grid), dim3(kPfThreads), smem, st, m.a0, m.a1, m.s0, m.s1, m.b,
-                    m.sb, p);
+  return launch_k(kern, dim3(grid), dim3(kPfThreads), smem, st, expert_pdl(p, true), m.a0, m.a1,
+                  m.s0, m.s1, m.b, m.sb, p);
 }
 
 cudaError_t launch_ffn_pf(int grid, const FfnMaps& m, const FfnParams& p, cudaStream_t st) {
