@@ -8,10 +8,10 @@ namespace moe {
 template <int NT, int PHASE>
 static cudaError_t launch_ffn_bs_ph(int grid, const FfnMaps& m, const FfnParams& p,
                                     cudaStream_t st) {
-  auto kern = ffn_bs_kernel<NT, PHASE>;
+  auto kern = p.det ? ffn_bs_kernel<NT, PHASE, true> : ffn_bs_kernel<NT, PHASE, false>;
   const int smem = BsGeom<NT>::SMEM;
-  static std::atomic<unsigned long long> done{0};
-  cudaError_t err = set_smem_once(kern, smem, done);
+  static std::atomic<unsigned long long> done[2] = {{0}, {0}};  // per variant
+  cudaError_t err = set_smem_once(kern, smem, done[p.det ? 1 : 0]);
   if (err != cudaSuccess) return err;
   return launch_k(kern, dim3(grid), dim3(kBsThreads), smem, st, expert_pdl(p, true), m.a0, m.a1,
                   m.s0, m.s1, m.b, p);

@@ -96,7 +96,7 @@ __device__ __forceinline__ uint4 ldg_nc_v4(const void* p) {
   return v;
 }
 
-template <int NT, int PHASE>
+template <int NT, int PHASE, bool DET>
 __global__ void __launch_bounds__(kBsThreads, 1)
     ffn_bs_kernel(const __grid_constant__ CUtensorMap tmA0,
                   const __grid_constant__ CUtensorMap tmA1,
@@ -167,7 +167,7 @@ __global__ void __launch_bounds__(kBsThreads, 1)
   const int cost_a = stage_cost_base((PHASE == 1) && !p.b_compact);
   int s_begin = cost_split_stage(pl, rtiles, KB, NT, cost_a, kTokenCost, blockIdx.x, gridDim.x);
   int s_end = cost_split_stage(pl, rtiles, KB, NT, cost_a, kTokenCost, blockIdx.x + 1, gridDim.x);
-  if (p.det) {
+  if (DET) {
     s_begin = (int)item_boundary(s_begin, KB);
     s_end = (int)item_boundary(s_end, KB);
   }
@@ -465,8 +465,8 @@ __global__ void __launch_bounds__(kBsThreads, 1)
             const float sc = __ldg(p.xinv + a / p.k);
             const int f = inf.rt * kRowsHalf + row;
             float* gr = p.gu + (size_t)arow * 2 * p.I + f;
-            put_f32(gr, acc[0][j] * sc * ts0, p.det);
-            put_f32(gr + p.I, acc[1][j] * sc * ts1, p.det);
+            put_f32(gr, acc[0][j] * sc * ts0, DET);
+            put_f32(gr + p.I, acc[1][j] * sc * ts1, DET);
           } else {
             const float sc = __ldcg(p.xinv + arow);  // hinv, written by the previous kernel
             const int hrow = inf.rt * 2 * kRowsHalf + row;
@@ -476,9 +476,9 @@ __global__ void __launch_bounds__(kBsThreads, 1)
               red_add_f32(orow, gw * acc[0][j] * ts0);
               red_add_f32(orow + kRowsHalf, gw * acc[1][j] * ts1);
             } else {
-              float* yrow = p.y_perm + (size_t)(p.det ? a : arow) * p.H + hrow;
-              put_f32(yrow, acc[0][j] * sc * ts0, p.det);
-              put_f32(yrow + kRowsHalf, acc[1][j] * sc * ts1, p.det);
+              float* yrow = p.y_perm + (size_t)(DET ? a : arow) * p.H + hrow;
+              put_f32(yrow, acc[0][j] * sc * ts0, DET);
+              put_f32(yrow + kRowsHalf, acc[1][j] * sc * ts1, DET);
             }
           }
         }

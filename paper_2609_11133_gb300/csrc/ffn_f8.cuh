@@ -60,7 +60,7 @@ __device__ __forceinline__ void tc_mma_f8(uint32_t d_tmem, uint64_t a_desc, uint
       : "memory");
 }
 
-template <int NT, int PHASE>
+template <int NT, int PHASE, bool DET>
 __global__ void __launch_bounds__(kF8Threads, 1)
     ffn_f8_kernel(const __grid_constant__ CUtensorMap tmA0,
                   const __grid_constant__ CUtensorMap tmA1,
@@ -145,14 +145,14 @@ __global__ void __launch_bounds__(kF8Threads, 1)
                                  (long long)blockIdx.x * snum, den);
   int s_end = cost_split_stage(pl, rtiles, KB, NT, cost_a, kTokenCost,
                                (long long)(blockIdx.x + 1) * snum, den);
-  if (p.det) {
+  if (DET) {
     s_begin = (int)item_boundary(s_begin, KB);
     s_end = (int)item_boundary(s_end, KB);
   }
   int s_dyn = tail ? cost_split_stage(pl, rtiles, KB, NT, cost_a, kTokenCost, snum, sden)
                    : total;
-  if (p.det) s_dyn = (int)item_boundary(s_dyn, KB);  // the last CTA's share ends here too
-  const int us = p.det ? KB : kUnitStages;  // stages per unit of the tail
+  if (DET) s_dyn = (int)item_boundary(s_dyn, KB);  // the last CTA's share ends here too
+  const int us = DET ? KB : kUnitStages;  // stages per unit of the tail
   uint32_t* units = p.units + 2 * (PHASE - 1);
   const uint32_t timeout_bit = (PHASE == 1) ? kStatusTimeoutGateUp : kStatusTimeoutDown;
   // B rows: per token (phase 1, tokens scattered) or one box per chunk
@@ -418,8 +418,8 @@ __global__ void __launch_bounds__(kF8Threads, 1)
               const float sc = __ldg(p.xinv + a / p.k);
               const int f = inf.rt * kRowsHalf + row;
               float* gr = p.gu + (size_t)arow * 2 * p.I + f;
-              put_f32(gr, acc0[j] * sc, p.det);
-              put_f32(gr + p.I, acc1[j] * sc, p.det);
+              put_f32(gr, acc0[j] * sc, DET);
+              put_f32(gr + p.I, acc1[j] * sc, DET);
             } else {
               const float sc = __ldcg(p.xinv + arow);  // hinv, written by the previous kernel
               const int hrow = inf.rt * 2 * kRowsHalf + row;
@@ -429,9 +429,9 @@ __global__ void __launch_bounds__(kF8Threads, 1)
                 red_add_f32(orow, gw * acc0[j]);
                 red_add_f32(orow + kRowsHalf, gw * acc1[j]);
               } else {
-                float* yrow = p.y_perm + (size_t)(p.det ? a : arow) * p.H + hrow;
-                put_f32(yrow, acc0[j] * sc, p.det);
-                put_f32(yrow + kRowsHalf, acc1[j] * sc, p.det);
+                float* yrow = p.y_perm + (size_t)(DET ? a : arow) * p.H + hrow;
+                put_f32(yrow, acc0[j] * sc, DET);
+                put_f32(yrow + kRowsHalf, acc1[j] * sc, DET);
               }
             }
           }
