@@ -13,7 +13,7 @@ static cudaError_t launch_ffn_f8_ph(int grid, const FfnMaps& m, const FfnParams&
   static std::atomic<unsigned long long> done[2] = {{0}, {0}};  // per variant
   cudaError_t err = set_smem_once(kern, smem, done[p.det ? 1 : 0]);
   if (err != cudaSuccess) return err;
-  return launch_k(kern, dim3(grid), dim3(kF8Threads), smem, st, expert_pdl(p, false), m.a0,
+  return launch_k(kern, dim3(grid), dim3(kF8Threads), smem, st, expert_pdl(p), m.a0,
                   m.a1, m.b, p);
 }
 

@@ -35,16 +35,14 @@ cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t sme
 // Whether an expert kernel of the tensor-core engines starts as a programmatic
 // dependent of the kernel before it.  The persistent grid divides its stages
 // by CTA index and assumes every CTA starts at once; launched early behind a
-// short kernel of many CTAs (the gather before gate/up, the SwiGLU rows kernel
-// before NVFP4 down), its CTAs start as those SMs free up, and the last ones
-// finish late.  Measured in a graph of layer calls, early launch off: FP8
-// 480B-shaped T=512 gate/up 1600 -> 1572 us a layer; NVFP4 235B-shaped T=128
-// gate/up 278.7 -> 273.8, down 278.7 -> 274.2; prefill-shaped T=2048 gate/up
-// 750 -> 742.  Up to 64 tokens (no gather, the quad SwiGLU) the early start
-// pays: NVFP4 T=64 243 us with it, 254 without.
-inline bool expert_pdl(const FfnParams& p, bool nvfp4) {
-  if (p.phase == 1) return !p.b_compact;
-  return !nvfp4 || p.T * p.k <= 512;
+// large gather (at least 2048 assignment rows), its CTAs start as the
+// gather's SMs free up and the last ones finish late.  Measured in graphs of
+// layer calls, gate/up without / with the early start: FP8 480B-shaped T=512
+// 1511 / 1539 us a layer, FP8 Zipf T=256 1280 / 1286; below 2048 rows the
+// early start pays (FP8 Zipf T=128 819 / 809 us; the NVFP4 94-layer stack at
+// T=128 26.40 / 26.14 ms, of which 0.19 ms came from the down kernel).
+inline bool expert_pdl(const FfnParams& p) {
+  return !(p.phase == 1 && p.b_compact && (long long)p.T * p.k >= 2048);
 }
 
 struct FfnMaps {

@@ -12,7 +12,7 @@ static cudaError_t launch_ffn_pf_ph(int grid, const FfnMaps& m, const FfnParams&
   static std::atomic<unsigned long long> done{0};
   cudaError_t err = set_smem_once(kern, smem, done);
   if (err != cudaSuccess) return err;
-  return launch_k(kern, dim3(grid), dim3(kPfThreads), smem, st, expert_pdl(p, true), m.a0, m.a1,
+  return launch_k(kern, dim3(grid), dim3(kPfThreads), smem, st, expert_pdl(p), m.a0, m.a1,
                   m.s0, m.s1, m.b, m.sb, p);
 }
 
