@@ -812,6 +812,8 @@ int moe_decode_layer_ex(const void* x, const float* router_w, const float* route
     g.qrow = fp4 ? H / 2 : H;
     g.sfrow = H / 16;
     g.inv = pf ? ws_ptr<int>(ws, L.inv) : nullptr;
+    g.status = ws_ptr<uint32_t>(ws, L.status);
+    g.wait_ns = wait_limit_ns();
     if (launch_gather(g, st) != cudaSuccess) return MOE_ERR_CUDA;
   }
   if (ev[1] && cudaEventRecord(ev[1], st) != cudaSuccess) return MOE_ERR_CUDA;

@@ -559,13 +559,40 @@ __global__ void __launch_bounds__(256) prep_kernel(const PrepParams p) {
 
 // grid ceil(T*k / 8): CTA b copies compact rows 8b..8b+7.  Compact row r is
 // position r - pre[e] of expert e's list, pre the exclusive prefix of the
-// per-expert counts (every CTA scans the counts; E <= 512).
-__global__ void __launch_bounds__(256) gather_kernel(const GatherParams p) {
+// per-expert counts (every CTA scans the counts; E <= 512).  A row's term rows
+// (and their scales) are one contiguous block in both arrays, so one thread
+// moves them with bulk copies: every block into shared memory under one
+// mbarrier, then every block out.
+constexpr int kGatherRows = 8;
+
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes,
+                                         uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::
+          "r"(dst),
+      "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_u32(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void bulk_s2g(void* dst, uint32_t src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(
+                   reinterpret_cast<uint64_t>(dst)),
+               "r"(src), "r"(bytes)
+               : "memory");
+}
+
+__global__ void __launch_bounds__(128) gather_kernel(const GatherParams p) {
+  extern __shared__ __align__(128) unsigned char g_rows[];
   __shared__ int s_pre[kMaxE + 1];
-  __shared__ int s_tok[8], s_row[8];
+  __shared__ int s_tok[kGatherRows], s_row[kGatherRows];
+  __shared__ __align__(8) uint64_t s_bar;
   pdl_wait();  // the routing that wrote the lists is complete
   pdl_launch_dependents();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 32) {
+    mbar_init(&s_bar, 1);
+    fence_mbar_init();
+  }
   if (warp == 0) {
     constexpr int PER = kMaxE / 32;  // counts per lane
     int c[PER], run = 0;
@@ -591,8 +618,8 @@ __global__ void __launch_bounds__(256) gather_kernel(const GatherParams p) {
   }
   __syncthreads();
   const int total = s_pre[kMaxE];
-  const int r0 = blockIdx.x * 8;
-  const int nj = min(8, total - r0);
+  const int r0 = blockIdx.x * kGatherRows;
+  const int nj = min(kGatherRows, total - r0);
   if (nj <= 0) return;
   if (threadIdx.x < nj) {
     const int r = r0 + threadIdx.x;
@@ -609,33 +636,26 @@ __global__ void __launch_bounds__(256) gather_kernel(const GatherParams p) {
     if (p.inv) p.inv[a] = r;
   }
   __syncthreads();
-  // 16-byte units, eight loads in flight per thread before their stores
-  auto copy = [&](const uint8_t* src, uint8_t* dst, int row_bytes) {
-    const int u16 = row_bytes / 16;  // units of one token's term rows
-    const int n = nj * u16;
-    constexpr int B = 8;
-    for (int base = 0; base < n; base += B * 256) {
-      uint4 v[B];
-#pragma unroll
-      for (int q = 0; q < B; ++q) {
-        const int i = base + q * 256 + threadIdx.x;
-        if (i < n) {
-          const int j = i / u16, u = i - j * u16;
-          v[q] = __ldcg(reinterpret_cast<const uint4*>(src + (size_t)s_tok[j] * row_bytes) + u);
-        }
-      }
-#pragma unroll
-      for (int q = 0; q < B; ++q) {
-        const int i = base + q * 256 + threadIdx.x;
-        if (i < n) {
-          const int j = i / u16, u = i - j * u16;
-          reinterpret_cast<uint4*>(dst + (size_t)s_row[j] * row_bytes)[u] = v[q];
-        }
-      }
-    }
-  };
-  copy(p.q, p.gq, p.terms * p.qrow);
-  if (p.sf) copy(p.sf, p.gsf, p.terms * p.sfrow);
+  if (threadIdx.x != 0) return;
+  const uint32_t rb = (uint32_t)(p.terms * p.qrow);              // term rows of a token
+  const uint32_t sb = p.sf ? (uint32_t)(p.terms * p.sfrow) : 0u;  // their scales
+  const uint32_t base = smem_u32(g_rows);
+  mbar_arrive_expect_tx(&s_bar, (uint32_t)nj * (rb + sb));
+  for (int j = 0; j < nj; ++j) {
+    bulk_g2s(base + j * rb, p.q + (size_t)s_tok[j] * rb, rb, &s_bar);
+    if (sb) bulk_g2s(base + kGatherRows * rb + j * sb, p.sf + (size_t)s_tok[j] * sb, sb, &s_bar);
+  }
+  if (!mbar_wait_bounded(&s_bar, 0, p.wait_ns, nullptr)) {
+    set_status(p.status, kStatusTimeoutRoute);
+    return;  // copies that never landed leave nothing to store
+  }
+  for (int j = 0; j < nj; ++j) {
+    bulk_s2g(p.gq + (size_t)s_row[j] * rb, base + j * rb, rb);
+    if (sb) bulk_s2g(p.gsf + (size_t)s_row[j] * sb, base + kGatherRows * rb + j * sb, sb);
+  }
+  asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+  // the shared memory is read out before the CTA exits
+  asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
 }
 
 __global__ void __launch_bounds__(256) combine_kernel(const CombineParams p) {
@@ -711,9 +731,16 @@ cudaError_t launch_route(const RouteParams& p, cudaStream_t st) {
 }
 
 cudaError_t launch_gather(const GatherParams& p, cudaStream_t st) {
+  // shared memory for the rows of the largest shape (H = 8192)
+  static std::atomic<unsigned long long> done{0};
+  const int smax = kGatherRows * (4 * 4096 + 4 * 512);
+  cudaError_t err = set_smem_once(gather_kernel, smax, done);
+  if (err != cudaSuccess) return err;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)(((size_t)p.T * p.k + 7) / 8));
-  cfg.blockDim = dim3(256);
+  cfg.gridDim = dim3((unsigned)(((size_t)p.T * p.k + kGatherRows - 1) / kGatherRows));
+  cfg.blockDim = dim3(128);
+  cfg.dynamicSmemBytes =
+      (size_t)kGatherRows * (p.terms * p.qrow + (p.sf ? p.terms * p.sfrow : 0));
   cfg.stream = st;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;

@@ -120,6 +120,8 @@ struct GatherParams {
   const int* alist;   // [E, T]
   int* inv;           // [T*k] compact row of each assignment, or null
   int T, k, E, terms, qrow, sfrow;
+  uint32_t* status;   // device status word (an expired copy wait)
+  uint64_t wait_ns;
 };
 
 struct CombineParams {
