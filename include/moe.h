@@ -32,7 +32,10 @@
  *   with moe_read_status().  No exception or abort crosses the ABI.
  *
  * Arithmetic of the GPU path: fp32 router and gates; expert products
- * accumulate in fp32.  Both formats feed their weights to the tensor cores
+ * accumulate in fp32.  Large batches compute the router logits on the tensor
+ * cores from the fp32 router split exactly into three bf16 parts (every
+ * product exact in fp32, fp32 accumulation: the fp32 GEMV up to the order of
+ * its additions).  Both formats feed their weights to the tensor cores
  * as stored, and the activations (x, and h between the gate/up and down
  * steps) are encoded in the weights' format family:
  * - NVFP4: block-scaled MMA (E2M1 x UE4M3 per 16 K); each activation row is
@@ -53,6 +56,13 @@
  *                         and 32 for FP8); 32 is not taken for NVFP4
  *   MOE_WAIT_LIMIT_MS=n   limit in ms of every bounded device wait, 1-60000
  *                         (default 1000; read once per process)
+ *   MOE_PF=0              prefill-shaped NVFP4 batches (T > 64, T*k >= 32*E)
+ *                         stay on the decode engine instead of the prefill
+ *                         engine (read once per process)
+ *   MOE_ROUTE_TC=0|1      router logits on the CUDA cores for every batch (0),
+ *                         or on the tensor cores for every batch with E <= 256
+ *                         (1), instead of the tensor cores from T*H >= 2^21
+ *                         (read once per process)
  *
  * Expert weight formats (moe_expert_weights_t)
  *   gate and up are [E, I, H]-shaped (N = I rows, K = H contiguous),
