@@ -166,6 +166,29 @@ int moe_route_workspace_size(int T, int E, size_t* bytes);
 int moe_cost_split_stage(const int32_t* counts, int E, int NT, int rtiles, int KB, int a, int b,
                          long long num, long long den, int* stage);
 
+/* The order in which the FP8 tensor-core kernel walks its stages: stages
+ * s_begin .. s_begin + n - 1 of the sequence, as the kernel's own cursor
+ * gives them, run on the host on the plan built from the counts.  Pure host
+ * computation; a diagnostic for tests, not a step of the decode layer.
+ *   Each (active expert, row tile) group holds the same stages as in
+ *   moe_cost_split_stage's order and keeps its place in the sequence.  Inside
+ *   a group whose expert has several chunks of NT tokens, the K-blocks are cut
+ *   into slabs of `slab` K-blocks (the last one shorter when slab does not
+ *   divide KB), and every chunk runs over one slab, K-blocks in order, before
+ *   any chunk runs over the next.  A group of one chunk, or slab = 0 or
+ *   slab >= KB, keeps the item order: chunk, then K-block.
+ *   item[i] (host, int32): the item (active expert, row tile, chunk), numbered
+ *     as in moe_cost_split_stage's order (chunk fastest); kb[i] its K-block;
+ *     run_end[i] = 1 on the last stage of a chunk's run within its slab,
+ *     where the kernel adds that chunk's partial sums out, else 0.
+ *   MOE_ERR_INVALID_ARG: null pointer (the outputs may be null when n = 0),
+ *     negative count, NT outside [1, 256], rtiles or KB below 1, slab, s_begin
+ *     or n negative, or s_begin + n past the last stage.
+ *   MOE_ERR_UNSUPPORTED_SHAPE: E outside [1, 512], more than 2^24 tokens or
+ *     2^31 stages or more. */
+int moe_stage_order(const int32_t* counts, int E, int NT, int rtiles, int KB, int slab,
+                    int s_begin, int n, int32_t* item, int32_t* kb, int32_t* run_end);
+
 /* Zero a workspace (cudaMemsetAsync).  A workspace must be zeroed once
  * before its first use; the library keeps it consistent afterwards (its
  * counters are reset by their last user).  After moe_read_status() reports

@@ -62,6 +62,7 @@ _SIGS = {
     "moe_layer_kernel_count": [ctypes.POINTER(ExpertWeightsC), _I, _I, ctypes.POINTER(_I)],
     "moe_cost_split_stage": [_P, _I, _I, _I, _I, _I, _I, ctypes.c_longlong, ctypes.c_longlong,
                              ctypes.POINTER(_I)],
+    "moe_stage_order": [_P, _I, _I, _I, _I, _I, _I, _I, _P, _P, _P],
     "moe_workspace_init": [_P, _SZ, _P],
     "moe_read_status": [_P, _SZ, ctypes.POINTER(_I), _P],
     "moe_route_topk": [_P, _P, _P, _I, _I, _I, _I, _I, _P, _P, _P, _P, _SZ, _P],
@@ -173,6 +174,16 @@ def moe_cost_split_stage(counts, NT: int, rtiles: int, KB: int, a: int, b: int, 
     _check(load().moe_cost_split_stage(arr, len(counts), NT, rtiles, KB, a, b, num, den,
                                        ctypes.byref(out)), "moe_cost_split_stage")
     return out.value
+
+
+def moe_stage_order(counts, NT: int, rtiles: int, KB: int, slab: int, s_begin: int, n: int):
+    """Stages s_begin .. s_begin + n - 1 in the FP8 tensor-core kernel's order, run on the
+    host: (item, K-block, run_end) lists."""
+    arr = (ctypes.c_int32 * len(counts))(*[int(c) for c in counts])
+    item, kb, end = ((ctypes.c_int32 * max(n, 1))() for _ in range(3))
+    _check(load().moe_stage_order(arr, len(counts), NT, rtiles, KB, slab, s_begin, n, item, kb,
+                                  end), "moe_stage_order")
+    return list(item[:n]), list(kb[:n]), list(end[:n])
 
 
 def alloc_workspace(nbytes: int, device=None) -> torch.Tensor:

@@ -23,6 +23,7 @@ constexpr int kFlagTestStall = 0x100;  // test hook, see the comment in moe.h
 struct DevInfo {
   std::atomic<int> ready{0};
   int sms = 0, ok = 0;
+  long long l2 = 0;  // L2 bytes
 };
 DevInfo g_dev[64];
 
@@ -31,18 +32,27 @@ int device_check(int* sms) {
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return MOE_ERR_CUDA;
   DevInfo& d = g_dev[dev];
   if (!d.ready.load(std::memory_order_acquire)) {
-    int major = 0, minor = 0, n = 0;
+    int major = 0, minor = 0, n = 0, l2 = 0;
     if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
         cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&l2, cudaDevAttrL2CacheSize, dev) != cudaSuccess)
       return MOE_ERR_CUDA;
     d.sms = n;
+    d.l2 = l2;
     d.ok = (major == 10 && minor == 3);
     d.ready.store(1, std::memory_order_release);
   }
   if (!d.ok) return MOE_ERR_UNSUPPORTED_DEVICE;
   *sms = d.sms;
   return MOE_OK;
+}
+
+// L2 size of the current device (after device_check).
+long long device_l2_bytes() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  return g_dev[dev].l2;
 }
 
 uint64_t wait_limit_ns() {
@@ -155,6 +165,27 @@ int nt_for(int T, int eng) {
   if (eng == kEngBs) return T <= 64 ? 8 : 16;
   if (eng == kEngF8) return T <= 64 ? 8 : 32;
   return T <= 64 ? 8 : 32;
+}
+
+// Slab order of the FP8 engine (SlabCursor, ffn.cuh) in a step whose whole
+// items would not keep their weight tiles in L2: the grid's current tiles
+// (KB stages of two 16 KB weight boxes per CTA) larger than the L2.  Measured
+// on the 480B-shaped layer with Zipf routing at T = 256: the gate/up step
+// (KB = 48, 239 MB of tiles on 152 CTAs) 839 -> 696 us with slabs of 16;
+// the down step (KB = 20, 100 MB) was slower with every slab length tried
+// (398 -> 517 us at 16, 612 at 8): its tiles stayed in L2 with whole items,
+// and every slab end adds the chunks' partial sums out.  MOE_F8_SLAB=n sets
+// the slab length (0: whole items always; for comparisons).
+constexpr int kF8Slab = 16;
+int f8_slab(int KB, int grid) {
+  static int v = -1;
+  if (v < 0) {
+    const char* s = std::getenv("MOE_F8_SLAB");
+    v = s ? std::atoi(s) : kF8Slab;
+    if (v < 0) v = 0;
+  }
+  const long long tiles = (long long)grid * KB * 2 * kRowsHalf * kRowBytes;
+  return tiles > device_l2_bytes() ? v : 0;
 }
 
 // Experts per router CTA: small batches spread the router rows over more
@@ -343,6 +374,7 @@ int run_experts(const ExpertRun& r, cudaStream_t st, cudaEvent_t ev_mid) {
   p1.hq = ws_ptr<uint8_t>(r.ws, r.L.hq);
   p1.hsf = ws_ptr<uint8_t>(r.ws, r.L.hsf);
   p1.test_stall = r.test_stall;
+  p1.slab = f8_slab(H / 128, r.sms);
 
   FfnParams p2 = p;
   p2.phase = 2;
@@ -358,6 +390,7 @@ int run_experts(const ExpertRun& r, cudaStream_t st, cudaEvent_t ev_mid) {
   p2.residual = r.residual;
   p2.bsf = ws_ptr<uint8_t>(r.ws, r.L.hsf);
   p2.acnt_reset = r.list_T ? ws_ptr<uint32_t>(r.ws, r.L.acnt) : nullptr;
+  p2.slab = f8_slab(I / 128, r.sms);
 
   auto launch = [&](const FfnMaps& m, const FfnParams& pp) {
     if (eng == kEngBs) return launch_ffn_bs(r.nt, r.sms, m, pp, st);
@@ -500,13 +533,8 @@ int moe_route_workspace_size(int T, int E, size_t* bytes) {
   return MOE_OK;
 }
 
-int moe_cost_split_stage(const int32_t* counts, int E, int NT, int rtiles, int KB, int a, int b,
-                         long long num, long long den, int* stage) {
-  if (!counts || !stage || NT < 1 || NT > 256 || rtiles < 1 || KB < 1) return MOE_ERR_INVALID_ARG;
-  if (a < 1 || b < 0 || den < 1 || num < 0 || num > den) return MOE_ERR_INVALID_ARG;
-  if (E < 1 || E > kMaxE) return MOE_ERR_UNSUPPORTED_SHAPE;
-  // the plan the kernels build in shared memory, built here by a plain scan
-  PlanSmem pl;
+// The plan the kernels build in shared memory, built here by a plain scan.
+static int host_plan(const int32_t* counts, int E, int NT, PlanSmem& pl, long long* assignments) {
   long long off = 0, ch = 0;
   int n = 0;
   for (int e = 0; e < E; ++e) {
@@ -525,6 +553,20 @@ int moe_cost_split_stage(const int32_t* counts, int E, int NT, int rtiles, int K
   pl.nA = n;
   pl.aoff[n] = (int)off;
   pl.cpre[n] = (int)ch;
+  *assignments = off;
+  return MOE_OK;
+}
+
+int moe_cost_split_stage(const int32_t* counts, int E, int NT, int rtiles, int KB, int a, int b,
+                         long long num, long long den, int* stage) {
+  if (!counts || !stage || NT < 1 || NT > 256 || rtiles < 1 || KB < 1) return MOE_ERR_INVALID_ARG;
+  if (a < 1 || b < 0 || den < 1 || num < 0 || num > den) return MOE_ERR_INVALID_ARG;
+  if (E < 1 || E > kMaxE) return MOE_ERR_UNSUPPORTED_SHAPE;
+  PlanSmem pl;
+  long long off = 0;
+  const int rc = host_plan(counts, E, NT, pl, &off);
+  if (rc) return rc;
+  const long long ch = pl.cpre[pl.nA];
   // stage indices are int; the scaled cost prefix C * num is long long
   const long long stages = ch * rtiles * KB;
   if (stages >= (1ll << 31)) return MOE_ERR_UNSUPPORTED_SHAPE;
@@ -532,6 +574,29 @@ int moe_cost_split_stage(const int32_t* counts, int E, int NT, int rtiles, int K
   const long long C = (long long)rtiles * KB * ((long long)a * ch + (long long)b * off);
   if (C > 0 && num > (1ll << 62) / C) return MOE_ERR_UNSUPPORTED_SHAPE;
   *stage = cost_split_stage(pl, rtiles, KB, NT, a, b, num, den);
+  return MOE_OK;
+}
+
+int moe_stage_order(const int32_t* counts, int E, int NT, int rtiles, int KB, int slab,
+                    int s_begin, int n, int32_t* item, int32_t* kb, int32_t* run_end) {
+  if (!counts || NT < 1 || NT > 256 || rtiles < 1 || KB < 1 || slab < 0 || s_begin < 0 || n < 0)
+    return MOE_ERR_INVALID_ARG;
+  if (n > 0 && (!item || !kb || !run_end)) return MOE_ERR_INVALID_ARG;
+  if (E < 1 || E > kMaxE) return MOE_ERR_UNSUPPORTED_SHAPE;
+  PlanSmem pl;
+  long long off = 0;
+  const int rc = host_plan(counts, E, NT, pl, &off);
+  if (rc) return rc;
+  const long long stages = (long long)pl.cpre[pl.nA] * rtiles * KB;
+  if (stages >= (1ll << 31)) return MOE_ERR_UNSUPPORTED_SHAPE;
+  if ((long long)s_begin + n > stages) return MOE_ERR_INVALID_ARG;
+  if (n == 0) return MOE_OK;
+  SlabCursor<1> c(pl, rtiles, KB, slab, s_begin);
+  for (int i = 0; i < n; ++i, c.next()) {
+    item[i] = c.it;
+    kb[i] = c.kb;
+    run_end[i] = c.run_end ? 1 : 0;
+  }
   return MOE_OK;
 }
 

@@ -116,6 +116,9 @@ struct FfnParams {
   // on it in the epilogue's unrolled loops made the default NVFP4 down
   // kernel 13% slower (16-token chunks, 82 -> 93 us a launch).
   int det;
+  // FP8 tensor-core engine: K-blocks per slab of an expert with several token
+  // chunks (SlabCursor); 0 or >= K/128 keeps each chunk's item whole
+  int slab;
   // routing: tokens per expert, and each expert's assignments (t*k + j).
   // list_T = 1: expert e's list starts at sorted[e*T] (the fused layer's
   // per-expert lists); 0: at sorted[offsets[e]] (one array sorted by expert).
@@ -301,6 +304,97 @@ struct StageCursor {
   __device__ __forceinline__ void seek(int s) {
     it = s / KB;
     kb = s - it * KB;
+  }
+};
+
+// The same sequence of stages in slab order (FP8 tensor-core engine).  The
+// stages of one (expert, row tile) group keep their place in the sequence,
+// but inside a group of several token chunks the K range is cut into slabs
+// of SL K-blocks, and every chunk runs over slab j before any runs over slab
+// j + 1: a weight box is read from HBM by the first chunk and from L2 by the
+// others while the CTA holds at most SL stages' boxes for them, where whole
+// items (SL = KB) left them to be read again from HBM once the boxes of all
+// CTAs' current tiles outgrew L2.  A group of one chunk is one slab of KB
+// stages, the item order of decode_item.  `it` is the item (expert, row
+// tile, chunk) for decode_item, `run_end` marks the last stage of a chunk's
+// run in its slab: its partial sums are added out there.
+template <int S>
+struct SlabCursor {
+  const PlanSmem* pl;
+  int rtiles, KB, SL;
+  int lo, rt, nch, it0;    // group: expert slot, row tile, chunks, first item
+  int chunk, ks0, sl, kbs;  // chunk, first K-block and length of the slab, offset
+  int it, kb, slot;
+  bool run_end;
+  uint32_t par;
+  __host__ __device__ __forceinline__ SlabCursor(const PlanSmem& plan, int rtiles_, int kb_per_item,
+                                        int slab, int s_begin)
+      : pl(&plan), rtiles(rtiles_), KB(kb_per_item),
+        SL(slab > 0 && slab < kb_per_item ? slab : kb_per_item), slot(0), par(0u) {
+    seek(s_begin);
+  }
+  __host__ __device__ __forceinline__ int group_slab() const { return nch > 1 ? SL : KB; }
+  __host__ __device__ __forceinline__ void settle() {
+    kb = ks0 + kbs;
+    it = it0 + chunk;
+    run_end = (kbs + 1 == sl);
+  }
+  // jump to stage s of the sequence; the ring position runs on
+  __host__ __device__ __forceinline__ void seek(int s) {
+    int a = 0, b = pl->nA - 1;  // last slot whose first stage is <= s
+    while (a < b) {
+      const int mid = (a + b + 1) >> 1;
+      if (pl->cpre[mid] * rtiles * KB <= s) a = mid; else b = mid - 1;
+    }
+    lo = a;
+    nch = pl->nA > 0 ? pl->cpre[lo + 1] - pl->cpre[lo] : 1;
+    if (nch < 1) nch = 1;
+    const int base = pl->nA > 0 ? pl->cpre[lo] : 0;
+    const int local = s - base * rtiles * KB;
+    rt = local / (nch * KB);
+    const int o = local - rt * nch * KB;
+    it0 = base * rtiles + rt * nch;
+    const int g = group_slab();
+    const int nfs = KB / g;
+    if (o < nfs * nch * g) {
+      const int j = o / (nch * g);
+      const int o1 = o - j * nch * g;
+      chunk = o1 / g;
+      kbs = o1 - chunk * g;
+      ks0 = j * g;
+      sl = g;
+    } else {
+      sl = KB - nfs * g;
+      const int o2 = o - nfs * nch * g;
+      chunk = o2 / sl;
+      kbs = o2 - chunk * sl;
+      ks0 = nfs * g;
+    }
+    settle();
+  }
+  __host__ __device__ __forceinline__ void next() {
+    if (++kbs == sl) {
+      kbs = 0;
+      if (++chunk == nch) {
+        chunk = 0;
+        ks0 += sl;
+        if (ks0 == KB) {
+          ks0 = 0;
+          it0 += nch;
+          if (++rt == rtiles) {
+            rt = 0;
+            if (++lo < pl->nA) nch = pl->cpre[lo + 1] - pl->cpre[lo];
+          }
+        }
+        const int g = group_slab();
+        sl = g < KB - ks0 ? g : KB - ks0;
+      }
+    }
+    settle();
+    if (++slot == S) {
+      slot = 0;
+      par ^= 1u;
+    }
   }
 };
 

@@ -2,13 +2,14 @@
 // as stored times E4M3 activation terms, fp32 accumulation in tensor memory.
 //
 // Work decomposition as in ffn.cuh / ffn_bs.cuh: a persistent grid, stream-K
-// over the K-stages of all (active expert, <=NT-token chunk, row tile) items.
+// over the K-stages of all (active expert, <=NT-token chunk, row tile) items,
+// the stages of an expert with several chunks in slab order (SlabCursor).
 // A stage is 128 K, which is exactly one column of the weights' 128x128 fp32
 // block scales.  The MMA has no block scaling for this format pair, so every
 // stage accumulates into its own slot of a ring of tensor-memory accumulators
 // and the epilogue warps multiply it by the stage's two block scales while
 // adding it into registers; an item's sums are flushed with red.add at its
-// last stage (in this CTA).  The activations arrive as two E4M3 terms per
+// last stage in this CTA, or at the end of its run in a slab.  The activations arrive as two E4M3 terms per
 // token (act_terms.cuh): B rows 2j, 2j+1 of token j; the epilogue adds the
 // two columns.
 //
@@ -153,6 +154,9 @@ __global__ void __launch_bounds__(kF8Threads, 1)
                    : total;
   if (DET) s_dyn = (int)item_boundary(s_dyn, KB);  // the last CTA's share ends here too
   const int us = DET ? KB : kUnitStages;  // stages per unit of the tail
+  // slab order for experts of several chunks; whole items in the
+  // deterministic mode (every item summed by one CTA in K order)
+  const int slab = DET ? 0 : p.slab;
   uint32_t* units = p.units + 2 * (PHASE - 1);
   const uint32_t timeout_bit = (PHASE == 1) ? kStatusTimeoutGateUp : kStatusTimeoutDown;
   // B rows: per token (phase 1, tokens scattered) or one box per chunk
@@ -167,9 +171,9 @@ __global__ void __launch_bounds__(kF8Threads, 1)
       tma_prefetch_desc(&tmA0);
       tma_prefetch_desc(&tmA1);
       if (!lead) tma_prefetch_desc(&tmB);
-      // weights stream through L2 once (evict first), except the tile of an
-      // item whose expert has tokens in a later chunk: that chunk's item,
-      // next in the order, reads the same tile again (evict last)
+      // weights stream through L2 once (evict first), except the boxes of an
+      // item whose expert has tokens in a later chunk: that chunk reads the
+      // same boxes again (evict last), within the slab in slab order
       const uint64_t pol_w = policy_evict_first();
       const uint64_t pol_keep = policy_evict_last();
       uint64_t pol_item = pol_w;
@@ -178,7 +182,7 @@ __global__ void __launch_bounds__(kF8Threads, 1)
       ItemInfo inf{};
       int issued = 0, uj = 0;
       bool ok = true;
-      StageCursor<S> c(s_begin, KB);
+      SlabCursor<S> c(pl, rtiles, KB, slab, s_begin);
       // segments: this CTA's own share, then units of the shared tail (the
       // lead takes them and publishes them; the second producer reads them)
       for (int a = s_begin, b = s_end; ok;) {
@@ -347,7 +351,7 @@ __global__ void __launch_bounds__(kF8Threads, 1)
     // c: this stage (it, kb) and its accumulator ring slot; the stage after
     // it is found first (its block scales load while this stage's
     // accumulator is awaited), reading the shared-tail units as they come
-    StageCursor<DR> c(s_begin, KB);
+    SlabCursor<DR> c(pl, rtiles, KB, slab, s_begin);
     int cs = s_begin, cend = s_end, uj = 0;
     bool ok = true;
     bool have = cs < cend;
@@ -363,7 +367,7 @@ __global__ void __launch_bounds__(kF8Threads, 1)
       // the next stage: the following one in this segment, or the first of
       // the next unit (a new accumulation even within the same item)
       int ns = cs + 1, nend = cend;
-      StageCursor<DR> nc = c;  // its accumulator slot is the next one in any case
+      SlabCursor<DR> nc = c;  // its accumulator slot is the next one in any case
       nc.next();
       bool have_next = ns < nend, jump = false;
       if (!have_next && tail) {
@@ -373,7 +377,7 @@ __global__ void __launch_bounds__(kF8Threads, 1)
       }
       float nb0 = 0.f, nb1 = 0.f;
       ItemInfo ninf = inf;
-      const bool closes = !have_next || jump || (c.kb + 1 == KB);
+      const bool closes = !have_next || jump || c.run_end;
       if (have_next) {
         if (nc.it != c.it) ninf = decode_item(nc.it, rtiles, pl, p, NT);
         scales(ninf, nc.kb, nb0, nb1);
