@@ -13,11 +13,14 @@
 // token (act_terms.cuh): B rows 2j, 2j+1 of token j; the epilogue adds the
 // two columns.
 //
-// Roles (224 threads):
+// Roles (224 threads; 352 in the down step with 32-token chunks):
 //   warps 0-3  epilogue: warp w reads TMEM lanes 32w..32w+31 (rows of the tile)
 //   warps 4,6  TMA producers (one thread each): warp 4 arms each stage's
 //              barrier and copies box A0, warp 6 box A1 and the activation rows
 //   warp 5     MMA issuer (one thread); allocates and frees tensor memory
+//   warps 7-10 (down step, 32-token chunks) a second epilogue group: warp w
+//              reads lanes 32(w%4).. like warp w%4, for the chunk's tokens
+//              16-31, warps 0-3 then taking tokens 0-15
 // Every wait is bounded (p.wait_ns); an expired wait sets the status word and
 // the kernel winds down, freeing its tensor memory.
 #pragma once
@@ -27,11 +30,20 @@
 
 namespace moe {
 
-constexpr int kF8Threads = 7 * 32;
-constexpr int kF8EpiWarp0 = 0, kF8ProducerWarp = 4, kF8MmaWarp = 5, kF8ProducerWarp2 = 6;
+constexpr int kF8ProducerWarp = 4, kF8MmaWarp = 5, kF8ProducerWarp2 = 6;
 
-template <int NT>
+template <int NT, int PHASE>
 struct F8Geom {
+  // epilogue warps: one per TMEM lane quadrant, or two in the down step with
+  // 32-token chunks, each adding half of the chunk's token columns.  Measured
+  // on the 480B-shaped layer with Zipf routing: the down step at T = 256
+  // 400 -> 380 us, at T = 128 267 -> 253 us; the gate/up step was no faster
+  // (696 -> 708 us at T = 256), so it keeps four.  (64-token chunks with
+  // eight warps of 32 tokens each and a 2-deep accumulator ring were slower
+  // in both steps.)
+  static constexpr int EPI = (NT >= 32 && PHASE == 2) ? 8 : 4;
+  static constexpr int NTH = NT * 4 / EPI;  // tokens per epilogue thread
+  static constexpr int THREADS = (EPI + 3) * 32;
   static constexpr int BN = kF8Terms * NT;  // B rows = MMA N
   static constexpr int A0 = 0;
   static constexpr int A1 = kRowsHalf * kRowBytes;      // 16 KB
@@ -62,11 +74,11 @@ __device__ __forceinline__ void tc_mma_f8(uint32_t d_tmem, uint64_t a_desc, uint
 }
 
 template <int NT, int PHASE, bool DET>
-__global__ void __launch_bounds__(kF8Threads, 1)
+__global__ void __launch_bounds__(F8Geom<NT, PHASE>::THREADS, 1)
     ffn_f8_kernel(const __grid_constant__ CUtensorMap tmA0,
                   const __grid_constant__ CUtensorMap tmA1,
                   const __grid_constant__ CUtensorMap tmB, const FfnParams p) {
-  using G = F8Geom<NT>;
+  using G = F8Geom<NT, PHASE>;
   constexpr int BN = G::BN;
   constexpr int S = G::STAGES;
   constexpr int DR = G::DR;
@@ -96,13 +108,13 @@ __global__ void __launch_bounds__(kF8Threads, 1)
     }
     for (int i = 0; i < DR; ++i) {
       mbar_init(&dfull_bar[i], 1);
-      mbar_init(&dempty_bar[i], 4);
+      mbar_init(&dempty_bar[i], G::EPI);
     }
     mbar_init(&final_bar, 1);
-    // readers of each unit: second producer, MMA issuer, 4 epilogue warps
+    // readers of each unit: second producer, MMA issuer, the epilogue warps
     for (int i = 0; i < kUnitRing; ++i) {
       mbar_init(&s_units.full[i], 1);
-      mbar_init(&s_units.empty[i], 6);
+      mbar_init(&s_units.empty[i], 2 + G::EPI);
     }
     fence_mbar_init();
   }
@@ -161,7 +173,7 @@ __global__ void __launch_bounds__(kF8Threads, 1)
   const uint32_t timeout_bit = (PHASE == 1) ? kStatusTimeoutGateUp : kStatusTimeoutDown;
   // B rows: per token (phase 1, tokens scattered) or one box per chunk
   const bool btok = (PHASE == 1) && !p.b_compact;
-  constexpr int kTeardown = 5 * 32;  // epilogue and MMA warps
+  constexpr int kTeardown = (G::EPI + 1) * 32;  // epilogue and MMA warps
 
   // ================================================================ producers
   if (warp == kF8ProducerWarp || warp == kF8ProducerWarp2) {
@@ -323,16 +335,19 @@ __global__ void __launch_bounds__(kF8Threads, 1)
   }
 
   // ================================================================ epilogue
-  // Warp q reads TMEM lanes 32q..32q+31: row 32q+lane of both boxes.
+  // Warp w reads TMEM lanes 32q..32q+31, q = w % 4: row 32q+lane of both
+  // boxes, for the chunk's tokens j0 .. j0 + NTH - 1.
   {
     if (early) pdl_wait();  // the row scales are the SwiGLU output
-    const int quad = warp - kF8EpiWarp0;
+    constexpr int NTH = G::NTH;
+    const int quad = warp & 3;
+    const int j0 = warp > kF8ProducerWarp2 ? NTH : 0;
     const int row = quad * 32 + lane;
     const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
     const int KB128 = K / 128;
-    float acc0[NT], acc1[NT];
+    float acc0[NTH], acc1[NTH];
 #pragma unroll
-    for (int j = 0; j < NT; ++j) acc0[j] = acc1[j] = 0.f;
+    for (int j = 0; j < NTH; ++j) acc0[j] = acc1[j] = 0.f;
     bool dead = false;
     ItemInfo inf{};
     // the block scales of a stage's two boxes
@@ -394,14 +409,15 @@ __global__ void __launch_bounds__(kF8Threads, 1)
       // columns are read with all loads in flight before one wait
 #pragma unroll
       for (int mat = 0; mat < 2; ++mat) {
-        const uint32_t d_t = tmem + lane_addr + (uint32_t)(2 * db + mat) * BN;
+        const uint32_t d_t = tmem + lane_addr + (uint32_t)((2 * db + mat) * BN + 2 * j0);
         const float bsc = mat == 0 ? bs0 : bs1;
-        uint32_t v[BN];
+        uint32_t v[2 * NTH];
 #pragma unroll
-        for (int c0 = 0; c0 < BN; c0 += 16) tmem_ld16(d_t + c0, *reinterpret_cast<uint32_t(*)[16]>(v + c0));
+        for (int c0 = 0; c0 < 2 * NTH; c0 += 16)
+          tmem_ld16(d_t + c0, *reinterpret_cast<uint32_t(*)[16]>(v + c0));
         tmem_ld_wait();
 #pragma unroll
-        for (int j = 0; j < NT; ++j) {
+        for (int j = 0; j < NTH; ++j) {
           const float t2 = __uint_as_float(v[2 * j]) + __uint_as_float(v[2 * j + 1]);
           if (mat == 0)
             acc0[j] = fmaf(bsc, t2, acc0[j]);
@@ -414,7 +430,8 @@ __global__ void __launch_bounds__(kF8Threads, 1)
       if (lane == 0) mbar_arrive(&dempty_bar[db]);
       if (closes) {
 #pragma unroll
-        for (int j = 0; j < NT; ++j) {
+        for (int jj = 0; jj < NTH; ++jj) {
+          const int j = j0 + jj;
           if (j < inf.nvalid) {
             const int arow = inf.arow0 + j;
             const int a = __ldg(p.sorted + inf.lrow0 + j);
@@ -422,24 +439,24 @@ __global__ void __launch_bounds__(kF8Threads, 1)
               const float sc = __ldg(p.xinv + a / p.k);
               const int f = inf.rt * kRowsHalf + row;
               float* gr = p.gu + (size_t)arow * 2 * p.I + f;
-              put_f32(gr, acc0[j] * sc, DET);
-              put_f32(gr + p.I, acc1[j] * sc, DET);
+              put_f32(gr, acc0[jj] * sc, DET);
+              put_f32(gr + p.I, acc1[jj] * sc, DET);
             } else {
               const float sc = __ldcg(p.xinv + arow);  // hinv, written by the previous kernel
               const int hrow = inf.rt * 2 * kRowsHalf + row;
               if (p.fused) {
                 const float gw = __ldg(p.gates + a) * sc;
                 float* orow = p.oacc + (size_t)(a / p.k) * p.H + hrow;
-                red_add_f32(orow, gw * acc0[j]);
-                red_add_f32(orow + kRowsHalf, gw * acc1[j]);
+                red_add_f32(orow, gw * acc0[jj]);
+                red_add_f32(orow + kRowsHalf, gw * acc1[jj]);
               } else {
                 float* yrow = p.y_perm + (size_t)(DET ? a : arow) * p.H + hrow;
-                put_f32(yrow, acc0[j] * sc, DET);
-                put_f32(yrow + kRowsHalf, acc1[j] * sc, DET);
+                put_f32(yrow, acc0[jj] * sc, DET);
+                put_f32(yrow + kRowsHalf, acc1[jj] * sc, DET);
               }
             }
           }
-          acc0[j] = acc1[j] = 0.f;
+          acc0[jj] = acc1[jj] = 0.f;
         }
       }
       inf = ninf;

@@ -9,12 +9,12 @@ template <int NT, int PHASE>
 static cudaError_t launch_ffn_f8_ph(int grid, const FfnMaps& m, const FfnParams& p,
                                     cudaStream_t st) {
   auto kern = p.det ? ffn_f8_kernel<NT, PHASE, true> : ffn_f8_kernel<NT, PHASE, false>;
-  const int smem = F8Geom<NT>::SMEM;
+  const int smem = F8Geom<NT, PHASE>::SMEM;
   static std::atomic<unsigned long long> done[2] = {{0}, {0}};  // per variant
   cudaError_t err = set_smem_once(kern, smem, done[p.det ? 1 : 0]);
   if (err != cudaSuccess) return err;
-  return launch_k(kern, dim3(grid), dim3(kF8Threads), smem, st, expert_pdl(p), m.a0,
-                  m.a1, m.b, p);
+  return launch_k(kern, dim3(grid), dim3(F8Geom<NT, PHASE>::THREADS), smem, st, expert_pdl(p),
+                  m.a0, m.a1, m.b, p);
 }
 
 template <int NT>
