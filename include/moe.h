@@ -64,9 +64,9 @@
  *                         (1), instead of the tensor cores from T*H >= 2^21
  *                         (read once per process)
  *   MOE_F8_SLAB=n         K-blocks per slab of the FP8 engine's experts with
- *                         several token chunks, in a step whose whole items'
- *                         weight tiles exceed the L2 (default 16; 0 keeps
- *                         whole items; read once per process)
+ *                         several 32-token chunks (T > 64), in a step whose
+ *                         whole items' weight tiles exceed the L2 (default 16;
+ *                         0 keeps whole items; read once per process)
  *
  * Expert weight formats (moe_expert_weights_t)
  *   gate and up are [E, I, H]-shaped (N = I rows, K = H contiguous),

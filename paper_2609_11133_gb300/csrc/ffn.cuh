@@ -116,8 +116,9 @@ struct FfnParams {
   // on it in the epilogue's unrolled loops made the default NVFP4 down
   // kernel 13% slower (16-token chunks, 82 -> 93 us a launch).
   int det;
-  // FP8 tensor-core engine: K-blocks per slab of an expert with several token
-  // chunks (SlabCursor); 0 or >= K/128 keeps each chunk's item whole
+  // FP8 tensor-core engine with 32-token chunks: K-blocks per slab of an
+  // expert with several chunks (SlabCursor); 0 or >= K/128 keeps each
+  // chunk's item whole
   int slab;
   // routing: tokens per expert, and each expert's assignments (t*k + j).
   // list_T = 1: expert e's list starts at sorted[e*T] (the fused layer's
@@ -307,6 +308,16 @@ struct StageCursor {
   }
 };
 
+// StageCursor with the constructor and run test of SlabCursor below: the item
+// order for kernels that take either.
+template <int S>
+struct ItemCursor : StageCursor<S> {
+  __device__ __forceinline__ ItemCursor(const PlanSmem&, int, int kb_per_item, int, int s_begin)
+      : StageCursor<S>(s_begin, kb_per_item) {}
+  // last stage of the item: its sums are added out
+  __device__ __forceinline__ bool ends_run() const { return this->kb + 1 == this->KB; }
+};
+
 // The same sequence of stages in slab order (FP8 tensor-core engine).  The
 // stages of one (expert, row tile) group keep their place in the sequence,
 // but inside a group of several token chunks the K range is cut into slabs
@@ -334,6 +345,7 @@ struct SlabCursor {
     seek(s_begin);
   }
   __host__ __device__ __forceinline__ int group_slab() const { return nch > 1 ? SL : KB; }
+  __host__ __device__ __forceinline__ bool ends_run() const { return run_end; }
   __host__ __device__ __forceinline__ void settle() {
     kb = ks0 + kbs;
     it = it0 + chunk;

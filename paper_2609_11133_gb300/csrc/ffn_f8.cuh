@@ -2,8 +2,9 @@
 // as stored times E4M3 activation terms, fp32 accumulation in tensor memory.
 //
 // Work decomposition as in ffn.cuh / ffn_bs.cuh: a persistent grid, stream-K
-// over the K-stages of all (active expert, <=NT-token chunk, row tile) items,
-// the stages of an expert with several chunks in slab order (SlabCursor).
+// over the K-stages of all (active expert, <=NT-token chunk, row tile) items;
+// with 32-token chunks, the stages of an expert with several chunks in slab
+// order (SlabCursor).
 // A stage is 128 K, which is exactly one column of the weights' 128x128 fp32
 // block scales.  The MMA has no block scaling for this format pair, so every
 // stage accumulates into its own slot of a ring of tensor-memory accumulators
@@ -24,6 +25,8 @@
 // Every wait is bounded (p.wait_ns); an expired wait sets the status word and
 // the kernel winds down, freeing its tensor memory.
 #pragma once
+
+#include <type_traits>
 
 #include "act_terms.cuh"
 #include "ffn.cuh"
@@ -166,8 +169,11 @@ __global__ void __launch_bounds__(F8Geom<NT, PHASE>::THREADS, 1)
                    : total;
   if (DET) s_dyn = (int)item_boundary(s_dyn, KB);  // the last CTA's share ends here too
   const int us = DET ? KB : kUnitStages;  // stages per unit of the tail
-  // slab order for experts of several chunks; whole items in the
-  // deterministic mode (every item summed by one CTA in K order)
+  // Slab order for experts of several 32-token chunks; whole items in the
+  // deterministic mode (every item summed by one CTA in K order) and with
+  // narrower chunks: with 8-token chunks slabs gained nothing (Zipf routing
+  // at T = 32: 486.5 -> 484.9 us) and the slab cursor cost the uniform
+  // 480B-shaped layer at T = 64 1.4% of its gate/up time (703 -> 713 us).
   const int slab = DET ? 0 : p.slab;
   uint32_t* units = p.units + 2 * (PHASE - 1);
   const uint32_t timeout_bit = (PHASE == 1) ? kStatusTimeoutGateUp : kStatusTimeoutDown;
@@ -194,7 +200,8 @@ __global__ void __launch_bounds__(F8Geom<NT, PHASE>::THREADS, 1)
       ItemInfo inf{};
       int issued = 0, uj = 0;
       bool ok = true;
-      SlabCursor<S> c(pl, rtiles, KB, slab, s_begin);
+      std::conditional_t<(NT >= 32), SlabCursor<S>, ItemCursor<S>> c(pl, rtiles, KB, slab,
+                                                                      s_begin);
       // segments: this CTA's own share, then units of the shared tail (the
       // lead takes them and publishes them; the second producer reads them)
       for (int a = s_begin, b = s_end; ok;) {
@@ -341,7 +348,7 @@ __global__ void __launch_bounds__(F8Geom<NT, PHASE>::THREADS, 1)
     if (early) pdl_wait();  // the row scales are the SwiGLU output
     constexpr int NTH = G::NTH;
     const int quad = warp & 3;
-    const int j0 = warp > kF8ProducerWarp2 ? NTH : 0;
+    const int j0 = (G::EPI > 4 && warp > kF8ProducerWarp2) ? NTH : 0;
     const int row = quad * 32 + lane;
     const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
     const int KB128 = K / 128;
@@ -366,7 +373,8 @@ __global__ void __launch_bounds__(F8Geom<NT, PHASE>::THREADS, 1)
     // c: this stage (it, kb) and its accumulator ring slot; the stage after
     // it is found first (its block scales load while this stage's
     // accumulator is awaited), reading the shared-tail units as they come
-    SlabCursor<DR> c(pl, rtiles, KB, slab, s_begin);
+    using Cursor = std::conditional_t<(NT >= 32), SlabCursor<DR>, ItemCursor<DR>>;
+    Cursor c(pl, rtiles, KB, slab, s_begin);
     int cs = s_begin, cend = s_end, uj = 0;
     bool ok = true;
     bool have = cs < cend;
@@ -382,7 +390,7 @@ __global__ void __launch_bounds__(F8Geom<NT, PHASE>::THREADS, 1)
       // the next stage: the following one in this segment, or the first of
       // the next unit (a new accumulation even within the same item)
       int ns = cs + 1, nend = cend;
-      SlabCursor<DR> nc = c;  // its accumulator slot is the next one in any case
+      Cursor nc = c;  // its accumulator slot is the next one in any case
       nc.next();
       bool have_next = ns < nend, jump = false;
       if (!have_next && tail) {
@@ -392,7 +400,7 @@ __global__ void __launch_bounds__(F8Geom<NT, PHASE>::THREADS, 1)
       }
       float nb0 = 0.f, nb1 = 0.f;
       ItemInfo ninf = inf;
-      const bool closes = !have_next || jump || c.run_end;
+      const bool closes = !have_next || jump || c.ends_run();
       if (have_next) {
         if (nc.it != c.it) ninf = decode_item(nc.it, rtiles, pl, p, NT);
         scales(ninf, nc.kb, nb0, nb1);
